@@ -1,0 +1,143 @@
+"""Exact output distribution of the verification rules, by enumeration.
+
+TEST INFRASTRUCTURE ONLY (see ``oracle/__init__.py``).
+
+No sampling happens here: every accept test is integrated over its uniform
+analytically (accept probability min(1, R(x)/q(x)), Sec. 3), and every
+candidate value is summed over with its draft probability q(x) (candidates
+are i.i.d. draws from q, Sec. 4).  The cost is V**k per node with k
+candidates, so this is for tiny vocabularies only.
+
+The shaping rules are written here a second time, independently of the C
+oracle and vectorised over the vocabulary:
+
+* SPECINFER: R' = (R - q)_+ / sum (R - q)_+                    (Eq. recur)
+* RESISPEC:  GetProxy of Algorithm 1 with budget Z = q(x0) - R(x0),
+  projection r = min(Z q, R) with r(x0) = 0, the deficit filled in
+  proportion to the remaining capacity R - r off x0, then
+  R' = norm(max(R - K, 0)) with K = R - r and K(x0) = q(x0).
+"""
+from __future__ import annotations
+
+from functools import lru_cache
+
+import numpy as np
+
+MODE_RESISPEC = 0
+MODE_SPECINFER = 1
+
+
+def shape_specinfer(R, q, x0=None):
+    d = np.maximum(R - q, 0.0)
+    s = d.sum()
+    return R.copy() if not s > 0 else d / s
+
+
+def proxy_resispec(R, q, x0):
+    """Returns (K, r, Z) of GetProxy(R, q, x0)."""
+    Z = q[x0] - R[x0]
+    r = np.minimum(Z * q, R)
+    r[x0] = 0.0
+    cap = R - r
+    cap[x0] = 0.0
+    deficit = Z - r.sum()
+    if cap.sum() > 0:
+        r = r + deficit * cap / cap.sum()
+    K = R - r
+    K[x0] = q[x0]
+    return K, r, Z
+
+
+def shape_resispec(R, q, x0):
+    K, r, Z = proxy_resispec(R, q, x0)
+    if not Z > 0:
+        return R.copy()
+    d = np.maximum(R - K, 0.0)
+    s = d.sum()
+    return R.copy() if not s > 0 else d / s
+
+
+def shape(mode, R, q, x0):
+    return shape_specinfer(R, q) if mode == MODE_SPECINFER else shape_resispec(R, q, x0)
+
+
+def single_position(p, q, k, mode):
+    """Exact distribution of the emitted token when k i.i.d. candidates from q
+    are tested in order against the residual chain starting at p, with the
+    residual sample after k rejections.
+
+    Returns (dist, accept_prob_by_position) where accept_prob_by_position[i]
+    is P(candidate i+1 is the accepted one).
+    """
+    p = np.asarray(p, dtype=np.float64)
+    q = np.asarray(q, dtype=np.float64)
+    V = p.size
+    acc = np.zeros(k)
+
+    def rec(R, m, weight, depth):
+        out = np.zeros(V)
+        if m == 0:
+            return R.copy()
+        for x in range(V):
+            if q[x] <= 0:
+                continue
+            a = min(1.0, R[x] / q[x])
+            out[x] += q[x] * a
+            acc[depth] += weight * q[x] * a
+            if a < 1.0:
+                R2 = shape(mode, R, q, x)
+                out += q[x] * (1.0 - a) * rec(R2, m - 1, weight * q[x] * (1.0 - a), depth + 1)
+        return out
+
+    dist = rec(p.copy(), k, 1.0, 0)
+    return dist, acc
+
+
+def tree_walk(parents, rows, mode):
+    """Exact distribution over emitted token tuples for a draft tree.
+
+    ``parents``: int [N] (parent < child, -1 = root).  ``rows(path)`` returns
+    (p, q) for the node reached by the token tuple ``path`` (rows depend on
+    the path only, so duplicate siblings share rows as a real model would).
+    The emitted tuple is the accepted tokens followed by the residual (all
+    children rejected) or bonus (accepted node without children) token.
+    Returns {tuple: probability}.
+    """
+    parents = list(int(x) for x in parents)
+    kids = {n: [c for c, pa in enumerate(parents) if pa == n]
+            for n in [-1] + list(range(len(parents)))}
+
+    @lru_cache(maxsize=None)
+    def visit(node, path):
+        p, q = rows(path)
+        p = np.asarray(p, dtype=np.float64)
+        q = np.asarray(q, dtype=np.float64)
+        ch = kids[node]
+        if not ch:
+            return {(y,): float(p[y]) for y in range(p.size) if p[y] > 0}
+
+        def rec(R, j):
+            out = {}
+            if j == len(ch):
+                for y in range(R.size):
+                    if R[y] > 0:
+                        out[(y,)] = out.get((y,), 0.0) + float(R[y])
+                return out
+            c = ch[j]
+            for x in range(q.size):
+                if q[x] <= 0:
+                    continue
+                a = min(1.0, R[x] / q[x])
+                if a > 0:
+                    for seq, pr in visit(c, path + (x,)).items():
+                        key = (x,) + seq
+                        out[key] = out.get(key, 0.0) + q[x] * a * pr
+                if a < 1.0:
+                    R2 = shape(mode, R, q, x)
+                    for seq, pr in rec(R2, j + 1).items():
+                        out[seq] = out.get(seq, 0.0) + q[x] * (1.0 - a) * pr
+            return out
+
+        return rec(p.copy(), 0)
+
+    return visit(-1, ())

@@ -1,0 +1,464 @@
+#!/usr/bin/env python3
+"""Benchmark of the fused ResiSpec verification kernel on GB300.
+
+One step = one resispec_verify call over one batch of synthetic input (the
+whole hot path: tempered normaliser, accept tests, residual shaping, tree
+walk, residual/bonus sampling, Philox).  Default workload: B = 64 sequences,
+V = 151936, fp32 logits, full binary tree of depth 5 (62 nodes per
+sequence), Zipf-plus-Gaussian logits (slope 1.0, scale 4, rho 0.8), T = 1.0,
+ResiSpec mode.
+
+Prints one JSON line (rank 0).  `value` is verified tree nodes per second
+over all ranks (B * N per call); the roofline object reports algorithmic
+logit bytes (only the rows the walk visits) per launch over the measured
+launch time against the measured HBM copy bandwidth.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import math
+import os
+import re
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = ("verified tree nodes/sec and HBM GB/s (fraction of 8 TB/s) at 1 GB300 vs CPU oracle")
+NOMINAL_HBM_GBS = 8000.0
+FALLBACK_HBM_GBS = 6800.0
+L2_BYTES = 129 * 1024 * 1024
+
+
+def parse_args(argv=None):
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=2000)
+    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", default="binary5-v151936-b64")
+    ap.add_argument("--rho", type=float, default=None)
+    ap.add_argument("--mode", choices=["resispec", "specinfer"], default="resispec")
+    ap.add_argument("--pool", type=int, default=0, help="input sets rotated between steps (0 = auto)")
+    ap.add_argument("--cluster-size", type=int, default=0)
+    ap.add_argument("--block-threads", type=int, default=0)
+    ap.add_argument("--e2e-steps", type=int, default=12)
+    ap.add_argument("--cpu-seqs", type=int, default=16)
+    ap.add_argument("--cpu-seconds", type=float, default=12.0)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-clocks", action="store_true")
+    ap.add_argument("--seed", type=int, default=1234)
+    return ap.parse_args(argv)
+
+
+def measured_peak():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "measured"
+    except Exception:
+        return FALLBACK_HBM_GBS, "fallback"
+
+
+def kernel_source_digest():
+    h = hashlib.sha256()
+    csrc = os.path.join(ROOT, "paper_2608_24411_gb300", "csrc")
+    for name in sorted(os.listdir(csrc)):
+        with open(os.path.join(csrc, name), "rb") as f:
+            h.update(name.encode())
+            h.update(f.read())
+    return h.hexdigest()[:16]
+
+
+def profiled_traffic(workload):
+    """DRAM bytes per launch from the committed ncu summary of this
+    workload, if it was taken on the current kernel source."""
+    path = os.path.join(ROOT, "profiles", f"verify_kernel_{workload}.md")
+    if not os.path.exists(path):
+        return None
+    text = open(path).read()
+    m_src = re.search(r"kernel_source_digest:\s*([0-9a-f]+)", text)
+    m_tr = re.search(r"dram_bytes_per_launch:\s*([0-9.eE+]+)", text)
+    if not m_src or not m_tr or m_src.group(1) != kernel_source_digest():
+        return None
+    return float(m_tr.group(1))
+
+
+# ------------------------------------------------------------------ clocks
+
+
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, device_index, enabled=True):
+        self.proc = None
+        self.path = None
+        self.dev = device_index
+        if not enabled:
+            return
+        try:
+            os.makedirs(os.path.join(ROOT, "gpurun_out"), exist_ok=True)
+            self.path = os.path.join(ROOT, "gpurun_out", f"clocks_rank{device_index}.csv")
+            self.fh = open(self.path, "w")
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={device_index}", f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=self.fh, stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        self.fh.close()
+        sm, mx, reasons = [], None, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in open(self.path):
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                mx = float(parts[2])
+            except ValueError:
+                continue
+            for n, v in zip(names, parts[5:9]):
+                if v.lower().startswith("active"):
+                    reasons.add(n)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": mx, "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# ------------------------------------------------------------------ helpers
+
+
+def rows_visited(nodes, accept_len, haschild):
+    """Logit rows each sequence read: 2 per visited node with children
+    (target + draft), 1 for a visited node without children (bonus: target
+    only).  Visited nodes are the root and every accepted node."""
+    a = accept_len.astype(np.int64)
+    D = nodes.shape[1]
+    root = 2 if haschild[0] else 1
+    rows = np.full(a.shape, root, dtype=np.int64)
+    for d in range(D):
+        mask = a > d
+        if not mask.any():
+            break
+        nd = nodes[mask, d]
+        rows[mask] += np.where(haschild[nd + 1], 2, 1)
+    return rows
+
+
+def cpu_oracle_rate(w, target_h, draft_h, parents, cand_h, seq_ids, mode, seconds, seed0):
+    """Time the fp64 oracle as it stands on this host's cores over a bounded
+    sample; returns (nodes/s, threads, sample description)."""
+    import oracle
+    S = cand_h.shape[0]
+    threads = min(os.cpu_count() or 1, S)
+    oracle.verify(target_h[:1], draft_h[:1], parents, cand_h[:1], w.temperature, seed0,
+                  mode=mode, max_depth=w.max_depth, seq_ids=seq_ids[:1], nthreads=1)
+    reps, t0 = 0, time.perf_counter()
+    while True:
+        oracle.verify(target_h, draft_h, parents, cand_h, w.temperature, seed0 + reps, mode=mode,
+                      max_depth=w.max_depth, seq_ids=seq_ids, nthreads=threads)
+        reps += 1
+        el = time.perf_counter() - t0
+        if el >= seconds or reps >= 200:
+            break
+    nodes = reps * S * w.num_nodes
+    sample = (f"{reps} calls x {S} sequences of {w.name} (rows copied to host), "
+              f"{nodes} verified nodes in {el:.2f} s")
+    return nodes / el, threads, sample
+
+
+# ------------------------------------------------------------------ reference arm
+
+
+def run_reference(args):
+    """The oracle as it stands on the host cores, on this arm's workload."""
+    import oracle
+    from paper_2608_24411_gb300 import workloads as W
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return 0
+    w = W.WORKLOADS[args.workload]
+    if args.rho is not None:
+        w = W.with_rho(w, args.rho)
+    mode = oracle.MODE_SPECINFER if args.mode == "specinfer" else oracle.MODE_RESISPEC
+    S = max(1, args.cpu_seqs)
+    inp = W.make_inputs_np(w, seed=args.seed, batch=S)
+    seq_ids = np.arange(S, dtype=np.int32)
+    threads = min(os.cpu_count() or 1, S)
+
+    def step(i):
+        oracle.verify(inp["target"], inp["draft"], inp["parents"], inp["cand"], w.temperature,
+                      args.seed + i, mode=mode, max_depth=w.max_depth, seq_ids=seq_ids,
+                      nthreads=threads)
+
+    for i in range(max(0, args.warmup)):
+        step(i)
+    t0 = time.perf_counter()
+    for i in range(args.steps):
+        step(args.warmup + i)
+    el = time.perf_counter() - t0
+    value = args.steps * S * w.num_nodes / el
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": "nodes/s",
+        "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": 1e3 * el / max(1, args.steps), "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": w.name, "batch_per_step": S, "vocab": w.vocab,
+                   "nodes_per_seq": w.num_nodes, "mode": args.mode, "rho": w.rho},
+        "cpu_baseline": {"value": value, "unit": "nodes/s", "cores": threads, "kind": "oracle",
+                         "sample": f"{S} sequences of {w.name} per step (host inputs)"},
+        "e2e": {"value": value, "unit": "nodes/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+# ------------------------------------------------------------------ our arm
+
+
+def run_ours(args):
+    import torch
+    import paper_2608_24411_gb300 as rs
+    from paper_2608_24411_gb300 import workloads as W
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world != args.gpus and world > 1:
+        raise SystemExit(f"--gpus {args.gpus} but WORLD_SIZE {world}")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=dev)
+
+    def barrier():
+        if dist is not None:
+            dist.barrier()
+
+    def max_over_ranks(x):
+        if dist is None:
+            return x
+        t = torch.tensor([x], dtype=torch.float64, device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        return float(t.item())
+
+    def sum_over_ranks(x):
+        if dist is None:
+            return x
+        t = torch.tensor([x], dtype=torch.float64, device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.SUM)
+        return float(t.item())
+
+    rs.build()
+    rs.load_library()
+    w = W.WORKLOADS[args.workload]
+    if args.rho is not None:
+        w = W.with_rho(w, args.rho)
+    mode = rs.MODE_SPECINFER if args.mode == "specinfer" else rs.MODE_RESISPEC
+    B, N, V, D = w.batch, w.num_nodes, w.vocab, w.max_depth
+    es = w.elem_bytes
+    set_bytes = 2 * B * (N + 1) * V * es
+    pool = args.pool or max(2, min(8, math.ceil(4 * L2_BYTES / max(1, 2 * B * V * es))))
+    sets = [W.make_inputs_torch(w, seed=args.seed + 7919 * rank + 31 * i, device=dev)
+            for i in range(pool)]
+    parents_np = w.parents
+    haschild = np.zeros(N + 1, dtype=bool)
+    for c, p in enumerate(parents_np):
+        haschild[p + 1] = True
+    K, Wm = args.steps, args.warmup
+    outs = [(torch.empty((B, D + 1), dtype=torch.int32, device=dev),
+             torch.empty((B,), dtype=torch.int32, device=dev),
+             torch.empty((B, max(D, 1)), dtype=torch.int32, device=dev)) for _ in range(K)]
+    status = torch.zeros((1,), dtype=torch.int32, device=dev)
+    kw = dict(max_depth=D, mode=mode, cluster_size=args.cluster_size,
+              block_threads=args.block_threads, status=status)
+    stream = torch.cuda.current_stream(dev)
+    plan = rs.plan(B, N, V, D, w.dtype, cluster_size=args.cluster_size,
+                   block_threads=args.block_threads)
+
+    def launch(i, out):
+        s = sets[i % pool]
+        rs.verify(s["target"], s["draft"], s["parents"], s["cand"], w.temperature,
+                  args.seed + i, out_tokens=out[0], out_accept_len=out[1], out_nodes=out[2],
+                  stream=stream, **kw)
+
+    for i in range(Wm):
+        launch(i, outs[i % K])
+    torch.cuda.synchronize()
+
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(K + 1)]
+    clocks = ClockSampler(local, enabled=not args.no_clocks)
+    time.sleep(0.3 if not args.no_clocks else 0)
+    barrier()
+    torch.cuda.synchronize()
+    wall0 = time.perf_counter()
+    ev[0].record(stream)
+    for i in range(K):
+        launch(Wm + i, outs[i])
+        ev[i + 1].record(stream)
+    torch.cuda.synchronize()
+    barrier()
+    wall = time.perf_counter() - wall0
+    clk = clocks.stop()
+    launch_ms = [ev[i].elapsed_time(ev[i + 1]) for i in range(K)]
+    elapsed_ms = ev[0].elapsed_time(ev[K])
+    elapsed_ms = max_over_ranks(elapsed_ms)
+    if int(status.item()) & ~rs.INFO_DEGENERATE:
+        raise SystemExit(f"kernel reported data errors: status {int(status.item())}")
+
+    alg_bytes = 0
+    emitted = 0
+    accepted = 0
+    for i in range(K):
+        alen = outs[i][1].cpu().numpy()
+        nodes = outs[i][2].cpu().numpy()[:, :D]
+        rows = rows_visited(nodes, alen, haschild)
+        alg_bytes += int(rows.sum()) * V * es
+        emitted += int((alen + 1).sum())
+        accepted += int(alen.sum())
+    total_nodes = sum_over_ranks(float(K * B * N))
+    value = total_nodes / (elapsed_ms / 1e3)
+    mean_launch_s = (sum(launch_ms) / K) / 1e3
+    achieved_gbs = (alg_bytes / K) / mean_launch_s / 1e9
+    peak, peak_kind = measured_peak()
+
+    result = {
+        "metric": METRIC, "value": value, "unit": "nodes/s", "n_gpus": world, "steps": K,
+        "warmup": Wm, "ms_per_step": elapsed_ms / K, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": w.dtype, "data": "synthetic",
+        "config": {
+            "workload": w.name, "batch": B, "vocab": V, "nodes_per_seq": N, "max_depth": D,
+            "tree": list(w.tree[1]) if w.tree[0] == "levels" else list(w.tree[1:]),
+            "logits": f"{w.gen} slope {w.slope} scale {w.scale} rho {w.rho}",
+            "temperature": w.temperature, "mode": args.mode,
+            "parallelism": f"replicas{world}" if world > 1 else "single",
+            "launch": {k: plan[k] for k in ("cluster_size", "block_threads", "smem_bytes",
+                                            "slice_elems", "uses_tma")},
+            "l2": f"rotating pool of {pool} input sets ({set_bytes / 1e9:.2f} GB each) "
+                  f"between steps; each step's visited rows exceed L2 together",
+        },
+        "roofline": {"bound": "hbm", "achieved": achieved_gbs, "peak": peak, "unit": "GB/s",
+                     "frac": achieved_gbs / peak, "traffic": profiled_traffic(w.name),
+                     "peak_kind": peak_kind, "frac_of_8tbs": achieved_gbs / NOMINAL_HBM_GBS,
+                     "alg_bytes_per_launch": alg_bytes / K,
+                     "mean_launch_us": mean_launch_s * 1e6},
+        "tokens_per_s": sum_over_ranks(float(emitted)) / (elapsed_ms / 1e3),
+        "mean_accept_len": accepted / (K * B),
+        "gpu_launches": K,
+        "wall_s": wall,
+    }
+    if clk:
+        result["clocks"] = clk
+
+    # ---- end to end through the public API with host buffers
+    if not args.no_e2e:
+        s0 = sets[0]
+        host = {k: s0[k].cpu().pin_memory() for k in ("target", "draft", "cand")}
+        host["parents"] = s0["parents"].cpu().pin_memory()
+        dbuf = {k: torch.empty_like(s0[k]) for k in ("target", "draft", "cand", "parents")}
+        h_tok = torch.empty((B, D + 1), dtype=torch.int32).pin_memory()
+        h_len = torch.empty((B,), dtype=torch.int32).pin_memory()
+        d_tok = torch.empty((B, D + 1), dtype=torch.int32, device=dev)
+        d_len = torch.empty((B,), dtype=torch.int32, device=dev)
+        h2d = sum(t.numel() * t.element_size() for t in host.values())
+        d2h = h_tok.numel() * 4 + h_len.numel() * 4
+        E = max(1, args.e2e_steps)
+
+        def e2e_step(i):
+            for k in dbuf:
+                dbuf[k].copy_(host[k], non_blocking=True)
+            rs.verify(dbuf["target"], dbuf["draft"], dbuf["parents"], dbuf["cand"],
+                      w.temperature, args.seed + i, out_tokens=d_tok, out_accept_len=d_len,
+                      max_depth=D, mode=mode, stream=stream)
+            h_tok.copy_(d_tok, non_blocking=True)
+            h_len.copy_(d_len, non_blocking=True)
+
+        e2e_step(0)
+        torch.cuda.synchronize()
+        barrier()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for i in range(E):
+            e2e_step(i + 1)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        barrier()
+        e_ms = max_over_ranks(e0.elapsed_time(e1))
+        result["e2e"] = {"value": sum_over_ranks(float(E * B * N)) / (e_ms / 1e3),
+                         "unit": "nodes/s", "h2d_bytes_per_step": h2d,
+                         "d2h_bytes_per_step": d2h, "steps": E}
+        del host, dbuf
+
+    # ---- the oracle as it stands on the host cores (rank 0, N = 1 only)
+    result = _finish_cpu(result, args, sets, w, mode, world, dev)
+    if rank == 0:
+        print(json.dumps(result), flush=True)
+    if dist is not None:
+        dist.destroy_process_group()
+    return 0
+
+
+def _host_logits(t):
+    import torch
+    if t.dtype == torch.bfloat16:
+        return t.contiguous().view(torch.int16).cpu().numpy().view(np.uint16)
+    return t.contiguous().cpu().numpy()
+
+
+def _finish_cpu(result, args, sets, w, mode, world, dev):
+    if args.no_cpu_baseline or world != 1:
+        return result
+    import torch
+    import oracle
+    S = max(1, min(args.cpu_seqs, w.batch))
+    s0 = sets[0]
+    idx = torch.arange(S, device=dev)
+    th = _host_logits(s0["target"].index_select(0, idx))
+    dh = _host_logits(s0["draft"].index_select(0, idx))
+    ch = s0["cand"].index_select(0, idx).cpu().numpy()
+    omode = oracle.MODE_SPECINFER if mode == 1 else oracle.MODE_RESISPEC
+    rate, threads, sample = cpu_oracle_rate(w, th, dh, w.parents, ch,
+                                            np.arange(S, dtype=np.int32), omode,
+                                            args.cpu_seconds, args.seed)
+    result["cpu_baseline"] = {"value": rate, "unit": "nodes/s", "cores": threads,
+                              "kind": "oracle", "sample": sample}
+    return result
+
+
+def main(argv=None):
+    args = parse_args(argv)
+    if args.impl == "reference":
+        return run_reference(args)
+    return run_ours(args)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

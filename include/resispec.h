@@ -1,0 +1,158 @@
+/*
+ * resispec.h -- C ABI of the ResiSpec verification library (GB300, sm_103a).
+ *
+ * One call verifies a batch of draft token trees against their target
+ * logits, as in the verification step of multi-candidate speculative
+ * sampling (paper: "ResiSpec: Enhancing Multi-Candidate Speculative Sampling
+ * via Residual Distribution Shaping", Sec. 3 and Algorithm 1):
+ *
+ *   for every sequence b: start at the root; turn the node's target and
+ *   draft logits into tempered distributions p, q (softmax(z / T)); test the
+ *   node's children in ascending node order with u < R(x) / q(x), R starting
+ *   at p; after each rejection reshape R (ResiSpec: GetProxy of Algorithm 1;
+ *   SpecInfer: Eq. recur); on acceptance emit the child's token and descend
+ *   into it; when every child is rejected emit x ~ R; when an accepted node
+ *   has no children emit a bonus token x ~ p of that node.
+ *
+ * Conventions for every entry point below:
+ *   - Pointers named *_logits, tree_parents, cand_tokens, out_* and status
+ *     are DEVICE pointers owned by the caller (e.g. the storage of torch
+ *     tensors).  The library allocates no device memory and keeps no
+ *     reference to any pointer after the call returns.
+ *   - Work is enqueued on `stream` (a cudaStream_t; NULL = legacy default
+ *     stream) and the call returns without synchronising.
+ *   - Argument errors are returned synchronously as a resispec_status and
+ *     nothing is launched.  Errors that depend on device data are reported
+ *     on the device (see RESISPEC_ERR_*): the kernel never traps.
+ *   - Randomness: u = U(seed, b, row, draw) from Philox4x64-10 (Salmon et
+ *     al., SC 2011) with key (seed, 0) and counter (row, b, 0, 0);
+ *     u = (word[draw] >> 40) * 2^-24.  The accept test of candidate node c
+ *     uses row c+1, draw 0; the residual / bonus draw at the node whose
+ *     logits are row r uses row r, draw 1.  Outputs are a pure function of
+ *     the inputs, seed and mode.
+ */
+#ifndef RESISPEC_H_
+#define RESISPEC_H_
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define RESISPEC_ABI_VERSION 1
+
+/* Synchronous return codes. */
+typedef enum {
+  RESISPEC_OK = 0,
+  RESISPEC_E_ARG = 1,         /* NULL pointer, temperature not finite or <= 0, bad option */
+  RESISPEC_E_SHAPE = 2,       /* a size outside the supported range */
+  RESISPEC_E_DTYPE = 3,       /* dtype not RESISPEC_F32 / RESISPEC_BF16 */
+  RESISPEC_E_UNSUPPORTED = 4, /* device is not sm_103 or cannot host the cluster */
+  RESISPEC_E_CUDA = 5         /* a CUDA runtime call failed; see resispec_last_error() */
+} resispec_status;
+
+typedef enum { RESISPEC_F32 = 0, RESISPEC_BF16 = 1 } resispec_dtype;
+
+/* RESISPEC: Algorithm 1 with GetProxy (budget Z = q(x0) - R(x0), deficit
+ *   filled in proportion to the remaining capacity R - r off x0).
+ * SPECINFER: the residual recurrence R <- (R - q)_+ / sum (Eq. recur). */
+typedef enum { RESISPEC_MODE_RESISPEC = 0, RESISPEC_MODE_SPECINFER = 1 } resispec_mode;
+
+/* Bits of the optional device status word (atomically OR-ed per sequence).
+ * A sequence with an ERR bit gets out_accept_len = -1 and an all -1 token
+ * row. */
+#define RESISPEC_ERR_TREE 1        /* tree_parents[c] not in [-1, c) */
+#define RESISPEC_ERR_TOKEN 2       /* a tested candidate token outside [0, V) */
+#define RESISPEC_ERR_NONFINITE 4   /* NaN or +inf in a visited logit row */
+#define RESISPEC_ERR_EMPTY_ROW 8   /* a visited row (or the residual) has no mass */
+#define RESISPEC_ERR_DEPTH 16      /* more accepted tokens than max_depth */
+#define RESISPEC_ERR_TIMEOUT 32    /* a bounded wait for a row copy gave up */
+#define RESISPEC_INFO_DEGENERATE 256 /* informational: a rejection left R unchanged */
+
+#define RESISPEC_MAX_VOCAB 262144
+#define RESISPEC_MAX_NODES 4096
+
+/* Sizes of one call.  Logit rows: row 0 is the root, row j+1 is node j. */
+typedef struct {
+  int32_t batch;     /* B >= 0 sequences (B = 0 launches nothing) */
+  int32_t num_nodes; /* N in [0, RESISPEC_MAX_NODES] tree nodes, root excluded */
+  int32_t vocab;     /* V in [1, RESISPEC_MAX_VOCAB] */
+  int32_t max_depth; /* D >= 0; out_tokens has D + 1 columns */
+  int32_t dtype;     /* resispec_dtype of both logit arrays */
+} resispec_dims;
+
+#define RESISPEC_FLAG_NO_TMA 1 /* force plain loads instead of bulk copies */
+
+typedef struct {
+  int32_t mode;          /* resispec_mode */
+  int32_t cluster_size;  /* CTAs per sequence: 0 = automatic, else 1, 2, 4, 8, 16 */
+  int32_t block_threads; /* 0 = automatic, else 256 or 512 */
+  int32_t flags;         /* RESISPEC_FLAG_* */
+  int64_t seq_stride;    /* elements between sequences in both logit arrays;
+                            -1 = (N + 1) * V; 0 shares one set of rows */
+  int32_t* status;       /* optional device int32 OR-ed with RESISPEC_ERR_* bits */
+  int32_t* out_nodes;    /* optional device [B, D] accepted node ids, -1 padded */
+  float* out_dist;       /* optional device [B, V] fp32: the distribution the
+                            last emitted token was drawn from (final residual
+                            R, or p of the accepted leaf) */
+  int32_t* out_rejects;  /* optional device [B] number of rejections */
+} resispec_opts;
+
+/* Fills *opts with the defaults (RESISPEC mode, automatic launch shape,
+ * seq_stride -1, no optional outputs). */
+void resispec_opts_default(resispec_opts* opts);
+
+/* Verify a batch of draft trees (Sec. 3; Algorithm 1; GetProxy).
+ *   target_logits  [B, N+1, V] dtype, row-major, 16-byte aligned for the
+ *                  bulk-copy path (otherwise plain loads are used)
+ *   draft_logits   [B, N+1, V] same layout
+ *   tree_parents   [N] int32, parent of node c (-1 = root), parent < c;
+ *                  siblings are tested in ascending node index
+ *   cand_tokens    [B, N] int32, token proposed at node c (drawn i.i.d. from
+ *                  the parent's tempered draft distribution by the caller)
+ *   temperature    T > 0, applied to target and draft logits alike
+ *   seed           Philox key (see the header comment)
+ *   out_tokens     [B, D+1] int32: accepted tokens, then the residual / bonus
+ *                  token, then -1 padding
+ *   out_accept_len [B] int32: number of accepted candidates (-1 on a
+ *                  per-sequence data error)
+ * Uses RESISPEC mode and automatic launch shape. */
+int resispec_verify(const void* target_logits, const void* draft_logits,
+                    const int32_t* tree_parents, const int32_t* cand_tokens,
+                    float temperature, uint64_t seed, int32_t* out_tokens,
+                    int32_t* out_accept_len, resispec_dims dims, void* stream);
+
+/* resispec_verify with options (mode, launch shape, stride, optional
+ * outputs).  opts may be NULL (defaults). */
+int resispec_verify_ex(const void* target_logits, const void* draft_logits,
+                       const int32_t* tree_parents, const int32_t* cand_tokens,
+                       float temperature, uint64_t seed, int32_t* out_tokens,
+                       int32_t* out_accept_len, resispec_dims dims,
+                       const resispec_opts* opts, void* stream);
+
+/* Launch shape resispec_verify_ex would use (no launch): CTAs per sequence,
+ * threads per CTA, dynamic shared memory bytes per CTA, vocabulary elements
+ * per CTA, and 1 if rows are fetched with bulk copies.  Any output pointer
+ * may be NULL. */
+int resispec_plan(resispec_dims dims, const resispec_opts* opts,
+                  int32_t* cluster_size, int32_t* block_threads,
+                  int32_t* smem_bytes, int32_t* slice_elems, int32_t* uses_tma);
+
+/* Device Philox draws for testing the counter-based generator: for i < n,
+ * u0[i] = U(seed, seq[i], row[i], 0) and u1[i] = U(seed, seq[i], row[i], 1).
+ * seq, row, u0, u1 are device arrays of length n. */
+int resispec_uniforms(uint64_t seed, const int32_t* seq, const int32_t* row,
+                      int32_t n, float* u0, float* u1, void* stream);
+
+/* Text of a status code / of the last CUDA error seen by this thread. */
+const char* resispec_status_string(int status);
+const char* resispec_last_error(void);
+
+int resispec_abi_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* RESISPEC_H_ */

@@ -77,6 +77,7 @@ class _Args(ctypes.Structure):
         ("out_accept_margin", ctypes.c_void_p), ("out_sample_margin", ctypes.c_void_p),
         ("out_status", ctypes.c_void_p), ("out_rejects", ctypes.c_void_p),
         ("out_rows", ctypes.c_void_p), ("out_inv_err", ctypes.c_void_p),
+        ("out_cond", ctypes.c_void_p),
     ]
 
 
@@ -224,6 +225,7 @@ def verify(target, draft, parents, cand, temperature, seed, *, mode=MODE_RESISPE
         "rejects": np.zeros(B, np.int32),
         "rows": np.zeros(B, np.int32),
         "inv_err": np.zeros(B),
+        "cond": np.ones(B),
     }
     if want_dist:
         out["dist"] = np.zeros((B, V))
@@ -249,6 +251,7 @@ def verify(target, draft, parents, cand, temperature, seed, *, mode=MODE_RESISPE
     a.out_rejects = out["rejects"].ctypes.data
     a.out_rows = out["rows"].ctypes.data
     a.out_inv_err = out["inv_err"].ctypes.data
+    a.out_cond = out["cond"].ctypes.data
     rc = lib.oracle_verify(ctypes.byref(a))
     if rc != 0:
         raise ValueError("oracle_verify rejected its arguments")

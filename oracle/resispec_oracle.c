@@ -199,6 +199,10 @@ static double residual_from(double* R, const double* K, int V, double* tmp) {
   return s;
 }
 
+int oracle_reject_ex(int mode, double* R, const double* q, int V, int x0,
+                     double* K, double* r, double* tmp, double* inv_err,
+                     double* norm_out);
+
 /* One rejection of token x0 applied to the residual R (length V).
  * mode SPECINFER: R <- norm(max(R - q, 0))              (Eq. recur)
  * mode RESISPEC:  K = GetProxy(R, q, x0); R <- norm(max(R - K, 0)) (Alg. 1)
@@ -207,8 +211,18 @@ static double residual_from(double* R, const double* K, int V, double* tmp) {
  * the largest violation is max-ed into *inv_err. */
 int oracle_reject(int mode, double* R, const double* q, int V, int x0,
                   double* K, double* r, double* tmp, double* inv_err) {
+  return oracle_reject_ex(mode, R, q, V, x0, K, r, tmp, inv_err, NULL);
+}
+
+/* As oracle_reject; *norm_out receives the SpecInfer normaliser
+ * sum (R - q)_+ of this rejection (1 in ResiSpec mode). */
+int oracle_reject_ex(int mode, double* R, const double* q, int V, int x0,
+                     double* K, double* r, double* tmp, double* inv_err,
+                     double* norm_out) {
+  if (norm_out) *norm_out = 1.0;
   if (mode == OR_MODE_SPECINFER) {
     double changed = residual_from(R, q, V, tmp);
+    if (norm_out && changed > 0.0) *norm_out = changed;
     if (inv_err && changed > 0.0) {
       double s = 0.0, e = 0.0;
       for (int i = 0; i < V; ++i) {
@@ -308,6 +322,8 @@ typedef struct {
   int32_t* out_rejects;    /* [B] rejections along the walk */
   int32_t* out_rows;       /* [B] logit rows read (target + draft) */
   double* out_inv_err;     /* [B] largest invariant violation */
+  double* out_cond;        /* [B] 1 / prod of the SpecInfer normalisers at the
+                              final node (1 without SpecInfer rejections) */
 } oracle_args;
 
 typedef struct {
@@ -329,7 +345,7 @@ static void verify_sequence(const oracle_args* a, int lb, int tree_bad,
   if (nodes)
     for (int i = 0; i < D; ++i) nodes[i] = -1;
   int status = 0, depth = 0, rejects = 0, rows = 0;
-  double amargin = INFINITY, smargin = INFINITY, inv = 0.0;
+  double amargin = INFINITY, smargin = INFINITY, inv = 0.0, cond = 1.0;
   double* inv_ptr = a->check_invariants ? &inv : NULL;
   const size_t seq_off = (size_t)(a->seq_stride * lb);
 
@@ -352,6 +368,7 @@ static void verify_sequence(const oracle_args* a, int lb, int tree_bad,
     }
     if (nk == 0) {
       /* bonus token: the accepted node has no children (or N == 0) */
+      cond = 1.0;
       double u = oracle_uniform(a->seed, gb, row, 1);
       int y = oracle_sample(p, V, u, &smargin);
       if (toks) toks[depth] = y;
@@ -366,6 +383,7 @@ static void verify_sequence(const oracle_args* a, int lb, int tree_bad,
       goto done;
     }
     memcpy(R, p, sizeof(double) * V); /* R <- P, D <- Q (Algorithm 1) */
+    cond = 1.0;
     int accepted = -1;
     for (int j = 0; j < nk; ++j) {
       int c = kids[j];
@@ -392,8 +410,10 @@ static void verify_sequence(const oracle_args* a, int lb, int tree_bad,
         break;
       }
       rejects += 1;
-      if (!oracle_reject(a->mode, R, q, V, x, K, r, tmp, inv_ptr))
+      double norm = 1.0;
+      if (!oracle_reject_ex(a->mode, R, q, V, x, K, r, tmp, inv_ptr, &norm))
         status |= OR_INFO_DEGENERATE;
+      cond /= norm;
     }
     if (accepted < 0) {
       double u = oracle_uniform(a->seed, gb, row, 1);
@@ -427,6 +447,7 @@ done:
   if (a->out_rejects) a->out_rejects[lb] = rejects;
   if (a->out_rows) a->out_rows[lb] = rows;
   if (a->out_inv_err) a->out_inv_err[lb] = inv;
+  if (a->out_cond) a->out_cond[lb] = cond;
 }
 
 static void* worker(void* arg) {

@@ -1,0 +1,294 @@
+// Host side of the C ABI declared in include/resispec.h: argument checks,
+// launch planning (cluster size, threads, shared memory) and the cluster
+// launch of the fused verification kernel on the caller's stream.
+#include <cuda_runtime.h>
+#include <math.h>
+#include <stdint.h>
+#include <stdio.h>
+#include <string.h>
+
+#include <mutex>
+
+#include "../../include/resispec.h"
+#include "verify_kernel.cuh"
+
+namespace {
+
+thread_local char g_last_error[256] = "";
+
+void set_error(const char* what, cudaError_t e) {
+  snprintf(g_last_error, sizeof g_last_error, "%s: %s (%d)", what, cudaGetErrorString(e),
+           (int)e);
+}
+
+constexpr int kMaxSmem = 227 * 1024;      // dynamic shared memory per CTA on sm_10x
+constexpr int kAutoSliceBytes = 96 * 1024; // target on-chip bytes per CTA (two fp32 rows)
+
+struct Plan {
+  int C = 1;
+  int threads = 512;
+  int L = 8;
+  int npad = 16;
+  int smem = 0;
+  int use_tma = 0;
+};
+
+int round_up(int x, int m) { return (x + m - 1) / m * m; }
+
+int slice_for(int V, int C) { return round_up((V + C - 1) / C, 8); }
+
+int smem_for(int L, int npad) {
+  const int tree = npad * 2 + npad * 2 + npad * 4 + (npad + 16);
+  return round_up(rs::kHeadBytes + 8 * L + tree, 128);
+}
+
+struct DeviceInfo {
+  int sms = 0;
+  int major = 0;
+  int minor = 0;
+};
+
+std::mutex g_mu;
+DeviceInfo g_dev[64];
+bool g_attr_set[64][4];
+
+int query_device(int* dev_out, DeviceInfo* info) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) { set_error("cudaGetDevice", e); return RESISPEC_E_CUDA; }
+  if (dev < 0 || dev >= 64) return RESISPEC_E_UNSUPPORTED;
+  std::lock_guard<std::mutex> lk(g_mu);
+  DeviceInfo& d = g_dev[dev];
+  if (d.sms == 0) {
+    cudaDeviceProp prop;
+    e = cudaGetDeviceProperties(&prop, dev);
+    if (e != cudaSuccess) { set_error("cudaGetDeviceProperties", e); return RESISPEC_E_CUDA; }
+    d.sms = prop.multiProcessorCount;
+    d.major = prop.major;
+    d.minor = prop.minor;
+  }
+  *dev_out = dev;
+  *info = d;
+  return RESISPEC_OK;
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+int check_dims(const resispec_dims& d) {
+  if (d.batch < 0 || d.num_nodes < 0 || d.max_depth < 0) return RESISPEC_E_SHAPE;
+  if (d.vocab < 1 || d.vocab > RESISPEC_MAX_VOCAB) return RESISPEC_E_SHAPE;
+  if (d.num_nodes > RESISPEC_MAX_NODES) return RESISPEC_E_SHAPE;
+  if (d.max_depth > d.num_nodes) return RESISPEC_E_SHAPE;
+  if (d.dtype != RESISPEC_F32 && d.dtype != RESISPEC_BF16) return RESISPEC_E_DTYPE;
+  return RESISPEC_OK;
+}
+
+// Launch shape.  sms = 0 means unknown (no device query): the batch-fill
+// rule is skipped.
+int make_plan(const resispec_dims& d, const resispec_opts& o, int sms, const void* zt,
+              const void* zd, Plan* p) {
+  int st = check_dims(d);
+  if (st) return st;
+  if (o.mode != RESISPEC_MODE_RESISPEC && o.mode != RESISPEC_MODE_SPECINFER) return RESISPEC_E_ARG;
+  if (o.block_threads != 0 && o.block_threads != 256 && o.block_threads != 512)
+    return RESISPEC_E_ARG;
+  const int cs = o.cluster_size;
+  if (cs != 0 && cs != 1 && cs != 2 && cs != 4 && cs != 8 && cs != 16) return RESISPEC_E_ARG;
+  if (o.seq_stride < -1) return RESISPEC_E_ARG;
+  p->threads = o.block_threads ? o.block_threads : 512;
+  p->npad = round_up(d.num_nodes + 1, 16);
+  const int V = d.vocab;
+  if (cs) {
+    p->C = cs;
+  } else {
+    int C = 1;
+    while (C < 16 && 8 * slice_for(V, C) > kAutoSliceBytes) C *= 2;
+    // small batches: spread each sequence over more SMs to cut latency
+    while (sms > 0 && C < 16 && (int64_t)d.batch * C * 2 <= sms) C *= 2;
+    p->C = C;
+  }
+  p->L = slice_for(V, p->C);
+  p->smem = smem_for(p->L, p->npad);
+  if (p->smem > kMaxSmem) return RESISPEC_E_SHAPE;
+  const int64_t es = d.dtype == RESISPEC_BF16 ? 2 : 4;
+  const int64_t stride = o.seq_stride < 0 ? (int64_t)(d.num_nodes + 1) * V : o.seq_stride;
+  p->use_tma = !(o.flags & RESISPEC_FLAG_NO_TMA) && (V * es) % 16 == 0 &&
+               (stride * es) % 16 == 0 && (zt == nullptr || aligned16(zt)) &&
+               (zd == nullptr || aligned16(zd));
+  return RESISPEC_OK;
+}
+
+template <int THREADS, bool BF16>
+cudaError_t launch_verify(const Plan& pl, const rs::VerifyParams& prm, cudaStream_t stream,
+                          int dev) {
+  auto kern = rs::verify_kernel<THREADS, BF16>;
+  const int slot = (THREADS == 512 ? 2 : 0) + (BF16 ? 1 : 0);
+  {
+    std::lock_guard<std::mutex> lk(g_mu);
+    if (!g_attr_set[dev][slot]) {
+      cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, kMaxSmem);
+      if (e != cudaSuccess) return e;
+      e = cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+      if (e != cudaSuccess) return e;
+      g_attr_set[dev][slot] = true;
+    }
+  }
+  cudaLaunchConfig_t cfg;
+  memset(&cfg, 0, sizeof cfg);
+  cfg.gridDim = dim3((unsigned)(prm.B * pl.C), 1, 1);
+  cfg.blockDim = dim3(THREADS, 1, 1);
+  cfg.dynamicSmemBytes = (size_t)pl.smem;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = (unsigned)pl.C;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kern, prm);
+}
+
+}  // namespace
+
+extern "C" {
+
+void resispec_opts_default(resispec_opts* o) {
+  if (!o) return;
+  memset(o, 0, sizeof *o);
+  o->mode = RESISPEC_MODE_RESISPEC;
+  o->seq_stride = -1;
+}
+
+int resispec_abi_version(void) { return RESISPEC_ABI_VERSION; }
+
+const char* resispec_status_string(int s) {
+  switch (s) {
+    case RESISPEC_OK: return "ok";
+    case RESISPEC_E_ARG: return "invalid argument";
+    case RESISPEC_E_SHAPE: return "size outside the supported range";
+    case RESISPEC_E_DTYPE: return "unsupported dtype";
+    case RESISPEC_E_UNSUPPORTED: return "unsupported device";
+    case RESISPEC_E_CUDA: return "CUDA runtime error";
+    default: return "unknown status";
+  }
+}
+
+const char* resispec_last_error(void) { return g_last_error; }
+
+int resispec_plan(resispec_dims dims, const resispec_opts* opts, int32_t* cluster_size,
+                  int32_t* block_threads, int32_t* smem_bytes, int32_t* slice_elems,
+                  int32_t* uses_tma) {
+  resispec_opts o;
+  resispec_opts_default(&o);
+  if (opts) o = *opts;
+  int sms = 0;
+  int dev = 0;
+  DeviceInfo info;
+  int ndev = 0;
+  if (cudaGetDeviceCount(&ndev) == cudaSuccess && ndev > 0 && query_device(&dev, &info) == 0)
+    sms = info.sms;
+  else
+    cudaGetLastError();  // clear a sticky "no device" error
+  Plan p;
+  const int st = make_plan(dims, o, sms, nullptr, nullptr, &p);
+  if (st) return st;
+  if (cluster_size) *cluster_size = p.C;
+  if (block_threads) *block_threads = p.threads;
+  if (smem_bytes) *smem_bytes = p.smem;
+  if (slice_elems) *slice_elems = p.L;
+  if (uses_tma) *uses_tma = p.use_tma;
+  return RESISPEC_OK;
+}
+
+int resispec_verify_ex(const void* target_logits, const void* draft_logits,
+                       const int32_t* tree_parents, const int32_t* cand_tokens,
+                       float temperature, uint64_t seed, int32_t* out_tokens,
+                       int32_t* out_accept_len, resispec_dims dims,
+                       const resispec_opts* opts, void* stream) {
+  resispec_opts o;
+  resispec_opts_default(&o);
+  if (opts) o = *opts;
+  int st = check_dims(dims);
+  if (st) return st;
+  if (!(temperature > 0.f) || !isfinite(temperature)) return RESISPEC_E_ARG;
+  if (dims.batch == 0) return RESISPEC_OK;
+  if (!target_logits || !draft_logits || !out_tokens || !out_accept_len) return RESISPEC_E_ARG;
+  if (dims.num_nodes > 0 && (!tree_parents || !cand_tokens)) return RESISPEC_E_ARG;
+  int dev = 0;
+  DeviceInfo info;
+  st = query_device(&dev, &info);
+  if (st) return st;
+  if (info.major != 10 || info.minor != 3) {
+    snprintf(g_last_error, sizeof g_last_error, "device is sm_%d%d, library is built for sm_103a",
+             info.major, info.minor);
+    return RESISPEC_E_UNSUPPORTED;
+  }
+  Plan pl;
+  st = make_plan(dims, o, info.sms, target_logits, draft_logits, &pl);
+  if (st) return st;
+  if ((int64_t)dims.batch * pl.C > 0x7fffffffLL) return RESISPEC_E_SHAPE;
+
+  rs::VerifyParams prm;
+  memset(&prm, 0, sizeof prm);
+  prm.zt = target_logits;
+  prm.zd = draft_logits;
+  prm.parents = tree_parents;
+  prm.cand = cand_tokens;
+  prm.out_tokens = out_tokens;
+  prm.out_len = out_accept_len;
+  prm.out_nodes = o.out_nodes;
+  prm.out_dist = o.out_dist;
+  prm.out_rejects = o.out_rejects;
+  prm.status = o.status;
+  prm.seq_stride = o.seq_stride < 0 ? (int64_t)(dims.num_nodes + 1) * dims.vocab : o.seq_stride;
+  prm.seed = seed;
+  prm.scale_log2 = (float)(1.4426950408889634 / (double)temperature);
+  prm.B = dims.batch;
+  prm.N = dims.num_nodes;
+  prm.V = dims.vocab;
+  prm.D = dims.max_depth;
+  prm.slice = pl.L;
+  prm.npad = pl.npad;
+  prm.mode = o.mode;
+  prm.use_tma = pl.use_tma;
+
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  cudaError_t e;
+  const bool bf16 = dims.dtype == RESISPEC_BF16;
+  if (pl.threads == 512)
+    e = bf16 ? launch_verify<512, true>(pl, prm, s, dev) : launch_verify<512, false>(pl, prm, s, dev);
+  else
+    e = bf16 ? launch_verify<256, true>(pl, prm, s, dev) : launch_verify<256, false>(pl, prm, s, dev);
+  if (e != cudaSuccess) {
+    set_error("verify launch", e);
+    return RESISPEC_E_CUDA;
+  }
+  return RESISPEC_OK;
+}
+
+int resispec_verify(const void* target_logits, const void* draft_logits,
+                    const int32_t* tree_parents, const int32_t* cand_tokens, float temperature,
+                    uint64_t seed, int32_t* out_tokens, int32_t* out_accept_len,
+                    resispec_dims dims, void* stream) {
+  return resispec_verify_ex(target_logits, draft_logits, tree_parents, cand_tokens, temperature,
+                            seed, out_tokens, out_accept_len, dims, nullptr, stream);
+}
+
+int resispec_uniforms(uint64_t seed, const int32_t* seq, const int32_t* row, int32_t n,
+                      float* u0, float* u1, void* stream) {
+  if (n < 0) return RESISPEC_E_SHAPE;
+  if (n == 0) return RESISPEC_OK;
+  if (!seq || !row || !u0 || !u1) return RESISPEC_E_ARG;
+  const int threads = 256;
+  rs::uniforms_kernel<<<(n + threads - 1) / threads, threads, 0,
+                        static_cast<cudaStream_t>(stream)>>>(seed, seq, row, n, u0, u1);
+  const cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) {
+    set_error("uniforms launch", e);
+    return RESISPEC_E_CUDA;
+  }
+  return RESISPEC_OK;
+}
+
+}  // extern "C"

@@ -174,8 +174,9 @@ def logits_np(rng: np.random.Generator, rows: int, V: int, gen: str, scale: floa
     """(z_t, z_d) float32 arrays of shape [rows, V]."""
     zt = scale * rng.standard_normal((rows, V))
     if gen == "zipf":
-        rank = np.argsort(rng.random((rows, V)), axis=1) + 1
-        zt = zt - slope * np.log(rank.astype(np.float64))
+        rank = rng.permuted(np.broadcast_to(np.arange(1, V + 1, dtype=np.float64), (rows, V)),
+                            axis=1)
+        zt = zt - slope * np.log(rank)
     elif gen != "gauss":
         raise ValueError(gen)
     zd = rho * zt + math.sqrt(max(0.0, 1.0 - rho * rho)) * scale * rng.standard_normal((rows, V))

@@ -1,0 +1,113 @@
+"""Helpers shared by the GPU parity tests: run the CUDA path and the fp64
+oracle on the same seeded inputs and compare them.
+
+Parity rule (the tolerances of the verification hot path):
+  * a sequence is "near tie" when the oracle saw an accept test with
+    |u - R(x)/q(x)| <= 1e-5 or a final draw whose relative CDF margin is
+    <= 1e-6; near-tie sequences are counted, not compared;
+  * every other sequence: accepted tokens, accept length, accepted node ids,
+    rejection count and the final token are bit-exact;
+  * the distribution of the final draw agrees within 1e-6 max-abs and 1e-5
+    L1 per row, and the GPU row sums to 1 within 1e-6.
+    SpecInfer residuals are the one exception: each rejection divides
+    (R - q)_+ by its mass S_j, so an fp32 rounding of p or q (about 1e-7
+    relative, the floor of any fp32 normaliser) reaches the residual
+    multiplied by 1 / prod_j S_j.  Their rows use the same bounds scaled by
+    that factor, which the oracle reports per row ("cond"; 1 in every other
+    case).
+"""
+import numpy as np
+
+import oracle
+import paper_2608_24411_gb300 as rs
+
+ACCEPT_TIE = 1e-5
+SAMPLE_TIE = 1e-6
+DIST_MAXABS = 1e-6
+DIST_L1 = 1e-5
+
+
+def to_host_logits(t):
+    """torch tensor (float32 or bfloat16) -> numpy array the oracle accepts."""
+    import torch
+    if t.dtype == torch.bfloat16:
+        return t.contiguous().view(torch.int16).cpu().numpy().view(np.uint16)
+    return t.contiguous().cpu().numpy()
+
+
+def to_device(arr, device="cuda"):
+    import torch
+    if arr.dtype == np.uint16:
+        return torch.from_numpy(arr.view(np.int16)).to(device).view(torch.bfloat16)
+    return torch.from_numpy(np.ascontiguousarray(arr)).to(device)
+
+
+def run_gpu(target, draft, parents, cand, T, seed, max_depth, mode=rs.MODE_RESISPEC,
+            want_dist=True, **kw):
+    """target/draft/parents/cand: torch CUDA tensors."""
+    import torch
+    B = cand.shape[0]
+    V = target.shape[-1]
+    dev = target.device
+    out = {
+        "nodes": torch.full((B, max(max_depth, 1)), -7, dtype=torch.int32, device=dev),
+        "rejects": torch.full((B,), -7, dtype=torch.int32, device=dev),
+        "status": torch.zeros((1,), dtype=torch.int32, device=dev),
+    }
+    if want_dist:
+        out["dist"] = torch.full((B, V), -1.0, dtype=torch.float32, device=dev)
+    toks, alen = rs.verify(target, draft, parents, cand, T, seed, max_depth=max_depth,
+                           mode=mode, out_nodes=out["nodes"], out_dist=out.get("dist"),
+                           out_rejects=out["rejects"], status=out["status"], **kw)
+    torch.cuda.synchronize()
+    res = {k: v.cpu().numpy() for k, v in out.items()}
+    res["tokens"] = toks.cpu().numpy()
+    res["accept_len"] = alen.cpu().numpy()
+    res["nodes"] = res["nodes"][:, :max_depth]
+    return res
+
+
+def run_oracle(target_h, draft_h, parents_h, cand_h, T, seed, max_depth, mode, seq_ids=None,
+               want_dist=True, seq_stride=None):
+    return oracle.verify(target_h, draft_h, parents_h, cand_h, T, seed, mode=mode,
+                         max_depth=max_depth, seq_ids=seq_ids, want_dist=want_dist,
+                         seq_stride=seq_stride)
+
+
+def compare(g, o, rows=None, check_dist=True):
+    """Compare GPU outputs g (rows `rows` of the batch, or all) with oracle
+    outputs o.  Returns (n_compared, n_near_tie)."""
+    idx = np.arange(len(o["accept_len"])) if rows is None else np.asarray(rows)
+    sel = lambda a: a[idx]
+    near = (o["accept_margin"] <= ACCEPT_TIE) | (o["sample_margin"] <= SAMPLE_TIE)
+    errs = (o["status"] & ~oracle.INFO_DEGENERATE) != 0
+    clean = ~near
+    gl, ol = sel(g["accept_len"]), o["accept_len"]
+    bad = np.nonzero(clean & (gl != ol))[0]
+    assert bad.size == 0, f"accept_len differs at {bad[:10]}: gpu {gl[bad[:10]]} oracle {ol[bad[:10]]}"
+    gt, ot = sel(g["tokens"]), o["tokens"]
+    bad = np.nonzero(clean & (gt != ot).any(axis=1))[0]
+    assert bad.size == 0, f"tokens differ at {bad[:5]}: gpu {gt[bad[:5]]} oracle {ot[bad[:5]]}"
+    if "nodes" in g and o["nodes"].shape[1]:
+        gn = sel(g["nodes"])[:, : o["nodes"].shape[1]]
+        bad = np.nonzero(clean & (gn != o["nodes"]).any(axis=1))[0]
+        assert bad.size == 0, f"nodes differ at {bad[:5]}"
+    if "rejects" in g:
+        gr = sel(g["rejects"])
+        ok = clean & ~errs
+        bad = np.nonzero(ok & (gr != o["rejects"]))[0]
+        assert bad.size == 0, f"rejects differ at {bad[:5]}: {gr[bad[:5]]} vs {o['rejects'][bad[:5]]}"
+    if check_dist and "dist" in g and "dist" in o:
+        gd = sel(g["dist"]).astype(np.float64)
+        ok = clean & ~errs
+        if ok.any():
+            diff = np.abs(gd[ok] - o["dist"][ok])
+            scale = np.maximum(1.0, o["cond"][ok])
+            worst = (diff.max(axis=1) / scale).max()
+            assert worst <= DIST_MAXABS, f"dist max-abs {worst:.3e} (scaled by cond)"
+            l1 = diff.sum(axis=1) / scale
+            assert l1.max() <= DIST_L1, f"dist L1 {l1.max():.3e}"
+            sums = gd[ok].sum(axis=1)
+            assert np.abs(sums - 1).max() <= 1e-6, f"residual sum off by {np.abs(sums - 1).max():.3e}"
+            assert (gd[ok] >= 0).all()
+    return int(clean.sum()), int(near.sum())

@@ -1,0 +1,103 @@
+"""The C ABI without a GPU: the library builds and loads, exports every
+function include/resispec.h declares, and rejects bad arguments
+synchronously (before any device work)."""
+import ctypes
+import os
+import re
+
+import pytest
+
+import paper_2608_24411_gb300 as rs
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "resispec.h")
+
+
+@pytest.fixture(scope="module")
+def lib():
+    rs.build()
+    return rs.load_library()
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    names = re.findall(r"^\s*(?:const\s+)?[a-z_0-9]+\s*\*?\s*(resispec_[a-z_0-9]+)\s*\(", text,
+                       flags=re.M)
+    return sorted(set(names))
+
+
+def test_header_declares_entry_points():
+    names = declared_functions()
+    for n in ("resispec_verify", "resispec_verify_ex", "resispec_plan", "resispec_uniforms",
+              "resispec_opts_default", "resispec_status_string", "resispec_last_error",
+              "resispec_abi_version"):
+        assert n in names
+
+
+def test_library_exports_every_declared_symbol(lib):
+    for n in declared_functions():
+        assert hasattr(lib, n), n
+    assert set(rs.EXPORTED) <= set(declared_functions())
+    assert lib.resispec_abi_version() == 1
+
+
+def test_opts_default_layout(lib):
+    o = rs.Opts()
+    ctypes.memset(ctypes.byref(o), 0x5A, ctypes.sizeof(o))
+    lib.resispec_opts_default(ctypes.byref(o))
+    assert o.mode == 0 and o.cluster_size == 0 and o.block_threads == 0 and o.flags == 0
+    assert o.seq_stride == -1
+    assert not o.status and not o.out_nodes and not o.out_dist and not o.out_rejects
+
+
+def _call(lib, dims, T=1.0, null=False, opts=None):
+    p = None if null else ctypes.c_void_p(16)
+    return lib.resispec_verify_ex(p, p, p, p, ctypes.c_float(T), 0, p, p, dims,
+                                  ctypes.byref(opts) if opts else None, None)
+
+
+def test_synchronous_argument_errors(lib):
+    D = rs.Dims
+    assert _call(lib, D(1, 2, 10, 1, rs.F32), T=0.0) == rs.E_ARG
+    assert _call(lib, D(1, 2, 10, 1, rs.F32), T=-1.0) == rs.E_ARG
+    assert _call(lib, D(1, 2, 10, 1, rs.F32), T=float("nan")) == rs.E_ARG
+    assert _call(lib, D(1, 2, 10, 1, rs.F32), T=float("inf")) == rs.E_ARG
+    assert _call(lib, D(1, 2, 0, 1, rs.F32)) == rs.E_SHAPE
+    assert _call(lib, D(1, 2, rs.MAX_VOCAB + 1, 1, rs.F32)) == rs.E_SHAPE
+    assert _call(lib, D(-1, 2, 10, 1, rs.F32)) == rs.E_SHAPE
+    assert _call(lib, D(1, rs.MAX_NODES + 1, 10, 1, rs.F32)) == rs.E_SHAPE
+    assert _call(lib, D(1, 2, 10, 3, rs.F32)) == rs.E_SHAPE      # depth > nodes
+    assert _call(lib, D(1, 2, 10, 1, 7)) == rs.E_DTYPE
+    assert _call(lib, D(1, 2, 10, 1, rs.F32), null=True) == rs.E_ARG
+    assert _call(lib, D(0, 2, 10, 1, rs.F32), null=True) == rs.E_OK   # empty batch: no launch
+
+
+def test_plan_without_device(lib):
+    p = rs.plan(64, 62, 151936, 5, "f32")
+    assert p["cluster_size"] in (8, 16)
+    assert p["slice_elems"] % 8 == 0
+    assert p["slice_elems"] * p["cluster_size"] >= 151936
+    assert p["smem_bytes"] <= 227 * 1024
+    assert p["uses_tma"] == 1
+    p = rs.plan(1, 12, 64, 4, "f32", cluster_size=1)
+    assert p["cluster_size"] == 1 and p["slice_elems"] == 64
+    p = rs.plan(1, 12, 61, 4, "f32", cluster_size=2)
+    assert p["uses_tma"] == 0                      # 61 * 4 bytes per row: not 16-byte aligned
+    p = rs.plan(1, 12, 64, 4, "bf16", no_tma=True)
+    assert p["uses_tma"] == 0
+    for V in (1, 7, 32000, 128256, 256000, rs.MAX_VOCAB):
+        p = rs.plan(128, 488, V, 6, "bf16")
+        assert p["smem_bytes"] <= 227 * 1024
+    with pytest.raises(rs.ResispecError):
+        rs.plan(1, 2, 10, 1, "f32", cluster_size=3)
+    with pytest.raises(rs.ResispecError):
+        rs.plan(1, 2, rs.MAX_VOCAB, 1, "f32", cluster_size=1)  # 2 MB on one CTA
+
+
+def test_no_cpu_path():
+    torch = pytest.importorskip("torch")
+    t = torch.zeros((1, 2, 8))
+    with pytest.raises(ValueError):
+        rs.verify(t, t, torch.zeros(1, dtype=torch.int32), torch.zeros((1, 1), dtype=torch.int32),
+                  1.0, 0, max_depth=1)

@@ -1,0 +1,325 @@
+"""GPU parity: the CUDA verification path against the fp64 oracle on the
+same seeded inputs, through the C ABI (see tests/parity.py for the rule)."""
+import numpy as np
+import pytest
+from scipy.special import softmax as sp_softmax
+
+import oracle
+import paper_2608_24411_gb300 as rs
+from oracle import enumerator as en
+from paper_2608_24411_gb300 import workloads as W
+from tests import parity as P
+from tests.test_oracle_walk import chisq_pvalue
+
+pytestmark = pytest.mark.gpu
+MODES = [rs.MODE_RESISPEC, rs.MODE_SPECINFER]
+
+
+@pytest.fixture(scope="module", autouse=True)
+def built():
+    rs.build()
+    rs.load_library()
+
+
+def _np_inputs_to_gpu(inp):
+    import torch
+    return (P.to_device(inp["target"]), P.to_device(inp["draft"]),
+            torch.as_tensor(inp["parents"], dtype=torch.int32, device="cuda"),
+            torch.as_tensor(inp["cand"], dtype=torch.int32, device="cuda"))
+
+
+def _check(inp, mode, seed, near_frac=0.01, **kw):
+    zt, zd, pa, ca = _np_inputs_to_gpu(inp)
+    D = int(inp["max_depth"])
+    g = P.run_gpu(zt, zd, pa, ca, inp["temperature"], seed, D, mode=mode, **kw)
+    o = P.run_oracle(inp["target"], inp["draft"], inp["parents"], inp["cand"],
+                     inp["temperature"], seed, D, mode)
+    n, near = P.compare(g, o)
+    assert near <= max(2, near_frac * len(o["accept_len"])), (near, n)
+    assert g["status"][0] & ~rs.INFO_DEGENERATE == 0
+    return g, o
+
+
+def test_device_philox_matches_numpy():
+    import torch
+    from tests.test_oracle_pins import _np_philox_block
+    rng = np.random.default_rng(0)
+    n = 4000
+    seq = rng.integers(0, 1 << 31, n).astype(np.int32)
+    row = rng.integers(0, 1 << 31, n).astype(np.int32)
+    for seed in (0, 1, 2 ** 64 - 1, 0x123456789ABCDEF0):
+        u0, u1 = rs.uniforms(seed, torch.as_tensor(seq, device="cuda"),
+                             torch.as_tensor(row, device="cuda"))
+        u0, u1 = u0.cpu().numpy(), u1.cpu().numpy()
+        for i in range(0, n, 97):
+            blk = _np_philox_block([int(row[i]), int(seq[i]), 0, 0], [seed, 0])
+            assert u0[i] == np.float32((int(blk[0]) >> 40) / 2.0 ** 24)
+            assert u1[i] == np.float32((int(blk[1]) >> 40) / 2.0 ** 24)
+
+
+@pytest.mark.parametrize("mode", MODES)
+@pytest.mark.parametrize("cluster", [0, 1, 16])
+def test_parity_tiny_chain_10000(mode, cluster):
+    """Chain depth 4 with k = 3, V = 64, fp32: 10,000 independent problems
+    from seed 0 (10,000 verify steps) in one batch."""
+    w = W.WORKLOADS["tiny-chain-v64"]
+    inp = W.make_inputs_np(w, seed=0, batch=10_000)
+    _check(inp, mode, seed=0, cluster_size=cluster)
+
+
+@pytest.mark.parametrize("mode", MODES)
+def test_parity_tree60_v32000(mode):
+    w = W.WORKLOADS["tree60-v32000"]
+    inp = W.make_inputs_np(w, seed=1, batch=256)
+    _check(inp, mode, seed=11)
+
+
+def test_parity_tree60_v32000_per_call_seeds():
+    """Batch 1, one call per step with seed = base + step (the paper's seed
+    schedule), launch shape chosen automatically for a single sequence."""
+    w = W.WORKLOADS["tree60-v32000"]
+    for step in range(12):
+        inp = W.make_inputs_np(w, seed=100 + step, batch=1)
+        _check(inp, rs.MODE_RESISPEC, seed=5000 + step)
+
+
+@pytest.mark.parametrize("mode", MODES)
+def test_parity_chain8x4_v128256(mode):
+    w = W.WORKLOADS["chain8x4-v128256-b16"]
+    for step in range(3):
+        inp = W.make_inputs_np(w, seed=20 + step, batch=16)
+        _check(inp, mode, seed=900 + step)
+
+
+@pytest.mark.parametrize("V", [1, 2, 3, 7, 61, 999, 1000, 1003, 4104])
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+@pytest.mark.parametrize("no_tma", [False, True])
+def test_parity_ragged_vocab(V, dtype, no_tma):
+    """Vocabularies that leave ragged slice tails, empty CTAs (V < cluster
+    slices) and rows that are not 16-byte aligned (plain-load path)."""
+    base = W.Workload(name="ragged", batch=64, vocab=V, dtype=dtype, gen="gauss", scale=2.0,
+                      slope=0.0, rho=0.6, temperature=0.9, tree=("levels", (3, 2, 1)), steps=1)
+    inp = W.make_inputs_np(base, seed=V, batch=64)
+    for cluster in (0, 4, 16):
+        for mode in MODES:
+            _check(inp, mode, seed=V + cluster, cluster_size=cluster, no_tma=no_tma)
+
+
+@pytest.mark.parametrize("threads", [256, 512])
+def test_launch_shapes_agree(threads):
+    w = W.WORKLOADS["tree60-v32000"]
+    inp = W.make_inputs_np(w, seed=2, batch=64)
+    ref = None
+    for cluster in (1, 2, 4, 8, 16):
+        g, o = _check(inp, rs.MODE_RESISPEC, seed=3, cluster_size=cluster, block_threads=threads)
+        clean = (o["accept_margin"] > P.ACCEPT_TIE) & (o["sample_margin"] > P.SAMPLE_TIE)
+        if ref is not None:
+            assert (g["tokens"][clean] == ref[clean]).all()
+        ref = g["tokens"]
+
+
+def test_repeat_runs_bit_identical():
+    w = W.WORKLOADS["chain8x4-v128256-b16"]
+    inp = W.make_inputs_np(w, seed=5, batch=16)
+    zt, zd, pa, ca = _np_inputs_to_gpu(inp)
+    a = P.run_gpu(zt, zd, pa, ca, inp["temperature"], 77, inp["max_depth"])
+    b = P.run_gpu(zt, zd, pa, ca, inp["temperature"], 77, inp["max_depth"])
+    for k in ("tokens", "accept_len", "nodes", "rejects", "dist"):
+        np.testing.assert_array_equal(a[k], b[k])
+
+
+def test_empty_tree_and_empty_batch():
+    import torch
+    V = 5000
+    rng = np.random.default_rng(4)
+    zt = rng.normal(0, 3, (40, 1, V)).astype(np.float32)
+    pa = np.zeros(0, np.int32)
+    ca = np.zeros((40, 0), np.int32)
+    g = P.run_gpu(P.to_device(zt), P.to_device(zt), torch.zeros(0, dtype=torch.int32, device="cuda"),
+                  torch.zeros((40, 0), dtype=torch.int32, device="cuda"), 1.0, 8, 0)
+    o = P.run_oracle(zt, zt, pa, ca, 1.0, 8, 0, rs.MODE_RESISPEC)
+    P.compare(g, o)
+    assert (g["accept_len"] == 0).all()
+    e = torch.zeros((0, 1, V), device="cuda")
+    toks, alen = rs.verify(e, e, torch.zeros(0, dtype=torch.int32, device="cuda"),
+                           torch.zeros((0, 0), dtype=torch.int32, device="cuda"), 1.0, 0,
+                           max_depth=0)
+    assert toks.shape == (0, 1) and alen.shape == (0,)
+
+
+def test_shared_rows_seq_stride_zero():
+    import torch
+    w = W.WORKLOADS["tiny-chain-v64"]
+    inp = W.make_inputs_np(w, seed=3, batch=1)
+    B = 3000
+    rng = np.random.default_rng(3)
+    cand = rng.integers(0, 64, (B, w.num_nodes)).astype(np.int32)
+    zt = P.to_device(inp["target"][0])
+    zd = P.to_device(inp["draft"][0])
+    pa = torch.as_tensor(inp["parents"], device="cuda")
+    g = P.run_gpu(zt, zd, pa, torch.as_tensor(cand, device="cuda"), 1.0, 6, w.max_depth,
+                  seq_stride=0)
+    o = P.run_oracle(inp["target"][0], inp["draft"][0], inp["parents"], cand, 1.0, 6,
+                     w.max_depth, rs.MODE_RESISPEC, seq_stride=0)
+    P.compare(g, o)
+
+
+def test_error_contract_matches_oracle():
+    import torch
+    parents = W.tree_levels([2, 2])
+    V, B = 1024, 8
+    rng = np.random.default_rng(1)
+    zt = rng.normal(0, 1, (B, 7, V)).astype(np.float32)
+    zd = zt.copy()
+    cand = rng.integers(0, V, (B, 6)).astype(np.int32)
+    cand[1, 0] = V
+    cand[5, 0] = -3
+    zt[2, 0, 3] = np.nan
+    zt[3, 0, :] = -np.inf
+    zt[4, 6, 0] = np.nan              # never visited
+    zd[6, 0, 100] = np.inf
+    g = P.run_gpu(P.to_device(zt), P.to_device(zd), torch.as_tensor(parents, device="cuda"),
+                  torch.as_tensor(cand, device="cuda"), 1.0, 0, 2, want_dist=False)
+    o = P.run_oracle(zt, zd, parents, cand, 1.0, 0, 2, rs.MODE_RESISPEC, want_dist=False)
+    np.testing.assert_array_equal(g["accept_len"] == -1, o["accept_len"] == -1)
+    assert list(np.nonzero(o["accept_len"] == -1)[0]) == [1, 2, 3, 5, 6]
+    assert (g["tokens"][[1, 2, 3, 5, 6]] == -1).all()
+    want = int(np.bitwise_or.reduce(o["status"]))
+    assert g["status"][0] & ~rs.INFO_DEGENERATE == want & ~oracle.INFO_DEGENERATE
+    # depth overflow and a tree that is not in topological order
+    g = P.run_gpu(P.to_device(zt[:1]), P.to_device(zd[:1]), torch.as_tensor(parents, device="cuda"),
+                  torch.as_tensor(cand[:1], device="cuda"), 1.0, 0, 1, want_dist=False)
+    assert g["accept_len"][0] == -1 and g["status"][0] == rs.ERR_DEPTH
+    bad = torch.as_tensor(np.array([-1, 1, 0, 0, 1, 1], np.int32), device="cuda")
+    g = P.run_gpu(P.to_device(zt[:2]), P.to_device(zd[:2]), bad,
+                  torch.as_tensor(cand[:2], device="cuda"), 1.0, 0, 3, want_dist=False)
+    assert (g["accept_len"] == -1).all() and g["status"][0] == rs.ERR_TREE
+
+
+def test_synchronous_errors_on_device():
+    import torch
+    t = torch.zeros((1, 2, 8), device="cuda")
+    pa = torch.zeros(1, dtype=torch.int32, device="cuda") - 1
+    ca = torch.zeros((1, 1), dtype=torch.int32, device="cuda")
+    with pytest.raises(rs.ResispecError):
+        rs.verify(t, t, pa, ca, 0.0, 0, max_depth=1)
+    with pytest.raises(rs.ResispecError):
+        rs.verify(t, t, pa, ca, 1.0, 0, max_depth=1, cluster_size=3)
+
+
+def test_nondefault_stream():
+    import torch
+    w = W.WORKLOADS["tree60-v32000"]
+    inp = W.make_inputs_np(w, seed=9, batch=32)
+    zt, zd, pa, ca = _np_inputs_to_gpu(inp)
+    s = torch.cuda.Stream()
+    s.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(s):
+        toks, alen = rs.verify(zt, zd, pa, ca, 1.0, 4, max_depth=inp["max_depth"])
+    s.synchronize()
+    o = P.run_oracle(inp["target"], inp["draft"], inp["parents"], inp["cand"], 1.0, 4,
+                     inp["max_depth"], rs.MODE_RESISPEC, want_dist=False)
+    P.compare({"tokens": toks.cpu().numpy(), "accept_len": alen.cpu().numpy()}, o,
+              check_dist=False)
+
+
+# ------------------------------------------------------------ full-size workloads
+
+
+def _sampled_parity(w, seed, call_seed, rows, mode=rs.MODE_RESISPEC, batch=None, rho=None):
+    """Full-size inputs drawn on the GPU; the oracle recomputes the sampled
+    sequences `rows` one by one from the same tensors."""
+    import torch
+    inp = W.make_inputs_torch(w, seed, "cuda", batch=batch, rho=rho)
+    D = inp["max_depth"]
+    g = P.run_gpu(inp["target"], inp["draft"], inp["parents"], inp["cand"], w.temperature,
+                  call_seed, D, mode=mode)
+    ridx = torch.as_tensor(rows, device="cuda")
+    th = P.to_host_logits(inp["target"].index_select(0, ridx))
+    dh = P.to_host_logits(inp["draft"].index_select(0, ridx))
+    ch = inp["cand"].index_select(0, ridx).cpu().numpy()
+    o = P.run_oracle(th, dh, inp["parents_np"], ch, w.temperature, call_seed, D, mode,
+                     seq_ids=np.asarray(rows, np.int32))
+    n, near = P.compare(g, o, rows=rows)
+    assert near <= 1
+    assert g["status"][0] & ~rs.INFO_DEGENERATE == 0
+    assert (g["accept_len"] >= 0).all()
+    del inp
+    torch.cuda.empty_cache()
+    return g
+
+
+@pytest.mark.parametrize("rho", [0.5, 0.8, 0.95])
+def test_parity_binary5_v151936_full_size(rho):
+    """B = 64, V = 151936 fp32, full binary tree of depth 5, in the launch
+    shape the benchmark times; 8 sampled sequences per call checked."""
+    w = W.WORKLOADS["binary5-v151936-b64"]
+    _sampled_parity(w, seed=31, call_seed=1000, rows=[0, 9, 17, 26, 35, 44, 53, 63], rho=rho)
+
+
+def test_parity_binary5_specinfer_full_size():
+    w = W.WORKLOADS["binary5-v151936-b64"]
+    _sampled_parity(w, seed=32, call_seed=1001, rows=[1, 20, 40, 62], mode=rs.MODE_SPECINFER)
+
+
+@pytest.mark.parametrize("k", [2, 16])
+def test_parity_single_position_v256000(k):
+    w = W.WORKLOADS[f"single-k{k}-v256000-b32"]
+    _sampled_parity(w, seed=40 + k, call_seed=77, rows=[0, 7, 15, 31])
+
+
+def test_parity_tree488_v256000():
+    w = W.WORKLOADS["tree488-v256000-b32"]
+    _sampled_parity(w, seed=50, call_seed=78, rows=[0, 5], batch=6)
+
+
+# ------------------------------------------------------------ exactness on the GPU
+
+
+def test_gpu_specinfer_million_draws_v32000():
+    """SpecInfer mode is distribution-exact: 1e6 GPU draws at V = 32000 (one
+    shared set of rows, fresh candidates per draw) do not reject p."""
+    import torch
+    V, k, n = 32000, 4, 1_000_000
+    w = W.WORKLOADS["tree60-v32000"]
+    rng = np.random.default_rng(12)
+    zt, zd = W.logits_np(rng, 1, V, "zipf", w.scale, w.slope, w.rho)
+    zt_b, zd_b = W.f32_to_bf16_bits(zt[0]), W.f32_to_bf16_bits(zd[0])
+    rows_t = np.ascontiguousarray(np.broadcast_to(zt_b, (k + 1, V)))
+    rows_d = np.ascontiguousarray(np.broadcast_to(zd_b, (k + 1, V)))
+    q = torch.softmax(torch.as_tensor(W.bf16_bits_to_f32(zd_b), dtype=torch.float64,
+                                      device="cuda"), dim=0)
+    gen = torch.Generator(device="cuda")
+    gen.manual_seed(3)
+    cand = torch.multinomial(q, n * k, replacement=True, generator=gen).to(torch.int32)
+    cand = cand.view(n, k).contiguous()
+    toks, alen = rs.verify(P.to_device(rows_t), P.to_device(rows_d),
+                           torch.full((k,), -1, dtype=torch.int32, device="cuda"), cand, 1.0,
+                           2024, max_depth=1, mode=rs.MODE_SPECINFER, seq_stride=0)
+    first = toks[:, 0].to(torch.int64)
+    assert int(first.min()) >= 0
+    counts = torch.bincount(first, minlength=V).cpu().numpy()
+    p = sp_softmax(W.bf16_bits_to_f32(zt_b).astype(np.float64))
+    pv, nb = chisq_pvalue(counts, p)
+    assert pv > 1e-4, (pv, nb)
+
+
+def test_gpu_resispec_million_draws_vs_enumerator():
+    """ResiSpec mode on the GPU follows the enumerated law of Algorithm 1
+    (and not p: the documented bias)."""
+    import torch
+    V, k, n = 16, 3, 1_000_000
+    rng = np.random.default_rng(5)
+    zt = (2.0 * rng.standard_normal(V)).astype(np.float32)
+    zd = (0.8 * zt + 1.2 * rng.standard_normal(V)).astype(np.float32)
+    p, q = sp_softmax(zt.astype(np.float64)), sp_softmax(zd.astype(np.float64))
+    cand = rng.choice(V, size=(n, k), p=q).astype(np.int32)
+    toks, _ = rs.verify(P.to_device(np.broadcast_to(zt, (k + 1, V)).copy()),
+                        P.to_device(np.broadcast_to(zd, (k + 1, V)).copy()),
+                        torch.full((k,), -1, dtype=torch.int32, device="cuda"),
+                        torch.as_tensor(cand, device="cuda"), 1.0, 99, max_depth=1,
+                        seq_stride=0)
+    counts = np.bincount(toks[:, 0].cpu().numpy(), minlength=V)
+    dist, _ = en.single_position(p, q, k, en.MODE_RESISPEC)
+    assert chisq_pvalue(counts, dist)[0] > 1e-4
+    assert chisq_pvalue(counts, p)[0] < 1e-12

@@ -48,6 +48,7 @@ def parse_args(argv=None):
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", default="binary5-v151936-b64")
     ap.add_argument("--rho", type=float, default=None)
+    ap.add_argument("--batch", type=int, default=None, help="override the workload's batch")
     ap.add_argument("--mode", choices=["resispec", "specinfer"], default="resispec")
     ap.add_argument("--pool", type=int, default=0, help="input sets rotated between steps (0 = auto)")
     ap.add_argument("--cluster-size", type=int, default=0)
@@ -283,11 +284,11 @@ def run_ours(args):
     if args.rho is not None:
         w = W.with_rho(w, args.rho)
     mode = rs.MODE_SPECINFER if args.mode == "specinfer" else rs.MODE_RESISPEC
-    B, N, V, D = w.batch, w.num_nodes, w.vocab, w.max_depth
+    B, N, V, D = (args.batch or w.batch), w.num_nodes, w.vocab, w.max_depth
     es = w.elem_bytes
     set_bytes = 2 * B * (N + 1) * V * es
     pool = args.pool or max(2, min(8, math.ceil(4 * L2_BYTES / max(1, 2 * B * V * es))))
-    sets = [W.make_inputs_torch(w, seed=args.seed + 7919 * rank + 31 * i, device=dev)
+    sets = [W.make_inputs_torch(w, seed=args.seed + 7919 * rank + 31 * i, device=dev, batch=B)
             for i in range(pool)]
     parents_np = w.parents
     haschild = np.zeros(N + 1, dtype=bool)
@@ -355,7 +356,7 @@ def run_ours(args):
         "warmup": Wm, "ms_per_step": elapsed_ms / K, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": w.dtype, "data": "synthetic",
         "config": {
-            "workload": w.name, "batch": B, "vocab": V, "nodes_per_seq": N, "max_depth": D,
+            "workload": w.name if B == w.batch else f"{w.name}@batch{B}", "batch": B, "vocab": V, "nodes_per_seq": N, "max_depth": D,
             "tree": list(w.tree[1]) if w.tree[0] == "levels" else list(w.tree[1:]),
             "logits": f"{w.gen} slope {w.slope} scale {w.scale} rho {w.rho}",
             "temperature": w.temperature, "mode": args.mode,
@@ -438,8 +439,8 @@ def _finish_cpu(result, args, sets, w, mode, world, dev):
         return result
     import torch
     import oracle
-    S = max(1, min(args.cpu_seqs, w.batch))
     s0 = sets[0]
+    S = max(1, min(args.cpu_seqs, int(s0["cand"].shape[0])))
     idx = torch.arange(S, device=dev)
     th = _host_logits(s0["target"].index_select(0, idx))
     dh = _host_logits(s0["draft"].index_select(0, idx))

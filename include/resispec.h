@@ -82,11 +82,13 @@ typedef struct {
   int32_t dtype;     /* resispec_dtype of both logit arrays */
 } resispec_dims;
 
-#define RESISPEC_FLAG_NO_TMA 1 /* force plain loads instead of bulk copies */
+#define RESISPEC_FLAG_NO_TMA 1   /* force plain loads instead of bulk copies */
+#define RESISPEC_FLAG_PREFETCH 2 /* warm L2 with the first child's rows during a visit */
 
 typedef struct {
   int32_t mode;          /* resispec_mode */
-  int32_t cluster_size;  /* CTAs per sequence: 0 = automatic, else 1, 2, 4, 8, 16 */
+  int32_t cluster_size;  /* CTAs per sequence (one thread-block cluster): 0 = automatic
+                            (most SMs engaged for this batch), else 1 .. 16 */
   int32_t block_threads; /* 0 = automatic, else 256 or 512 */
   int32_t flags;         /* RESISPEC_FLAG_* */
   int64_t seq_stride;    /* elements between sequences in both logit arrays;

@@ -33,6 +33,7 @@ ERR_DEPTH = 16
 ERR_TIMEOUT = 32
 INFO_DEGENERATE = 256
 FLAG_NO_TMA = 1
+FLAG_PREFETCH = 2
 
 MAX_VOCAB = 262144
 MAX_NODES = 4096
@@ -143,14 +144,14 @@ def _ptr(t):
 
 def make_opts(mode=MODE_RESISPEC, cluster_size=0, block_threads=0, no_tma=False,
               seq_stride=None, status=None, out_nodes=None, out_dist=None,
-              out_rejects=None) -> Opts:
+              out_rejects=None, prefetch=False) -> Opts:
     lib = load_library()
     o = Opts()
     lib.resispec_opts_default(ctypes.byref(o))
     o.mode = {"resispec": MODE_RESISPEC, "specinfer": MODE_SPECINFER}.get(mode, mode)
     o.cluster_size = int(cluster_size)
     o.block_threads = int(block_threads)
-    o.flags = FLAG_NO_TMA if no_tma else 0
+    o.flags = (FLAG_NO_TMA if no_tma else 0) | (FLAG_PREFETCH if prefetch else 0)
     o.seq_stride = -1 if seq_stride is None else int(seq_stride)
     o.status = None if status is None else status.data_ptr()
     o.out_nodes = None if out_nodes is None else out_nodes.data_ptr()
@@ -176,7 +177,7 @@ def plan(batch, num_nodes, vocab, max_depth, dtype="f32", **opt_kw) -> dict:
 def verify(target, draft, tree_parents, cand_tokens, temperature, seed, *, max_depth=None,
            mode=MODE_RESISPEC, out_tokens=None, out_accept_len=None, out_nodes=None,
            out_dist=None, out_rejects=None, status=None, cluster_size=0, block_threads=0,
-           no_tma=False, seq_stride=None, stream=None):
+           no_tma=False, seq_stride=None, stream=None, prefetch=False):
     """Verify a batch of draft trees on the GPU.
 
     target, draft: CUDA tensors [B, N+1, V] (float32 or bfloat16); with
@@ -215,7 +216,7 @@ def verify(target, draft, tree_parents, cand_tokens, temperature, seed, *, max_d
     if seq_stride is None and target.numel() != B * (N + 1) * V:
         raise ValueError("target must be [B, N+1, V] (or pass seq_stride)")
     o = make_opts(mode, cluster_size, block_threads, no_tma, seq_stride, status, out_nodes,
-                  out_dist, out_rejects)
+                  out_dist, out_rejects, prefetch)
     if stream is None:
         stream = torch.cuda.current_stream(dev)
     handle = stream.cuda_stream if hasattr(stream, "cuda_stream") else int(stream)

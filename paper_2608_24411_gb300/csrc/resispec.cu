@@ -7,7 +7,9 @@
 #include <stdio.h>
 #include <string.h>
 
+#include <map>
 #include <mutex>
+#include <tuple>
 
 #include "../../include/resispec.h"
 #include "verify_kernel.cuh"
@@ -37,8 +39,11 @@ int round_up(int x, int m) { return (x + m - 1) / m * m; }
 
 int slice_for(int V, int C) { return round_up((V + C - 1) / C, 8); }
 
+// Head, two fp32 rows, then the tree: parent / first child / next sibling
+// (int16), the candidate tokens of the sequence (int32) and two uniforms per
+// logit row (fp32).
 int smem_for(int L, int npad) {
-  const int tree = npad * 2 + npad * 2 + npad * 4 + (npad + 16);
+  const int tree = npad * 2 + (npad + 16) * 2 + npad * 2 + npad * 4 + npad * 8;
   return round_up(rs::kHeadBytes + 8 * L + tree, 128);
 }
 
@@ -83,27 +88,93 @@ int check_dims(const resispec_dims& d) {
   return RESISPEC_OK;
 }
 
-// Launch shape.  sms = 0 means unknown (no device query): the batch-fill
-// rule is skipped.
-int make_plan(const resispec_dims& d, const resispec_opts& o, int sms, const void* zt,
-              const void* zd, Plan* p) {
+// Clusters of this shape that can be resident at once (0: the shape cannot
+// be launched).  Cached per device and shape.
+using OccKey = std::tuple<int, int, int, int, int>;  // dev, threads, bf16, C, smem
+std::map<OccKey, int> g_occ;
+
+template <int THREADS, bool BF16>
+int query_clusters(int C, int smem) {
+  auto kern = rs::verify_kernel<THREADS, BF16>;
+  if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, kMaxSmem) !=
+          cudaSuccess ||
+      cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) !=
+          cudaSuccess) {
+    cudaGetLastError();
+    return 0;
+  }
+  cudaLaunchConfig_t cfg;
+  memset(&cfg, 0, sizeof cfg);
+  cfg.gridDim = dim3((unsigned)(C * 64), 1, 1);
+  cfg.blockDim = dim3(THREADS, 1, 1);
+  cfg.dynamicSmemBytes = (size_t)smem;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = (unsigned)C;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  int n = 0;
+  if (cudaOccupancyMaxActiveClusters(&n, (void*)kern, &cfg) != cudaSuccess) {
+    cudaGetLastError();
+    return 0;
+  }
+  return n;
+}
+
+int active_clusters(int dev, int threads, bool bf16, int C, int smem) {
+  const OccKey key{dev, threads, bf16 ? 1 : 0, C, smem};
+  {
+    std::lock_guard<std::mutex> lk(g_mu);
+    auto it = g_occ.find(key);
+    if (it != g_occ.end()) return it->second;
+  }
+  int n;
+  if (threads == 512)
+    n = bf16 ? query_clusters<512, true>(C, smem) : query_clusters<512, false>(C, smem);
+  else
+    n = bf16 ? query_clusters<256, true>(C, smem) : query_clusters<256, false>(C, smem);
+  std::lock_guard<std::mutex> lk(g_mu);
+  g_occ[key] = n;
+  return n;
+}
+
+// Launch shape.  dev < 0 means no device to query: the automatic cluster
+// size then follows a size-only rule.
+int make_plan(const resispec_dims& d, const resispec_opts& o, int dev, int sms,
+              const void* zt, const void* zd, Plan* p) {
   int st = check_dims(d);
   if (st) return st;
   if (o.mode != RESISPEC_MODE_RESISPEC && o.mode != RESISPEC_MODE_SPECINFER) return RESISPEC_E_ARG;
   if (o.block_threads != 0 && o.block_threads != 256 && o.block_threads != 512)
     return RESISPEC_E_ARG;
   const int cs = o.cluster_size;
-  if (cs != 0 && cs != 1 && cs != 2 && cs != 4 && cs != 8 && cs != 16) return RESISPEC_E_ARG;
+  if (cs < 0 || cs > rs::kMaxCluster) return RESISPEC_E_ARG;
   if (o.seq_stride < -1) return RESISPEC_E_ARG;
   p->threads = o.block_threads ? o.block_threads : 512;
   p->npad = round_up(d.num_nodes + 1, 16);
   const int V = d.vocab;
   if (cs) {
     p->C = cs;
+  } else if (dev >= 0) {
+    // Most SMs engaged: resident clusters (capped by the batch) times their
+    // size; ties go to the larger cluster (shorter per-sequence latency).
+    int best = 0;
+    int64_t best_score = -1;
+    for (int C = 1; C <= rs::kMaxCluster; ++C) {
+      const int smem = smem_for(slice_for(V, C), p->npad);
+      if (smem > kMaxSmem) continue;
+      const int n = active_clusters(dev, p->threads, d.dtype == RESISPEC_BF16, C, smem);
+      if (n <= 0) continue;
+      const int64_t score = std::min<int64_t>(d.batch, n) * C;
+      if (score >= best_score) { best_score = score; best = C; }
+    }
+    if (best == 0) return RESISPEC_E_UNSUPPORTED;
+    p->C = best;
   } else {
     int C = 1;
     while (C < 16 && 8 * slice_for(V, C) > kAutoSliceBytes) C *= 2;
-    // small batches: spread each sequence over more SMs to cut latency
     while (sms > 0 && C < 16 && (int64_t)d.batch * C * 2 <= sms) C *= 2;
     p->C = C;
   }
@@ -183,15 +254,18 @@ int resispec_plan(resispec_dims dims, const resispec_opts* opts, int32_t* cluste
   resispec_opts_default(&o);
   if (opts) o = *opts;
   int sms = 0;
-  int dev = 0;
+  int dev = -1;
   DeviceInfo info;
   int ndev = 0;
-  if (cudaGetDeviceCount(&ndev) == cudaSuccess && ndev > 0 && query_device(&dev, &info) == 0)
+  if (cudaGetDeviceCount(&ndev) == cudaSuccess && ndev > 0 && query_device(&dev, &info) == 0 &&
+      info.major == 10 && info.minor == 3) {
     sms = info.sms;
-  else
+  } else {
+    dev = -1;
     cudaGetLastError();  // clear a sticky "no device" error
+  }
   Plan p;
-  const int st = make_plan(dims, o, sms, nullptr, nullptr, &p);
+  const int st = make_plan(dims, o, dev, sms, nullptr, nullptr, &p);
   if (st) return st;
   if (cluster_size) *cluster_size = p.C;
   if (block_threads) *block_threads = p.threads;
@@ -225,7 +299,7 @@ int resispec_verify_ex(const void* target_logits, const void* draft_logits,
     return RESISPEC_E_UNSUPPORTED;
   }
   Plan pl;
-  st = make_plan(dims, o, info.sms, target_logits, draft_logits, &pl);
+  st = make_plan(dims, o, dev, info.sms, target_logits, draft_logits, &pl);
   if (st) return st;
   if ((int64_t)dims.batch * pl.C > 0x7fffffffLL) return RESISPEC_E_SHAPE;
 
@@ -252,6 +326,7 @@ int resispec_verify_ex(const void* target_logits, const void* draft_logits,
   prm.npad = pl.npad;
   prm.mode = o.mode;
   prm.use_tma = pl.use_tma;
+  prm.prefetch = (o.flags & RESISPEC_FLAG_PREFETCH) != 0;
 
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   cudaError_t e;

@@ -2,25 +2,35 @@
 // draft tree (Sec. 3, Algorithm 1, GetProxy).
 //
 // Data layout on chip.  The vocabulary is cut into C contiguous slices of L
-// elements (L % 8 == 0), one per CTA of the cluster.  Each CTA keeps two fp32
-// rows of its slice in shared memory:
-//   W  the target row: raw logits -> exp((z - max) / T) -> the current
-//      residual R, materialised after each rejection pass,
-//   Q  the draft row:  raw logits -> exp((z - max) / T).
-// bf16 rows land (bulk copy) in the upper half of W / Q and are widened in
-// place.  A rejection never leaves the chip: its pass reads W and Q, writes
-// the new residual back to W and produces the two sums the next residual
-// needs; the cluster combines per-CTA sums through distributed shared
-// memory.  The rows of a node are read from HBM exactly once.
+// elements, one per CTA of the cluster.  A slice is a sequence of vectors of
+// VEC elements (4 fp32 or 8 bf16 logits = 16 bytes of input); vector g
+// belongs to thread g % THREADS in every pass, so per-thread constants stay
+// valid across passes.  Each CTA keeps two fp32 rows of its slice in shared
+// memory:
+//   W  target row: exp((z - m_t) / T), then the current residual R,
+//      materialised by every rejection pass,
+//   Q  draft row:  exp((z - m_t) / T),
+// where m_t is a per-thread exponent reference (the first logit maximum the
+// thread saw, raised only when a later logit exceeds it by 64 binary
+// orders).  The rows arrive by bulk copy in chunks of 2 * THREADS vectors,
+// each with its own mbarrier, and are normalised chunk by chunk while later
+// chunks are still in flight; bf16 rows land in the upper half of W / Q and
+// are widened in place.  The rows of a node are read from HBM exactly once.
 //
-// Lazy residual.  After rejection j the kernel knows only scalars
-// (x0, Z, lambda, 1/norm) of the map R_j -> R_{j+1}; the next pass applies it
-// element-wise while it computes the sums of rejection j+1.  The owner CTA of
-// the next candidate publishes that candidate's stored values in the same
-// exchange, so every CTA evaluates the next accept test from bit-identical
-// operands without an extra round trip.
+// Cluster exchanges.  A visit needs one exchange for the normaliser (online
+// max/sum pairs) and one per rejection (two sums).  Each exchange is a push:
+// every CTA stores its partial into every peer's receive slot with st.async
+// and counts bytes on the peer's mbarrier, so no cluster-wide barrier is
+// needed on the hot path.  The owner CTA of the next candidate publishes
+// that candidate's stored values in the same exchange, so every CTA
+// evaluates the next accept test from bit-identical operands.
+//
+// Lazy residual.  After rejection j the kernel holds only scalars
+// (x0, Z, lambda, 1/norm) of the map R_j -> R_{j+1}; the next pass applies
+// it element-wise while it computes the sums of rejection j+1.
 #pragma once
 #include <cuda_bf16.h>
+#include <float.h>
 #include <math.h>
 #include <stdint.h>
 
@@ -37,14 +47,17 @@ constexpr int kErrDepth = 16;
 constexpr int kErrTimeout = 32;
 constexpr int kInfoDegenerate = 256;
 
-// Internal flag bits carried through the max exchange.
+// Internal flag bits carried through exchanges.
 constexpr int kFlagTargetBad = 1;
 constexpr int kFlagDraftBad = 2;
 constexpr int kFlagTimeout = 4;
 
-constexpr uint32_t kSpinLimit = 1u << 22;   // try_wait attempts before giving up
-constexpr uint32_t kCopyChunk = 32768;      // bytes per bulk copy instruction
+constexpr uint32_t kSpinLimit = 1u << 22;  // try_wait attempts before giving up
 constexpr int kMaxCluster = 16;
+constexpr int kMaxChunks = 32;             // bulk-copy chunks per row
+constexpr int kSlotFloats = 12;
+constexpr uint32_t kSlotBytes = 48;
+constexpr float kRebaseLog2 = 64.f;        // exponent headroom before a reference moves
 
 struct VerifyParams {
   const void* zt;
@@ -61,30 +74,31 @@ struct VerifyParams {
   uint64_t seed;
   float scale_log2;    // log2(e) / T
   int32_t B, N, V, D;
-  int32_t slice;       // L, elements per CTA
+  int32_t slice;       // L, elements per CTA (multiple of 8)
   int32_t npad;        // padded node count of the tree arrays
   int32_t mode;        // 0 ResiSpec, 1 SpecInfer
   int32_t use_tma;
+  int32_t prefetch;    // L2 prefetch of the first child's rows
 };
 
 struct __align__(16) Slot {
-  float v[8];  // [0..3] reduced values, [4..5] published point values, [6] flags
-  double d;    // sampler: this CTA's residual mass
-  double pad;
+  float v[kSlotFloats];  // [0..3] partials, [4..7] published values, [8] flags
 };
 
 struct __align__(16) Head {
-  unsigned long long mbar[2];
-  Slot slot[2];
-  float red[32][8];
-  float bc[8];
-  double wsum[32];
-  double cta_tot[kMaxCluster];
-  int wcnt[32];
-  int misc[4];
-  double miscd[4];
+  unsigned long long tbar[2][kMaxChunks];
+  unsigned long long xbar[2];
+  Slot rx[2][kMaxCluster];  // receive slots: [exchange parity][source rank]
+  float wpart[32][4];       // per-warp partials
+  int wflag[32];
+  float pubv[4];            // values published by the owner thread of a token
+  float bc[kSlotFloats];
+  float part[kMaxCluster][4];  // per-CTA partials of the latest exchange
+  unsigned long long seg[32];   // sampler: fixed-point warp-segment masses
+  unsigned long long fixd[2];   // sampler: fixed-point thresholds
+  int misc[8];
 };
-constexpr int kHeadBytes = 2048;
+constexpr int kHeadBytes = 4608;
 static_assert(sizeof(Head) <= kHeadBytes, "head too large");
 
 // ---------------------------------------------------------------- residual map
@@ -93,17 +107,19 @@ enum : int { kScale = 0, kIdent = 1, kResi = 2, kSpec = 3 };
 struct Pending {
   int kind;
   int x0;     // rejected token (kResi)
-  float a;    // scale (kScale) or 1 / norm (kResi, kSpec)
+  float a;    // 1 / norm (kResi, kSpec)
   float Z;    // budget (kResi)
   float lam;  // filled fraction of the capacity (kResi)
 };
 
-// R_{j+1}(x) from the stored R_j(x) = w and q(x) = qq.  Written with
-// explicitly rounded intrinsics so that every caller computes the same bits.
+// R_{j+1}(x) from the stored value w = R_j(x) and q(x) = qq; `sc` is the
+// per-thread normaliser scale used while the map is still p = w * sc.
+// Explicitly rounded intrinsics keep every caller's bits identical.
 template <int KIND>
-__device__ __forceinline__ float apply_map(const Pending& P, float w, float qq, int idx) {
+__device__ __forceinline__ float apply_map(const Pending& P, float w, float qq, int idx,
+                                           float sc) {
   if constexpr (KIND == kScale) {
-    return __fmul_rn(w, P.a);
+    return __fmul_rn(w, sc);
   } else if constexpr (KIND == kIdent) {
     return w;
   } else if constexpr (KIND == kResi) {
@@ -118,178 +134,42 @@ __device__ __forceinline__ float apply_map(const Pending& P, float w, float qq, 
   }
 }
 
-__device__ __forceinline__ float apply_any(const Pending& P, float w, float qq, int idx) {
+__device__ __forceinline__ float apply_any(const Pending& P, float w, float qq, int idx,
+                                           float sc) {
   switch (P.kind) {
-    case kScale: return apply_map<kScale>(P, w, qq, idx);
-    case kIdent: return apply_map<kIdent>(P, w, qq, idx);
-    case kResi: return apply_map<kResi>(P, w, qq, idx);
-    default: return apply_map<kSpec>(P, w, qq, idx);
+    case kScale: return apply_map<kScale>(P, w, qq, idx, sc);
+    case kIdent: return apply_map<kIdent>(P, w, qq, idx, sc);
+    case kResi: return apply_map<kResi>(P, w, qq, idx, sc);
+    default: return apply_map<kSpec>(P, w, qq, idx, sc);
   }
+}
+
+// 2^(m - M) / S for a stored reference m in log2 units (0 when m = -inf).
+__device__ __forceinline__ float ref_scale(float m, float M, float inv) {
+  return m == -INFINITY ? 0.f : __fmul_rn(ex2(__fsub_rn(m, M)), inv);
 }
 
 // ---------------------------------------------------------------- reductions
-__device__ __forceinline__ float warp_sum(float v) {
+__device__ __forceinline__ float warp_max(float v) {
 #pragma unroll
-  for (int o = 16; o; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  for (int o = 16; o; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
   return v;
 }
 
-// CTA reduction then cluster reduction through DSMEM.  v[0], v[1] are
-// max-reduced when max01, otherwise summed; v[2..5] are summed; flags are
-// OR-ed.  Butterfly reductions give bit-identical results in every lane and,
-// because every CTA combines the same per-CTA partials in the same lanes, in
-// every CTA of the cluster.
-template <int NWARPS>
-__device__ __forceinline__ void exchange(Head& H, const float (&v)[6], int flags, bool max01,
-                                         int& par, uint32_t C, float (&out)[6], int& oflags) {
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  float r[6];
+__device__ __forceinline__ float warp_sum(float v) {
 #pragma unroll
-  for (int k = 0; k < 6; ++k) r[k] = v[k];
-  int f = flags;
-#pragma unroll
-  for (int o = 16; o; o >>= 1) {
-#pragma unroll
-    for (int k = 0; k < 6; ++k) {
-      const float x = __shfl_xor_sync(0xffffffffu, r[k], o);
-      r[k] = (max01 && k < 2) ? fmaxf(r[k], x) : r[k] + x;
-    }
-    f |= __shfl_xor_sync(0xffffffffu, f, o);
-  }
-  if (lane == 0) {
-#pragma unroll
-    for (int k = 0; k < 6; ++k) H.red[warp][k] = r[k];
-    H.red[warp][6] = __int_as_float(f);
-  }
-  __syncthreads();
-  if (warp == 0) {
-#pragma unroll
-    for (int k = 0; k < 6; ++k)
-      r[k] = lane < NWARPS ? H.red[lane][k] : ((max01 && k < 2) ? -INFINITY : 0.f);
-    f = lane < NWARPS ? __float_as_int(H.red[lane][6]) : 0;
-#pragma unroll
-    for (int o = 16; o; o >>= 1) {
-#pragma unroll
-      for (int k = 0; k < 6; ++k) {
-        const float x = __shfl_xor_sync(0xffffffffu, r[k], o);
-        r[k] = (max01 && k < 2) ? fmaxf(r[k], x) : r[k] + x;
-      }
-      f |= __shfl_xor_sync(0xffffffffu, f, o);
-    }
-    if (lane == 0) {
-      Slot& s = H.slot[par];
-#pragma unroll
-      for (int k = 0; k < 6; ++k) s.v[k] = r[k];
-      s.v[6] = __int_as_float(f);
-      s.v[7] = 0.f;
-    }
-  }
-  cluster_sync();
-  if (warp == 0) {
-    const float id01 = max01 ? -INFINITY : 0.f;
-    float4 a = make_float4(id01, id01, 0.f, 0.f);
-    float4 b = make_float4(0.f, 0.f, 0.f, 0.f);
-    if (lane < (int)C) {
-      const uint32_t addr = map_to_rank(smem_addr(&H.slot[par]), lane);
-      a = ld_cluster_f4(addr);
-      b = ld_cluster_f4(addr + 16);
-    }
-    r[0] = a.x; r[1] = a.y; r[2] = a.z; r[3] = a.w; r[4] = b.x; r[5] = b.y;
-    f = lane < (int)C ? __float_as_int(b.z) : 0;
-#pragma unroll
-    for (int o = 16; o; o >>= 1) {
-#pragma unroll
-      for (int k = 0; k < 6; ++k) {
-        const float x = __shfl_xor_sync(0xffffffffu, r[k], o);
-        r[k] = (max01 && k < 2) ? fmaxf(r[k], x) : r[k] + x;
-      }
-      f |= __shfl_xor_sync(0xffffffffu, f, o);
-    }
-    if (lane == 0) {
-#pragma unroll
-      for (int k = 0; k < 6; ++k) H.bc[k] = r[k];
-      H.bc[6] = __int_as_float(f);
-    }
-  }
-  __syncthreads();
-#pragma unroll
-  for (int k = 0; k < 6; ++k) out[k] = H.bc[k];
-  oflags = __float_as_int(H.bc[6]);
-  par ^= 1;
+  for (int o = 16; o; o >>= 1) v = __fadd_rn(v, __shfl_xor_sync(0xffffffffu, v, o));
+  return v;
 }
 
-// ---------------------------------------------------------------- tree
-// Children of `node` in ascending index order (children have larger
-// indices than their parent) and their candidate tokens.  Uniform result.
-template <int THREADS>
-__device__ int gather_children(Head& H, const int16_t* par, int16_t* kids, int32_t* kidtok,
-                               int node, int N, const int32_t* cand_b) {
-  constexpr int NW = THREADS / 32;
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  int count = 0;
-  __syncthreads();
-  for (int base = node + 1; base < N; base += THREADS) {
-    const int c = base + (int)threadIdx.x;
-    const bool f = c < N && par[c] == node;
-    const unsigned m = __ballot_sync(0xffffffffu, f);
-    if (lane == 0) H.wcnt[warp] = __popc(m);
-    __syncthreads();
-    int pre = 0, tot = 0;
-#pragma unroll
-    for (int w = 0; w < NW; ++w) {
-      const int x = H.wcnt[w];
-      pre += w < warp ? x : 0;
-      tot += x;
-    }
-    if (f) {
-      const int pos = count + pre + __popc(m & ((1u << lane) - 1u));
-      kids[pos] = (int16_t)c;
-      kidtok[pos] = __ldg(cand_b + c);
-    }
-    count += tot;
-    __syncthreads();
-  }
-  return count;
-}
-
-// ---------------------------------------------------------------- row I/O
-// Starts the copies of this CTA's slice [lo, lo + nloc) of the target row
-// (and of the draft row when need_draft) that begin at element row_base.
-template <int THREADS, bool BF16>
-__device__ __forceinline__ void issue_rows(Head& H, const VerifyParams& P, float* W, float* Q,
-                                           size_t row_base, bool need_draft, int lo, int nloc) {
-  const size_t row_off = row_base + (size_t)lo;
-  const int L = P.slice;
-  // Earlier generic accesses to W / Q must be ordered before the copies.
-  fence_proxy_async_smem();
-  __syncthreads();
-  constexpr uint32_t es = BF16 ? 2u : 4u;
-  if (P.use_tma) {
-    if (threadIdx.x == 0) {
-      const uint32_t bytes = (uint32_t)nloc * es;
-      const uint32_t dst_off = BF16 ? 2u * (uint32_t)L : 0u;
-      for (int which = 0; which < (need_draft ? 2 : 1); ++which) {
-        const uint32_t bar = smem_addr(&H.mbar[which]);
-        const char* src = static_cast<const char*>(which ? P.zd : P.zt) + row_off * es;
-        const uint32_t dst = smem_addr(which ? Q : W) + dst_off;
-        mbar_arrive_expect_tx(bar, bytes);
-        for (uint32_t o = 0; o < bytes; o += kCopyChunk)
-          bulk_g2s(dst + o, src + o, min(kCopyChunk, bytes - o), bar);
-      }
-    }
-  } else {
-    for (int which = 0; which < (need_draft ? 2 : 1); ++which) {
-      float* dst = which ? Q : W;
-      if constexpr (BF16) {
-        const uint16_t* src = static_cast<const uint16_t*>(which ? P.zd : P.zt) + row_off;
-        uint16_t* raw = reinterpret_cast<uint16_t*>(dst) + L;
-        for (int i = threadIdx.x; i < nloc; i += THREADS) raw[i] = __ldg(src + i);
-      } else {
-        const float* src = static_cast<const float*>(which ? P.zd : P.zt) + row_off;
-        for (int i = threadIdx.x; i < nloc; i += THREADS) dst[i] = __ldg(src + i);
-      }
-    }
-  }
+// (reference, sum of 2^(z c - reference)) pairs of a warp, references in
+// log2 units: max first, then each lane rescales its sum to the common
+// reference, then a sum.  Butterflies leave the same bits in every lane.
+__device__ __forceinline__ void warp_pair(float& m, float& s) {
+  const float M = warp_max(m);
+  const float t = (m == -INFINITY) ? 0.f : __fmul_rn(s, ex2(__fsub_rn(m, M)));
+  s = warp_sum(t);
+  m = M;
 }
 
 __device__ __forceinline__ bool wait_bar(uint32_t bar, uint32_t parity) {
@@ -298,314 +178,569 @@ __device__ __forceinline__ bool wait_bar(uint32_t bar, uint32_t parity) {
   return false;
 }
 
-__device__ __forceinline__ bool bad_logit(float x) { return isnan(x) || x == INFINITY; }
-
-__device__ __forceinline__ float bf16_lo(uint32_t w) { return __uint_as_float(w << 16); }
-__device__ __forceinline__ float bf16_hi(uint32_t w) { return __uint_as_float(w & 0xffff0000u); }
-
-// Max over the valid part of the slice of both raw rows, with the
-// non-finite check of the error contract.
-template <int THREADS, bool BF16>
-__device__ __forceinline__ void max_pass(const float* W, const float* Q, int L, int nloc,
-                                         bool need_draft, float& mt, float& md, int& flags) {
-  mt = -INFINITY;
-  md = -INFINITY;
-  for (int which = 0; which < (need_draft ? 2 : 1); ++which) {
-    const float* buf = which ? Q : W;
-    float m = -INFINITY;
-    bool bad = false;
-    if constexpr (BF16) {
-      const uint16_t* raw = reinterpret_cast<const uint16_t*>(buf) + L;
-      for (int i = threadIdx.x * 8; i < nloc; i += THREADS * 8) {
-        const uint4 r = *reinterpret_cast<const uint4*>(raw + i);
-        const uint32_t w[4] = {r.x, r.y, r.z, r.w};
-#pragma unroll
-        for (int k = 0; k < 4; ++k) {
-          const float a = bf16_lo(w[k]), b = bf16_hi(w[k]);
-          if (i + 2 * k < nloc) { bad |= bad_logit(a); m = fmaxf(m, a); }
-          if (i + 2 * k + 1 < nloc) { bad |= bad_logit(b); m = fmaxf(m, b); }
-        }
-      }
+// Two-level reduction of per-thread partials, then an all-to-all push of the
+// CTA partial to every CTA of the cluster and the same reduction over the C
+// received partials.  Every CTA combines identical partials in identical
+// lanes, so all CTAs obtain the same bits.
+//   NORM: (a0, a1) and (a2, a3) are (max, scaled sum) pairs of the target
+//         and draft rows; SUM: a0, a1 are sums (a2, a3 unused).
+//   H.pubv holds the values published by the owner thread of a token (zero
+//   in CTAs without an owner); they travel unreduced and are summed across
+//   CTAs, where exactly one CTA contributes.  flags are OR-ed.
+// out[0..3]: reduced partials, out[4..7]: published values.
+template <int NWARPS, bool NORM>
+__device__ __forceinline__ void exchange(Head& H, float a0, float a1, float a2, float a3,
+                                         int flags, int& xp, uint32_t& xph, uint32_t rank,
+                                         uint32_t C, float (&out)[8], int& oflags) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  if constexpr (NORM) {
+    warp_pair(a0, a1);
+    warp_pair(a2, a3);
+  } else {
+    a0 = warp_sum(a0);
+    a1 = warp_sum(a1);
+  }
+  flags = __reduce_or_sync(0xffffffffu, flags);
+  if (lane == 0) {
+    H.wpart[warp][0] = a0;
+    H.wpart[warp][1] = a1;
+    H.wpart[warp][2] = a2;
+    H.wpart[warp][3] = a3;
+    H.wflag[warp] = flags;
+  }
+  __syncthreads();
+  if (warp == 0) {
+    const float id = NORM ? -INFINITY : 0.f;
+    a0 = lane < NWARPS ? H.wpart[lane][0] : id;
+    a1 = lane < NWARPS ? H.wpart[lane][1] : 0.f;
+    a2 = lane < NWARPS ? H.wpart[lane][2] : id;
+    a3 = lane < NWARPS ? H.wpart[lane][3] : 0.f;
+    int f = lane < NWARPS ? H.wflag[lane] : 0;
+    if constexpr (NORM) {
+      warp_pair(a0, a1);
+      warp_pair(a2, a3);
     } else {
-      for (int i = threadIdx.x * 4; i < nloc; i += THREADS * 4) {
-        const float4 r = *reinterpret_cast<const float4*>(buf + i);
-        const float x[4] = {r.x, r.y, r.z, r.w};
-#pragma unroll
-        for (int k = 0; k < 4; ++k)
-          if (i + k < nloc) { bad |= bad_logit(x[k]); m = fmaxf(m, x[k]); }
-      }
+      a0 = warp_sum(a0);
+      a1 = warp_sum(a1);
     }
-    if (which) { md = m; flags |= bad ? kFlagDraftBad : 0; }
-    else { mt = m; flags |= bad ? kFlagTargetBad : 0; }
+    f = __reduce_or_sync(0xffffffffu, f);
+    const float p0 = H.pubv[0], p1 = H.pubv[1], p2 = H.pubv[2], p3 = H.pubv[3];
+    __syncwarp();
+    if (lane < 4) H.pubv[lane] = 0.f;  // ready for the next publication
+    const int p = xp;
+    if (lane < (int)C) {
+      const uint32_t dst = map_to_rank(smem_addr(&H.rx[p][rank]), lane);
+      const uint32_t bar = map_to_rank(smem_addr(&H.xbar[p]), lane);
+      st_async_v4(dst, __float_as_uint(a0), __float_as_uint(a1), __float_as_uint(a2),
+                  __float_as_uint(a3), bar);
+      st_async_v4(dst + 16, __float_as_uint(p0), __float_as_uint(p1), __float_as_uint(p2),
+                  __float_as_uint(p3), bar);
+      st_async_v4(dst + 32, (uint32_t)f, 0u, 0u, 0u, bar);
+    }
+    if (lane == 0) mbar_arrive_expect_tx(smem_addr(&H.xbar[p]), C * kSlotBytes);
+    const bool ok = __all_sync(0xffffffffu, wait_bar(smem_addr(&H.xbar[p]), (xph >> p) & 1u));
+    xph ^= 1u << p;
+    float q[4] = {0.f, 0.f, 0.f, 0.f};
+    a0 = id; a1 = 0.f; a2 = id; a3 = 0.f; f = 0;
+    if (lane < (int)C) {
+      const Slot& sl = H.rx[p][lane];
+      a0 = sl.v[0]; a1 = sl.v[1]; a2 = sl.v[2]; a3 = sl.v[3];
+      q[0] = sl.v[4]; q[1] = sl.v[5]; q[2] = sl.v[6]; q[3] = sl.v[7];
+      f = __float_as_int(sl.v[8]);
+      H.part[lane][0] = a0; H.part[lane][1] = a1; H.part[lane][2] = a2; H.part[lane][3] = a3;
+    }
+    if constexpr (NORM) {
+      warp_pair(a0, a1);
+      warp_pair(a2, a3);
+    } else {
+      a0 = warp_sum(a0);
+      a1 = warp_sum(a1);
+    }
+#pragma unroll
+    for (int k = 0; k < 4; ++k) q[k] = warp_sum(q[k]);
+    f = __reduce_or_sync(0xffffffffu, f);
+    if (lane == 0) {
+      H.bc[0] = a0; H.bc[1] = a1; H.bc[2] = a2; H.bc[3] = a3;
+      H.bc[4] = q[0]; H.bc[5] = q[1]; H.bc[6] = q[2]; H.bc[7] = q[3];
+      H.bc[8] = __int_as_float(f | (ok ? 0 : kFlagTimeout));
+    }
+  }
+  __syncthreads();
+#pragma unroll
+  for (int k = 0; k < 8; ++k) out[k] = H.bc[k];
+  oflags = __float_as_int(H.bc[8]);
+  xp ^= 1;
+}
+
+// ---------------------------------------------------------------- tree
+// first_child[n + 1] / next_sibling[c] in ascending node order, built by one
+// warp from the highest index down (siblings found with __match_any_sync).
+__device__ void build_children(const int16_t* par, int16_t* first_child, int16_t* next_sib,
+                               int N) {
+  const int lane = threadIdx.x & 31;
+  if ((threadIdx.x >> 5) != 0 || N == 0) return;
+  for (int base = (N - 1) & ~31; base >= 0; base -= 32) {
+    const int c = base + lane;
+    const bool valid = c < N && par[c] >= -1;
+    const int key = valid ? par[c] : -1000 - lane;
+    const unsigned m = __match_any_sync(0xffffffffu, key);
+    const unsigned above = m & ~((2u << lane) - 1u);
+    int nxt = -1;
+    if (valid) nxt = above ? base + __ffs(above) - 1 : first_child[key + 1];
+    __syncwarp();
+    if (valid) {
+      next_sib[c] = (int16_t)nxt;
+      if (lane == __ffs(m) - 1) first_child[key + 1] = (int16_t)c;
+    }
+    __syncwarp();
   }
 }
 
-// e = exp((z - M) / T) over the slice (0 beyond the valid part), sums, and
-// the stored values of token `x1` when this CTA owns it.
+// ---------------------------------------------------------------- row I/O
+// Starts the copies of this CTA's slice [lo, lo + nloc) of the target row
+// (and of the draft row when need_draft) that begins at element row_base.
 template <int THREADS, bool BF16>
-__device__ __forceinline__ void exp_pass(float* W, float* Q, int L, int nloc, int lo,
-                                         bool need_draft, float Mt, float Md, float c,
-                                         int x1, float& st, float& sd, float& pubW,
-                                         float& pubQ) {
-  st = 0.f;
-  sd = 0.f;
-  pubW = 0.f;
-  pubQ = 0.f;
-  if constexpr (BF16) {
-    constexpr int CH = THREADS * 8;
-    for (int base = 0; base < L; base += CH) {
-      const int i = base + (int)threadIdx.x * 8;
-      float et[8], ed[8];
-#pragma unroll
-      for (int which = 0; which < 2; ++which) {
-        float* e = which ? ed : et;
-#pragma unroll
-        for (int k = 0; k < 8; ++k) e[k] = 0.f;
-        if (which == 1 && !need_draft) continue;
-        if (i < nloc) {
-          const uint16_t* raw = reinterpret_cast<const uint16_t*>(which ? Q : W) + L;
-          const uint4 r = *reinterpret_cast<const uint4*>(raw + i);
-          const uint32_t w[4] = {r.x, r.y, r.z, r.w};
-          const float M = which ? Md : Mt;
-#pragma unroll
-          for (int k = 0; k < 4; ++k) {
-            if (i + 2 * k < nloc) e[2 * k] = exp2f(__fmul_rn(__fsub_rn(bf16_lo(w[k]), M), c));
-            if (i + 2 * k + 1 < nloc)
-              e[2 * k + 1] = exp2f(__fmul_rn(__fsub_rn(bf16_hi(w[k]), M), c));
-          }
-        }
-      }
-      __syncthreads();  // every raw value of this chunk has been read
-      if (i < L) {
-        float4* wt = reinterpret_cast<float4*>(W + i);
-        wt[0] = make_float4(et[0], et[1], et[2], et[3]);
-        wt[1] = make_float4(et[4], et[5], et[6], et[7]);
-        if (need_draft) {
-          float4* wd = reinterpret_cast<float4*>(Q + i);
-          wd[0] = make_float4(ed[0], ed[1], ed[2], ed[3]);
-          wd[1] = make_float4(ed[4], ed[5], ed[6], ed[7]);
-        }
-#pragma unroll
-        for (int k = 0; k < 8; ++k) {
-          st += et[k];
-          sd += ed[k];
-          if (lo + i + k == x1) { pubW = et[k]; pubQ = ed[k]; }
+__device__ __forceinline__ void issue_rows(Head& H, const VerifyParams& P, float* W, float* Q,
+                                           size_t row_base, bool need_draft, int lo, int nloc) {
+  const int L = P.slice;
+  const size_t off = row_base + (size_t)lo;
+  constexpr uint32_t es = BF16 ? 2u : 4u;
+  constexpr uint32_t kChunkBytes = 2u * THREADS * 16u;
+  // Earlier generic accesses to W / Q must be ordered before the copies.
+  fence_proxy_async_smem();
+  __syncthreads();
+  if (P.use_tma) {
+    if (threadIdx.x == 0) {
+      const uint32_t bytes = (uint32_t)nloc * es;
+      const uint32_t dst_off = BF16 ? 2u * (uint32_t)L : 0u;
+      for (int which = 0; which < (need_draft ? 2 : 1); ++which) {
+        const char* src = static_cast<const char*>(which ? P.zd : P.zt) + off * es;
+        const uint32_t dst = smem_addr(which ? Q : W) + dst_off;
+        int k = 0;
+        for (uint32_t o = 0; o < bytes; o += kChunkBytes, ++k) {
+          const uint32_t n = min(kChunkBytes, bytes - o);
+          const uint32_t bar = smem_addr(&H.tbar[which][k]);
+          mbar_arrive_expect_tx(bar, n);
+          bulk_g2s(dst + o, src + o, n, bar);
         }
       }
     }
   } else {
-    for (int i = threadIdx.x * 4; i < L; i += THREADS * 4) {
-      for (int which = 0; which < (need_draft ? 2 : 1); ++which) {
-        float* buf = which ? Q : W;
-        const float M = which ? Md : Mt;
-        float4 r = *reinterpret_cast<float4*>(buf + i);
-        float x[4] = {r.x, r.y, r.z, r.w};
+    for (int which = 0; which < (need_draft ? 2 : 1); ++which) {
+      float* dst = which ? Q : W;
+      if constexpr (BF16) {
+        const uint16_t* src = static_cast<const uint16_t*>(which ? P.zd : P.zt) + off;
+        uint16_t* raw = reinterpret_cast<uint16_t*>(dst) + L;
+        for (int i = threadIdx.x; i < nloc; i += THREADS) raw[i] = __ldg(src + i);
+      } else {
+        const float* src = static_cast<const float*>(which ? P.zd : P.zt) + off;
+        for (int i = threadIdx.x; i < nloc; i += THREADS) dst[i] = __ldg(src + i);
+      }
+    }
+    __syncthreads();
+  }
+}
+
+__device__ __forceinline__ float bf16_lo(uint32_t w) { return __uint_as_float(w << 16); }
+__device__ __forceinline__ float bf16_hi(uint32_t w) { return __uint_as_float(w & 0xffff0000u); }
+
+// Tempered normaliser, first half (S2): one pass over this CTA's slice of a
+// row as its chunks land.  With c = log2(e) / T and the thread's reference
+// mref (log2 units: the rounded product of its largest logit so far and c)
+// it stores e = 2^(z c - mref), one fused multiply-add and one 2^x per
+// element (0 beyond the valid part), and returns (mref, sum e).  A NaN or
+// +inf logit makes the thread's sum non-finite, which is how the error
+// contract detects it.  Returns false if a chunk wait timed out.
+template <int THREADS, bool BF16>
+__device__ __forceinline__ bool normalize_row(float* buf, int L, int nloc, float c,
+                                              uint32_t bar0, uint32_t parity, int nk_tma,
+                                              bool wait_tma, float& mref, float& ssum) {
+  constexpr int VEC = BF16 ? 8 : 4;
+  constexpr int CV = 2 * THREADS;
+  const int NV = L / VEC;
+  const int NVV = nloc / VEC;  // vectors whose VEC elements are all valid
+  const int NK = (NV + CV - 1) / CV;
+  const int tid = threadIdx.x;
+  const uint16_t* raw = reinterpret_cast<const uint16_t*>(buf) + L;
+  bool ok = true;
+  mref = -INFINITY;
+  ssum = 0.f;
+  for (int k = 0; k < NK; ++k) {
+    if (wait_tma && k < nk_tma) ok = wait_bar(bar0 + 8u * (uint32_t)k, parity) && ok;
+    float z[2][VEC];
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+      const int g = k * CV + h * THREADS + tid;
+#pragma unroll
+      for (int j = 0; j < VEC; ++j) z[h][j] = -INFINITY;
+      if (g < NVV || (g < NV && g * VEC < nloc)) {
+        if constexpr (BF16) {
+          const uint4 r = *reinterpret_cast<const uint4*>(raw + (size_t)g * 8);
+          const uint32_t w[4] = {r.x, r.y, r.z, r.w};
+#pragma unroll
+          for (int j = 0; j < 4; ++j) {
+            z[h][2 * j] = bf16_lo(w[j]);
+            z[h][2 * j + 1] = bf16_hi(w[j]);
+          }
+        } else {
+          const float4 r = *reinterpret_cast<const float4*>(buf + (size_t)g * 4);
+          z[h][0] = r.x; z[h][1] = r.y; z[h][2] = r.z; z[h][3] = r.w;
+        }
+        if (g >= NVV) {  // ragged tail of the slice (plain-load path only)
+#pragma unroll
+          for (int j = 0; j < VEC; ++j)
+            if (g * VEC + j >= nloc) z[h][j] = -INFINITY;
+        }
+      }
+    }
+    float vmax = -INFINITY;
+#pragma unroll
+    for (int h = 0; h < 2; ++h)
+#pragma unroll
+      for (int j = 0; j < VEC; ++j) vmax = fmaxf(vmax, z[h][j]);
+    if (__fmaf_rn(vmax, c, -mref) > kRebaseLog2) {
+      // Move this thread's reference up: rescale what it stored so far.
+      const float mnew = __fmul_rn(vmax, c);
+      if (mref != -INFINITY) {
+        const float f = ex2(__fsub_rn(mref, mnew));
+        ssum = __fmul_rn(ssum, f);
+        for (int k2 = 0; k2 < k; ++k2)
+          for (int h = 0; h < 2; ++h) {
+            const int g = k2 * CV + h * THREADS + tid;
+            if (g < NV)
+              for (int j = 0; j < VEC; ++j) buf[g * VEC + j] = __fmul_rn(buf[g * VEC + j], f);
+          }
+      }
+      mref = mnew;
+    }
+    float e[2][VEC];
+    if (mref == -INFINITY) {  // nothing finite seen yet: every value is -inf or NaN
+#pragma unroll
+      for (int h = 0; h < 2; ++h)
+#pragma unroll
+        for (int j = 0; j < VEC; ++j) {
+          e[h][j] = 0.f;
+          if (isnan(z[h][j])) ssum = __int_as_float(0x7fc00000);
+        }
+    } else {
+#pragma unroll
+      for (int h = 0; h < 2; ++h) {
         float s = 0.f;
 #pragma unroll
-        for (int k = 0; k < 4; ++k) {
-          x[k] = (i + k < nloc) ? exp2f(__fmul_rn(__fsub_rn(x[k], M), c)) : 0.f;
-          s += x[k];
-          if (lo + i + k == x1) { if (which) pubQ = x[k]; else pubW = x[k]; }
+        for (int j = 0; j < VEC; ++j) {
+          e[h][j] = ex2(__fmaf_rn(z[h][j], c, -mref));
+          s += e[h][j];
         }
-        *reinterpret_cast<float4*>(buf + i) = make_float4(x[0], x[1], x[2], x[3]);
-        if (which) sd += s; else st += s;
+        ssum += s;
+      }
+    }
+    if constexpr (BF16) __syncthreads();  // this chunk's raw values are all read
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+      const int g = k * CV + h * THREADS + tid;
+      if (g < NV) {
+        float4* d = reinterpret_cast<float4*>(buf + (size_t)g * VEC);
+#pragma unroll
+        for (int j = 0; j < VEC / 4; ++j)
+          d[j] = make_float4(e[h][4 * j], e[h][4 * j + 1], e[h][4 * j + 2], e[h][4 * j + 3]);
       }
     }
   }
+  return ok;
 }
 
 // One rejection pass: materialise R_j = map(W) into W and accumulate the
 // sums of rejection j (ResiSpec: sum min(Z q, R) and sum (R - min(Z q, R))
-// over x != x0; SpecInfer: sum (R - q)_+), publishing the next candidate.
-template <int THREADS, int KIND, bool RESI>
-__device__ __forceinline__ void reject_pass(float* W, const float* Q, int L, int lo,
-                                            const Pending& P, float invSd, int x0, float Z,
-                                            int xn, float& s1, float& s2, float& pubW,
-                                            float& pubQ) {
-  s1 = 0.f;
-  s2 = 0.f;
-  pubW = 0.f;
-  pubQ = 0.f;
-  for (int i = threadIdx.x * 4; i < L; i += THREADS * 4) {
-    float4 wv = *reinterpret_cast<float4*>(W + i);
-    const float4 qv = *reinterpret_cast<const float4*>(Q + i);
-    float w[4] = {wv.x, wv.y, wv.z, wv.w};
-    const float qr[4] = {qv.x, qv.y, qv.z, qv.w};
+// over x != x0; SpecInfer: sum (R - q)_+), publishing token xn's values.
+// Per-element index tests are needed only in the (at most three) vectors
+// that hold x0, xn or the previous map's x0.
+template <int VEC, int KIND, bool RESI, bool CHECK>
+__device__ __forceinline__ void reject_vector(float (&w)[VEC], const float (&q)[VEC], int base,
+                                              const Pending& P, float at, float bt, float mt,
+                                              float md, int x0, float Z, int xn, float& t1,
+                                              float& t2, float* pubv) {
 #pragma unroll
-    for (int k = 0; k < 4; ++k) {
-      const int idx = lo + i + k;
-      const float qq = __fmul_rn(qr[k], invSd);
-      const float R = apply_map<KIND>(P, w[k], qq, idx);
-      w[k] = R;
-      if constexpr (RESI) {
-        if (idx != x0) {
-          const float m = fminf(__fmul_rn(Z, qq), R);
-          s1 += m;
-          s2 += __fsub_rn(R, m);
-        }
-      } else {
-        s1 += fmaxf(__fsub_rn(R, qq), 0.f);
-      }
-      if (idx == xn) { pubW = R; pubQ = qr[k]; }
+  for (int j = 0; j < VEC; ++j) {
+    const int idx = base + j;
+    const float qq = __fmul_rn(q[j], bt);
+    float R;
+    if constexpr (KIND == kResi && !CHECK) {
+      const float m = fminf(__fmul_rn(P.Z, qq), w[j]);
+      R = __fmul_rn(__fmaf_rn(P.lam, __fsub_rn(w[j], m), m), P.a);
+    } else {
+      R = apply_map<KIND>(P, w[j], qq, idx, at);
     }
-    *reinterpret_cast<float4*>(W + i) = make_float4(w[0], w[1], w[2], w[3]);
+    if (CHECK && idx == xn) { pubv[0] = R; pubv[1] = mt; pubv[2] = q[j]; pubv[3] = md; }
+    w[j] = R;
+    if constexpr (RESI) {
+      if (!CHECK || idx != x0) {
+        const float m = fminf(__fmul_rn(Z, qq), R);
+        t1 += m;
+        t2 += __fsub_rn(R, m);
+      }
+    } else {
+      t1 += fmaxf(__fsub_rn(R, qq), 0.f);
+    }
   }
 }
 
-template <int THREADS, bool RESI>
+template <int THREADS, bool BF16, int KIND, bool RESI>
+__device__ __forceinline__ void reject_pass(float* W, const float* Q, int L, int lo,
+                                            const Pending& P, float at, float bt, float mt,
+                                            float md, int x0, float Z, int xn, float* pubv,
+                                            float& s1out, float& s2out) {
+  constexpr int VEC = BF16 ? 8 : 4;
+  const int NV = L / VEC;
+  // vectors that need per-element index tests (-1: none in this slice)
+  auto vec_of = [&](int x) { return (x >= lo && x < lo + L) ? (x - lo) / VEC : -1; };
+  const int s0 = vec_of(x0), s1 = vec_of(xn), s2 = KIND == kResi ? vec_of(P.x0) : -1;
+  float s1sum = 0.f, s2sum = 0.f;
+  for (int g = threadIdx.x; g < NV; g += THREADS) {
+    float w[VEC], q[VEC];
+#pragma unroll
+    for (int j = 0; j < VEC / 4; ++j) {
+      const float4 a = reinterpret_cast<const float4*>(W + (size_t)g * VEC)[j];
+      const float4 b = reinterpret_cast<const float4*>(Q + (size_t)g * VEC)[j];
+      w[4 * j] = a.x; w[4 * j + 1] = a.y; w[4 * j + 2] = a.z; w[4 * j + 3] = a.w;
+      q[4 * j] = b.x; q[4 * j + 1] = b.y; q[4 * j + 2] = b.z; q[4 * j + 3] = b.w;
+    }
+    float t1 = 0.f, t2 = 0.f;
+    if (g == s0 || g == s1 || g == s2)
+      reject_vector<VEC, KIND, RESI, true>(w, q, lo + g * VEC, P, at, bt, mt, md, x0, Z, xn, t1,
+                                           t2, pubv);
+    else
+      reject_vector<VEC, KIND, RESI, false>(w, q, lo + g * VEC, P, at, bt, mt, md, x0, Z, xn,
+                                            t1, t2, pubv);
+    s1sum += t1;
+    s2sum += t2;
+#pragma unroll
+    for (int j = 0; j < VEC / 4; ++j)
+      reinterpret_cast<float4*>(W + (size_t)g * VEC)[j] =
+          make_float4(w[4 * j], w[4 * j + 1], w[4 * j + 2], w[4 * j + 3]);
+  }
+  s1out = s1sum;
+  s2out = s2sum;
+}
+
+template <int THREADS, bool BF16, bool RESI>
 __device__ __forceinline__ void reject_pass_any(float* W, const float* Q, int L, int lo,
-                                                const Pending& P, float invSd, int x0, float Z,
-                                                int xn, float& s1, float& s2, float& pubW,
-                                                float& pubQ) {
+                                                const Pending& P, float at, float bt, float mt,
+                                                float md, int x0, float Z, int xn, float* pubv,
+                                                float& s1, float& s2) {
   switch (P.kind) {
     case kScale:
-      reject_pass<THREADS, kScale, RESI>(W, Q, L, lo, P, invSd, x0, Z, xn, s1, s2, pubW, pubQ);
+      reject_pass<THREADS, BF16, kScale, RESI>(W, Q, L, lo, P, at, bt, mt, md, x0, Z, xn, pubv,
+                                               s1, s2);
       break;
     case kIdent:
-      reject_pass<THREADS, kIdent, RESI>(W, Q, L, lo, P, invSd, x0, Z, xn, s1, s2, pubW, pubQ);
+      reject_pass<THREADS, BF16, kIdent, RESI>(W, Q, L, lo, P, at, bt, mt, md, x0, Z, xn, pubv,
+                                               s1, s2);
       break;
     case kResi:
-      reject_pass<THREADS, kResi, RESI>(W, Q, L, lo, P, invSd, x0, Z, xn, s1, s2, pubW, pubQ);
+      reject_pass<THREADS, BF16, kResi, RESI>(W, Q, L, lo, P, at, bt, mt, md, x0, Z, xn, pubv,
+                                              s1, s2);
       break;
     default:
-      reject_pass<THREADS, kSpec, RESI>(W, Q, L, lo, P, invSd, x0, Z, xn, s1, s2, pubW, pubQ);
+      reject_pass<THREADS, BF16, kSpec, RESI>(W, Q, L, lo, P, at, bt, mt, md, x0, Z, xn, pubv,
+                                              s1, s2);
       break;
   }
 }
 
 // ---------------------------------------------------------------- sampler
-// Inverse-CDF draw: the smallest token x with C(x) > u * C(V-1), found
-// hierarchically (CTA slice, then warp range, then 32-token group, then
-// lane).  Groups of 32 are summed in fp32; the running sums above them are
-// kept in fp64 (a few dozen additions per CTA) so that the prefix rounding
-// stays far below the near-tie margin.  Each level falls back to its last
-// unit with positive mass, so the result always has R(x) > 0.  Returns
-// false when the residual has no mass.
-template <int THREADS>
-__device__ bool sample_final(Head& H, const VerifyParams& P, const float* W, const float* Q,
-                             const Pending& Pm, float invSd, int b, int row, int depth,
-                             int lo, int nloc, uint32_t rank, uint32_t C, int& par) {
+// The inverse-CDF search runs on exact 64-bit fixed-point masses
+// (probability * 2^44, rounded): integer sums are associative, so every
+// level of the hierarchical search agrees with every other.
+constexpr float kFix = 17592186044416.f;  // 2^44
+
+__device__ __forceinline__ unsigned long long to_fix(float x) {
+  return __float2ull_rn(__fmul_rn(x, kFix));
+}
+
+__device__ __forceinline__ unsigned long long warp_sum_u64(unsigned long long v) {
+#pragma unroll
+  for (int o = 16; o; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+
+// Per-CTA mass of the final distribution, from the partials of the exchange
+// that defined it (kind 1: normaliser pairs; 2: ResiSpec sums; 3: SpecInfer
+// sums; 4: direct sums).
+__device__ __forceinline__ float cta_mass(const Head& H, int r, int kind, const Pending& Pm,
+                                          float Mt, float invSt) {
+  const float* p = H.part[r];
+  switch (kind) {
+    case 1: return __fmul_rn(p[1], ref_scale(p[0], Mt, invSt));
+    case 2: return __fmul_rn(__fmaf_rn(Pm.lam, p[1], p[0]), Pm.a);
+    case 3: return __fmul_rn(p[0], Pm.a);
+    default: return p[0];
+  }
+}
+
+// Inverse-CDF draw: the smallest token x with C(x) > u * C(V-1), u = k 2^-24.
+// Every CTA picks the CTA whose mass range holds u * total (masses from the
+// exchange partials); that CTA materialises the final distribution in W,
+// sums NW contiguous warp segments, then one warp splits its segment into 32
+// contiguous lane ranges and one lane walks its range.  When rounding puts
+// the threshold past a unit's own total, the search falls back to the last
+// token with positive mass, so the result always has R(x) > 0.  Returns
+// false when the distribution has no mass.
+template <int THREADS, bool BF16>
+__device__ bool sample_final(Head& H, const VerifyParams& P, float* W, const float* Q,
+                             const Pending& Pm, int mass_kind, float at, float bt, float Mt,
+                             float invSt, float u, int b, int depth, int lo, int nloc,
+                             uint32_t rank, uint32_t C, int& xp, uint32_t& xph) {
+  constexpr int VEC = BF16 ? 8 : 4;
   constexpr int NW = THREADS / 32;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int L = P.slice;
-  const int Lw = ((L + NW * 32 - 1) / (NW * 32)) * 32;
-  const int wb = warp * Lw;
-  const int we = min(wb + Lw, nloc);
-  float* dist = P.out_dist ? P.out_dist + (size_t)b * P.V + lo : nullptr;
-  double acc = 0.0;
-  for (int g = wb; g < we; g += 32) {
-    const int i = g + lane;
-    float v = 0.f;
-    if (i < we) {
-      v = apply_any(Pm, W[i], __fmul_rn(Q[i], invSd), lo + i);
-      if (dist) dist[i] = v;
-    }
-    acc += (double)warp_sum(v);
-  }
-  if (lane == 0) H.wsum[warp] = acc;
-  __syncthreads();
-  if (threadIdx.x == 0) {
-    double t = 0.0;
-    for (int w = 0; w < NW; ++w) t += H.wsum[w];
-    H.slot[par].d = t;
-  }
-  cluster_sync();
-  if (warp == 0) {
-    if (lane < (int)C) {
-      const uint32_t addr = map_to_rank(smem_addr(&H.slot[par].d), lane);
-      H.cta_tot[lane] = ld_cluster_f64(addr);
-    }
-    __syncwarp();
-    if (lane == 0) {
-      const double u = (double)uniform_draw(P.seed, (uint32_t)b, (uint32_t)row, 1);
-      double total = 0.0;
-      for (uint32_t r = 0; r < C; ++r) total += H.cta_tot[r];
-      int cstar = -1, force = 0;
-      double before = 0.0;
-      if (total > 0.0) {
-        const double tau = u * total;
-        double a = 0.0, last_before = 0.0;
-        int last = -1;
-        for (uint32_t r = 0; r < C; ++r) {
-          const double nx = a + H.cta_tot[r];
-          if (H.cta_tot[r] > 0.0) { last = (int)r; last_before = a; }
-          if (nx > tau) { cstar = (int)r; before = a; break; }
-          a = nx;
-        }
-        if (cstar < 0) { cstar = last; before = last_before; force = 1; }
-        H.miscd[0] = tau - before;
+  const int NV = L / VEC;
+  bool materialised = false;
+  // Owners turn their stored values into the final distribution, in place.
+  auto materialise = [&](float* dist) -> float {
+    float s = 0.f;
+    for (int g = threadIdx.x; g < NV; g += THREADS) {
+      float vals[VEC];
+#pragma unroll
+      for (int j = 0; j < VEC; ++j) {
+        const int li = g * VEC + j;
+        vals[j] = li < nloc ? apply_any(Pm, W[li], __fmul_rn(Q[li], bt), lo + li, at) : 0.f;
+        s += vals[j];
+        if (dist && li < nloc) dist[li] = vals[j];
       }
-      H.misc[0] = cstar;
-      H.misc[1] = force;
+#pragma unroll
+      for (int j = 0; j < VEC / 4; ++j)
+        reinterpret_cast<float4*>(W + (size_t)g * VEC)[j] =
+            make_float4(vals[4 * j], vals[4 * j + 1], vals[4 * j + 2], vals[4 * j + 3]);
+    }
+    return s;
+  };
+  const bool need_direct = mass_kind == 0;
+  if (P.out_dist || need_direct) {
+    const float s = materialise(P.out_dist ? P.out_dist + (size_t)b * P.V + lo : nullptr);
+    materialised = true;
+    if (need_direct) {
+      float o[8];
+      int of;
+      exchange<NW, false>(H, s, 0.f, 0.f, 0.f, 0, xp, xph, rank, C, o, of);
+      mass_kind = 4;
     }
   }
+  if (threadIdx.x == 0) {
+    unsigned long long total = 0;
+    for (uint32_t r = 0; r < C; ++r) total += to_fix(cta_mass(H, r, mass_kind, Pm, Mt, invSt));
+    int cstar = -1;
+    unsigned long long before = 0;
+    if (total > 0) {
+      // tau = floor(k * total / 2^24) with u = k / 2^24, exactly
+      const unsigned long long k = (unsigned long long)(u * 16777216.f);
+      const unsigned long long lo64 = k * total, hi64 = __umul64hi(k, total);
+      const unsigned long long tau = (hi64 << 40) | (lo64 >> 24);
+      unsigned long long a = 0;
+      for (uint32_t r = 0; r < C; ++r) {
+        const unsigned long long m = to_fix(cta_mass(H, r, mass_kind, Pm, Mt, invSt));
+        if (a + m > tau) { cstar = (int)r; before = a; break; }
+        a += m;
+      }
+      H.fixd[0] = tau - before;
+    }
+    H.misc[0] = cstar;
+  }
   __syncthreads();
-  par ^= 1;
   const int cstar = H.misc[0];
   if (cstar < 0) return false;
   if ((int)rank != cstar) return true;
-  // This CTA holds the draw: find the warp range, then the group, then the lane.
+
+  if (!materialised) {
+    materialise(nullptr);
+    __syncthreads();
+  }
+  // warp segments of SEG elements (multiple of 4); W holds 0 beyond nloc
+  const int SEG = ((L + NW * 4 - 1) / (NW * 4)) * 4;
+  {
+    const int s0 = warp * SEG, s1 = min(s0 + SEG, L);
+    unsigned long long acc = 0;
+    for (int i = s0 + 4 * lane; i < s1; i += 128) {
+      const float4 x = *reinterpret_cast<const float4*>(W + i);
+      acc += to_fix(x.x) + to_fix(x.y) + to_fix(x.z) + to_fix(x.w);
+    }
+    acc = warp_sum_u64(acc);
+    if (lane == 0) H.seg[warp] = acc;
+  }
+  __syncthreads();
   if (threadIdx.x == 0) {
-    const double t = H.miscd[0];
-    int force = H.misc[1];
-    double a = 0.0, last_before = 0.0;
+    const unsigned long long t = H.fixd[0];
+    unsigned long long a = 0;
     int wstar = -1, last = -1;
     for (int w = 0; w < NW; ++w) {
-      const double s = H.wsum[w];
-      if (s > 0.0) { last = w; last_before = a; }
-      if (!force && a + s > t) { wstar = w; break; }
-      a += s;
+      const unsigned long long m = H.seg[w];
+      if (m > 0) last = w;
+      if (a + m > t) { wstar = w; break; }
+      a += m;
     }
-    if (wstar < 0) { wstar = last; a = last_before; force = 1; }
-    H.misc[2] = wstar;
-    H.misc[3] = force;
-    H.miscd[1] = t - a;
+    H.misc[3] = wstar < 0;  // threshold beyond this CTA's total: take the last token
+    H.misc[2] = wstar < 0 ? max(last, 0) : wstar;
+    H.fixd[1] = wstar < 0 ? 0 : t - a;
   }
   __syncthreads();
   if (warp == H.misc[2]) {
-    const double t = H.miscd[1];
-    bool force = H.misc[3] != 0;
-    double a = 0.0, last_before = 0.0;
-    int gstar = -1, last = -1;
-    for (int g = wb; g < we; g += 32) {
-      const int i = g + lane;
-      const float v = i < we ? apply_any(Pm, W[i], __fmul_rn(Q[i], invSd), lo + i) : 0.f;
-      const double s = (double)warp_sum(v);
-      if (s > 0.0) { last = g; last_before = a; }
-      if (!force && a + s > t) { gstar = g; break; }
-      a += s;
+    const int s0 = warp * SEG, s1 = min(s0 + SEG, L);
+    const int SUB = (SEG + 31) / 32;
+    const int r0 = s0 + lane * SUB, r1 = min(r0 + SUB, s1);
+    unsigned long long m = 0;
+    int lastpos = -1;
+    for (int i = r0; i < r1; ++i) {
+      const float x = W[i];
+      m += to_fix(x);
+      if (x > 0.f) lastpos = i;
     }
-    if (gstar < 0) { gstar = last; a = last_before; force = true; }
-    const int i = gstar + lane;
-    const float v = i < we ? apply_any(Pm, W[i], __fmul_rn(Q[i], invSd), lo + i) : 0.f;
-    double s = (double)v;
+    unsigned long long incl = m;
 #pragma unroll
     for (int o = 1; o < 32; o <<= 1) {
-      const double n = __shfl_up_sync(0xffffffffu, s, o);
-      if (lane >= o) s += n;
+      const unsigned long long n = __shfl_up_sync(0xffffffffu, incl, o);
+      if (lane >= o) incl += n;
     }
-    const double tl = t - a;
-    const unsigned cross = __ballot_sync(0xffffffffu, !force && s > tl);
-    const unsigned pos = __ballot_sync(0xffffffffu, v > 0.f);
-    const int l = cross ? __ffs(cross) - 1 : 31 - __clz(pos);
-    if (lane == 0) P.out_tokens[(size_t)b * (P.D + 1) + depth] = lo + gstar + l;
+    const unsigned long long t = H.fixd[1];
+    const bool force = H.misc[3] != 0;
+    const unsigned cross = __ballot_sync(0xffffffffu, !force && incl > t);
+    const unsigned pos = __ballot_sync(0xffffffffu, lastpos >= 0);
+    const int sel = cross ? __ffs(cross) - 1 : (pos ? 31 - __clz(pos) : 0);
+    if (lane == sel) {
+      int pick = -1;
+      if (cross) {
+        const unsigned long long tl = t - (incl - m);
+        unsigned long long a = 0;
+        for (int i = r0; i < r1; ++i) {
+          a += to_fix(W[i]);
+          if (a > tl) { pick = i; break; }
+        }
+      }
+      if (pick < 0) pick = lastpos >= 0 ? lastpos : r0;
+      P.out_tokens[(size_t)b * (P.D + 1) + depth] = lo + pick;
+    }
   }
   return true;
 }
 
 // ---------------------------------------------------------------- kernel
 template <int THREADS, bool BF16>
-__global__ void __launch_bounds__(THREADS, 1) verify_kernel(const VerifyParams P) {
+__global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 3)
+    verify_kernel(const VerifyParams P) {
   constexpr int NW = THREADS / 32;
+  constexpr int VEC = BF16 ? 8 : 4;
+  constexpr uint32_t es = BF16 ? 2u : 4u;
+  constexpr uint32_t kChunkBytes = 2u * THREADS * 16u;
   extern __shared__ __align__(128) unsigned char smem[];
   Head& H = *reinterpret_cast<Head*>(smem);
   const int L = P.slice;
   float* W = reinterpret_cast<float*>(smem + kHeadBytes);
   float* Q = W + L;
   int16_t* par = reinterpret_cast<int16_t*>(Q + L);
-  int16_t* kids = par + P.npad;
-  int32_t* kidtok = reinterpret_cast<int32_t*>(kids + P.npad);
-  uint8_t* haschild = reinterpret_cast<uint8_t*>(kidtok + P.npad);
+  int16_t* first_child = par + P.npad;
+  int16_t* next_sib = first_child + P.npad + 16;
+  int32_t* cand_s = reinterpret_cast<int32_t*>(next_sib + P.npad);
+  float* u_acc = reinterpret_cast<float*>(cand_s + P.npad);  // [r]: accept test of node r - 1
+  float* u_fin = u_acc + P.npad;                             // [r]: final draw at row r
 
   const int tid = threadIdx.x;
   const uint32_t rank = cluster_ctarank();
@@ -614,148 +749,196 @@ __global__ void __launch_bounds__(THREADS, 1) verify_kernel(const VerifyParams P
   const int N = P.N, V = P.V, D = P.D;
   const int lo = (int)rank * L;
   const int nloc = max(0, min(V, lo + L) - lo);
-  const int32_t* cand_b = P.cand + (size_t)b * N;
+  const int nk_tma = (int)(((uint32_t)nloc * es + kChunkBytes - 1) / kChunkBytes);
+  const float c = P.scale_log2;
 
+  if (tid < 4) H.pubv[tid] = 0.f;
   if (tid == 0) {
-    mbar_init(smem_addr(&H.mbar[0]), 1);
-    mbar_init(smem_addr(&H.mbar[1]), 1);
+    for (int w = 0; w < 2; ++w)
+      for (int k = 0; k < kMaxChunks; ++k) mbar_init(smem_addr(&H.tbar[w][k]), 1);
+    mbar_init(smem_addr(&H.xbar[0]), 1);
+    mbar_init(smem_addr(&H.xbar[1]), 1);
     fence_mbar_init();
   }
-  for (int i = tid; i <= N; i += THREADS) haschild[i] = 0;
   __syncthreads();
+  // Root rows first: a valid tree with N > 0 always has root children.
+  issue_rows<THREADS, BF16>(H, P, W, Q, (size_t)b * P.seq_stride, N > 0, lo, nloc);
+
+  for (int i = tid; i < P.npad + 16; i += THREADS) first_child[i] = -1;
   int bad = 0;
-  for (int c = tid; c < N; c += THREADS) {
-    const int p = __ldg(P.parents + c);
-    const bool ok = p >= -1 && p < c;
+  for (int i = tid; i < N; i += THREADS) {
+    const int p = __ldg(P.parents + i);
+    const bool ok = p >= -1 && p < i;
     bad |= !ok;
-    par[c] = (int16_t)(ok ? p : -2);
-    if (ok) haschild[p + 1] = 1;
+    par[i] = (int16_t)(ok ? p : -2);
+    cand_s[i] = __ldg(P.cand + (size_t)b * N + i);
+  }
+  // Every uniform this sequence can use, off the critical path: one Philox
+  // block per logit row r gives the accept draw of node r - 1 (word 0) and
+  // the final draw at row r (word 1).
+  for (int r = tid; r <= N; r += THREADS) {
+    const U64x4 blk = philox4x64_10((uint64_t)r, (uint64_t)(uint32_t)b, 0, 0, P.seed, 0);
+    u_acc[r] = u24(blk.w[0]);
+    u_fin[r] = u24(blk.w[1]);
   }
   const bool tree_bad = __syncthreads_or(bad) != 0;
+  build_children(par, first_child, next_sib, N);
+  __syncthreads();
+  cluster_sync();  // every peer has started: its receive slots may now be written
 
   int err = tree_bad ? kErrTree : 0;
   int info = 0;
   int depth = 0, rejects = 0;
   int node = -1, row = 0;
-  uint32_t ph0 = 0, ph1 = 0;
-  int rpar = 0;
-  bool timed_out = false;
-  const float c = P.scale_log2;
-
-  if (!err)
-    issue_rows<THREADS, BF16>(H, P, W, Q, (size_t)b * P.seq_stride, haschild[0] != 0, lo, nloc);
+  uint32_t tph = 0, xph = 0;
+  int xp = 0;
+  uint32_t inflight = N > 0 ? 3u : 1u;  // rows whose copies are not yet consumed
 
   while (!err) {
-    const bool need_draft = haschild[node + 1] != 0;
-    const int nk = need_draft ? gather_children<THREADS>(H, par, kids, kidtok, node, N, cand_b) : 0;
+    const int c1 = first_child[node + 1];
+    const bool need_draft = c1 >= 0;
 
-    // ---- rows of this node: wait for the copies
-    if (P.use_tma) {
-      bool ok = wait_bar(smem_addr(&H.mbar[0]), ph0);
-      ph0 ^= 1;
-      if (need_draft) {
-        ok = wait_bar(smem_addr(&H.mbar[1]), ph1) && ok;
-        ph1 ^= 1;
-      }
-      timed_out |= !ok;
-    } else {
-      __syncthreads();
+    // ---- tempered normaliser (S2): one pass per row, then one exchange
+    float mref_t, sum_t, mref_d = -INFINITY, sum_d = 0.f;
+    bool ok = normalize_row<THREADS, BF16>(W, L, nloc, c, smem_addr(&H.tbar[0][0]), tph & 1u,
+                                           nk_tma, P.use_tma, mref_t, sum_t);
+    if (need_draft)
+      ok = normalize_row<THREADS, BF16>(Q, L, nloc, c, smem_addr(&H.tbar[1][0]),
+                                        (tph >> 1) & 1u, nk_tma, P.use_tma, mref_d, sum_d) && ok;
+    const bool bad_t = !(sum_t <= FLT_MAX), bad_d = !(sum_d <= FLT_MAX);
+    if (ok) {
+      tph ^= need_draft ? 3u : 1u;
+      inflight = 0;
     }
-
-    // ---- tempered normaliser: max, then exp and sums (S2)
-    float mt, md;
-    int flags = timed_out ? kFlagTimeout : 0;
-    if (!timed_out) max_pass<THREADS, BF16>(W, Q, L, nloc, need_draft, mt, md, flags);
-    else { mt = 0.f; md = 0.f; }
-    float v[6] = {mt, md, 0.f, 0.f, 0.f, 0.f}, o[6];
+    const int x1 = need_draft ? cand_s[c1] : -1;
+    if (x1 >= lo && x1 < lo + nloc && ((x1 - lo) / VEC) % THREADS == tid) {
+      H.pubv[0] = W[x1 - lo];
+      H.pubv[1] = mref_t;
+      H.pubv[2] = Q[x1 - lo];
+      H.pubv[3] = mref_d;
+    }
+    const int flags = (bad_t ? kFlagTargetBad : 0) | (bad_d ? kFlagDraftBad : 0) |
+                      (ok ? 0 : kFlagTimeout);
+    float o[8];
     int oflags;
-    exchange<NW>(H, v, flags, true, rpar, C, o, oflags);
-    const float Mt = o[0], Md = o[1];
+    exchange<NW, true>(H, mref_t, sum_t, mref_d, sum_d, flags, xp, xph, rank, C, o, oflags);
     if (oflags & kFlagTimeout) { err |= kErrTimeout; break; }
     if (oflags & kFlagTargetBad) { err |= kErrNonfinite; break; }
-    if (Mt == -INFINITY) { err |= kErrEmpty; break; }
+    if (o[0] == -INFINITY) { err |= kErrEmpty; break; }
     if (need_draft && (oflags & kFlagDraftBad)) { err |= kErrNonfinite; break; }
-    if (need_draft && Md == -INFINITY) { err |= kErrEmpty; break; }
-
-    const int x1 = nk > 0 ? kidtok[0] : -1;
-    float st, sd, pw, pq;
-    exp_pass<THREADS, BF16>(W, Q, L, nloc, lo, need_draft, Mt, Md, c, x1, st, sd, pw, pq);
-    float v2[6] = {st, sd, 0.f, 0.f, pw, pq};
-    exchange<NW>(H, v2, 0, false, rpar, C, o, oflags);
-    const float invSt = __frcp_rn(o[0]);
-    const float invSd = need_draft ? __frcp_rn(o[1]) : 0.f;
-    float pubW = o[4], pubQ = o[5];
-    Pending Pm{kScale, -1, invSt, 0.f, 0.f};
+    if (need_draft && o[2] == -INFINITY) { err |= kErrEmpty; break; }
+    const float Mt = o[0], invSt = __frcp_rn(o[1]);
+    const float Md = o[2], invSd = need_draft ? __frcp_rn(o[3]) : 0.f;
+    const float at = ref_scale(mref_t, Mt, invSt);
+    const float bt = need_draft ? ref_scale(mref_d, Md, invSd) : 0.f;
+    float pub[4] = {o[4], o[5], o[6], o[7]};
+    Pending Pm{kScale, -1, 0.f, 0.f, 0.f};
+    int mass_kind = 1;
 
     if (!need_draft) {
       // accepted leaf (or a root without children): bonus token from p
-      if (!sample_final<THREADS>(H, P, W, Q, Pm, invSd, b, row, depth, lo, nloc, rank, C, rpar))
+      if (!sample_final<THREADS, BF16>(H, P, W, Q, Pm, mass_kind, at, bt, Mt, invSt, u_fin[row],
+                                       b, depth, lo, nloc, rank, C, xp, xph))
         err |= kErrEmpty;
       break;
+    }
+    if (P.prefetch && tid == 0) {
+      // The first child is the most likely to be accepted: warm L2 with its rows.
+      const size_t base = ((size_t)b * P.seq_stride + (size_t)(c1 + 1) * V + lo) * es;
+      const uint32_t bytes = (uint32_t)nloc * es;
+      const int nrows = first_child[c1 + 1] >= 0 ? 2 : 1;
+      for (int w = 0; w < nrows; ++w) {
+        const char* src = static_cast<const char*>(w ? P.zd : P.zt) + base;
+        for (uint32_t o2 = 0; o2 < bytes; o2 += kChunkBytes)
+          prefetch_l2(src + o2, min(kChunkBytes, bytes - o2));
+      }
     }
 
     // ---- sequential accept tests over the children (S3), shaping on reject
     int accepted = -1, acc_tok = -1;
-    for (int j = 0; j < nk; ++j) {
-      const int cnode = kids[j];
-      const int x = kidtok[j];
+    for (int cn = c1; cn >= 0;) {
+      const int x = cand_s[cn];
       if (x < 0 || x >= V) { err |= kErrToken; break; }
-      const float qx = __fmul_rn(pubQ, invSd);
-      const float Rx = apply_any(Pm, pubW, qx, x);
-      const float u = uniform_draw(P.seed, (uint32_t)b, (uint32_t)(cnode + 1), 0);
-      if (__fmul_rn(u, qx) < Rx) { accepted = cnode; acc_tok = x; break; }
+      const float qx = __fmul_rn(pub[2], ref_scale(pub[3], Md, invSd));
+      const float Rx = Pm.kind == kScale ? __fmul_rn(pub[0], ref_scale(pub[1], Mt, invSt))
+                                         : apply_any(Pm, pub[0], qx, x, 0.f);
+      const float u = u_acc[cn + 1];
+      if (__fmul_rn(u, qx) < Rx) { accepted = cn; acc_tok = x; break; }
       rejects += 1;
-      const int xn = j + 1 < nk ? kidtok[j + 1] : -1;
-      float s1 = 0.f, s2 = 0.f, pw2 = 0.f, pq2 = 0.f;
+      const int nxt = next_sib[cn];
+      const int xn = nxt >= 0 ? cand_s[nxt] : -1;
+      float s1 = 0.f, s2 = 0.f;
       if (P.mode == 0) {
         const float Z = __fsub_rn(qx, Rx);
         if (!(Z > 0.f)) {
           // degenerate rejection: keep R, fetch the next candidate's values
           info |= kInfoDegenerate;
-          if (tid == 0 && xn >= lo && xn < lo + nloc) { pw2 = W[xn - lo]; pq2 = Q[xn - lo]; }
-          float v3[6] = {0.f, 0.f, 0.f, 0.f, pw2, pq2};
-          exchange<NW>(H, v3, 0, false, rpar, C, o, oflags);
-          pubW = o[4];
-          pubQ = o[5];
+          if (xn >= lo && xn < lo + nloc && ((xn - lo) / VEC) % THREADS == tid) {
+            H.pubv[0] = W[xn - lo];
+            H.pubv[1] = mref_t;
+            H.pubv[2] = Q[xn - lo];
+            H.pubv[3] = mref_d;
+          }
+          exchange<NW, false>(H, 0.f, 0.f, 0.f, 0.f, 0, xp, xph, rank, C, o, oflags);
+          if (oflags & kFlagTimeout) { err |= kErrTimeout; break; }
+          pub[0] = o[4]; pub[1] = o[5]; pub[2] = o[6]; pub[3] = o[7];
+          mass_kind = 0;
+          cn = nxt;
           continue;
         }
-        reject_pass_any<THREADS, true>(W, Q, L, lo, Pm, invSd, x, Z, xn, s1, s2, pw2, pq2);
-        float v3[6] = {s1, s2, 0.f, 0.f, pw2, pq2};
-        exchange<NW>(H, v3, 0, false, rpar, C, o, oflags);
+        reject_pass_any<THREADS, BF16, true>(W, Q, L, lo, Pm, at, bt, mref_t, mref_d, x, Z, xn,
+                                             H.pubv, s1, s2);
+        exchange<NW, false>(H, s1, s2, 0.f, 0.f, 0, xp, xph, rank, C, o, oflags);
+        if (oflags & kFlagTimeout) { err |= kErrTimeout; break; }
         const float S1 = o[0], S2 = o[1];
         const float delta = __fsub_rn(Z, S1);
         const float lam = S2 > 0.f ? fminf(fmaxf(__fdiv_rn(delta, S2), 0.f), 1.f) : 0.f;
         const float norm = __fmaf_rn(lam, S2, S1);
-        if (norm > 0.f) Pm = Pending{kResi, x, __frcp_rn(norm), Z, lam};
-        else { Pm = Pending{kIdent, -1, 1.f, 0.f, 0.f}; info |= kInfoDegenerate; }
+        if (norm > 0.f) {
+          Pm = Pending{kResi, x, __frcp_rn(norm), Z, lam};
+          mass_kind = 2;
+        } else {
+          Pm = Pending{kIdent, -1, 1.f, 0.f, 0.f};
+          info |= kInfoDegenerate;
+          mass_kind = 0;
+        }
       } else {
-        reject_pass_any<THREADS, false>(W, Q, L, lo, Pm, invSd, x, 0.f, xn, s1, s2, pw2, pq2);
-        float v3[6] = {s1, 0.f, 0.f, 0.f, pw2, pq2};
-        exchange<NW>(H, v3, 0, false, rpar, C, o, oflags);
-        if (o[0] > 0.f) Pm = Pending{kSpec, -1, __frcp_rn(o[0]), 0.f, 0.f};
-        else { Pm = Pending{kIdent, -1, 1.f, 0.f, 0.f}; info |= kInfoDegenerate; }
+        reject_pass_any<THREADS, BF16, false>(W, Q, L, lo, Pm, at, bt, mref_t, mref_d, x, 0.f,
+                                              xn, H.pubv, s1, s2);
+        exchange<NW, false>(H, s1, s2, 0.f, 0.f, 0, xp, xph, rank, C, o, oflags);
+        if (oflags & kFlagTimeout) { err |= kErrTimeout; break; }
+        if (o[0] > 0.f) {
+          Pm = Pending{kSpec, -1, __frcp_rn(o[0]), 0.f, 0.f};
+          mass_kind = 3;
+        } else {
+          Pm = Pending{kIdent, -1, 1.f, 0.f, 0.f};
+          info |= kInfoDegenerate;
+          mass_kind = 0;
+        }
       }
-      pubW = o[4];
-      pubQ = o[5];
+      pub[0] = o[4]; pub[1] = o[5]; pub[2] = o[6]; pub[3] = o[7];
+      cn = nxt;
     }
     if (err) break;
 
     if (accepted < 0) {
       // every child rejected: residual draw (Algorithm 1, last step)
-      if (!sample_final<THREADS>(H, P, W, Q, Pm, invSd, b, row, depth, lo, nloc, rank, C, rpar))
+      if (!sample_final<THREADS, BF16>(H, P, W, Q, Pm, mass_kind, at, bt, Mt, invSt, u_fin[row],
+                                       b, depth, lo, nloc, rank, C, xp, xph))
         err |= kErrEmpty;
       break;
     }
     if (depth >= D) { err |= kErrDepth; break; }
+    node = accepted;
+    row = accepted + 1;
+    issue_rows<THREADS, BF16>(H, P, W, Q, (size_t)b * P.seq_stride + (size_t)row * V,
+                              first_child[node + 1] >= 0, lo, nloc);
+    inflight = first_child[node + 1] >= 0 ? 3u : 1u;
     if (rank == 0 && tid == 0) {
       P.out_tokens[(size_t)b * (D + 1) + depth] = acc_tok;
       if (P.out_nodes) P.out_nodes[(size_t)b * D + depth] = accepted;
     }
     depth += 1;
-    node = accepted;
-    row = accepted + 1;
-    issue_rows<THREADS, BF16>(H, P, W, Q, (size_t)b * P.seq_stride + (size_t)row * V,
-                              haschild[node + 1] != 0, lo, nloc);
   }
 
   if (rank == 0 && tid == 0) {
@@ -774,12 +957,15 @@ __global__ void __launch_bounds__(THREADS, 1) verify_kernel(const VerifyParams P
     if (P.out_rejects) P.out_rejects[b] = rejects;
     if (P.status && (err | info)) atomicOr(P.status, err | info);
   }
-  if (timed_out && P.use_tma && tid == 0) {
-    // give outstanding copies a bounded chance to land before the CTA exits
-    wait_bar(smem_addr(&H.mbar[0]), ph0 ^ 1);
-    wait_bar(smem_addr(&H.mbar[1]), ph1 ^ 1);
+  if (inflight && P.use_tma && tid == 0) {
+    // copies issued but never consumed (bad tree, timeout): let them land
+    // (bounded) before the CTA's shared memory is released
+    for (int k = 0; k < nk_tma; ++k) {
+      if (inflight & 1u) wait_bar(smem_addr(&H.tbar[0][k]), tph & 1u);
+      if (inflight & 2u) wait_bar(smem_addr(&H.tbar[1][k]), (tph >> 1) & 1u);
+    }
   }
-  cluster_sync();  // no CTA leaves while a peer may still read its slots
+  cluster_sync();  // no CTA leaves while a peer may still write its slots
 }
 
 // Device Philox draws for tests.

@@ -2,13 +2,17 @@
 oracle on the same seeded inputs and compare them.
 
 Parity rule (the tolerances of the verification hot path):
-  * a sequence is "near tie" when the oracle saw an accept test with
-    |u - R(x)/q(x)| <= 1e-5 or a final draw whose relative CDF margin is
-    <= 1e-6; near-tie sequences are counted, not compared;
-  * every other sequence: accepted tokens, accept length, accepted node ids,
-    rejection count and the final token are bit-exact;
-  * the distribution of the final draw agrees within 1e-6 max-abs and 1e-5
-    L1 per row, and the GPU row sums to 1 within 1e-6.
+  * every sequence is compared: accepted tokens, accept length, accepted
+    node ids, rejection count and the final token must be bit-exact;
+  * a difference is allowed only for a sequence where the oracle saw a near
+    tie: an accept test with |u - R(x)/q(x)| <= 1e-5, or a final draw whose
+    relative CDF margin is <= 1e-6 (the fp32 distribution the kernel draws
+    from carries about 1e-7 relative rounding per probability, so a margin
+    below that bound can legitimately fall either way); such differences
+    are counted and reported;
+  * the distribution of the final draw (for every sequence whose path
+    matches) agrees within 1e-6 max-abs and 1e-5 L1 per row, and the GPU
+    row sums to 1 within 1e-6.
     SpecInfer residuals are the one exception: each rejection divides
     (R - q)_+ by its mass S_j, so an fp32 rounding of p or q (about 1e-7
     relative, the floor of any fp32 normaliser) reaches the residual
@@ -76,30 +80,28 @@ def run_oracle(target_h, draft_h, parents_h, cand_h, T, seed, max_depth, mode, s
 
 def compare(g, o, rows=None, check_dist=True):
     """Compare GPU outputs g (rows `rows` of the batch, or all) with oracle
-    outputs o.  Returns (n_compared, n_near_tie)."""
+    outputs o.  Returns (n_compared, n_near_tie_mismatches)."""
     idx = np.arange(len(o["accept_len"])) if rows is None else np.asarray(rows)
     sel = lambda a: a[idx]
     near = (o["accept_margin"] <= ACCEPT_TIE) | (o["sample_margin"] <= SAMPLE_TIE)
     errs = (o["status"] & ~oracle.INFO_DEGENERATE) != 0
-    clean = ~near
     gl, ol = sel(g["accept_len"]), o["accept_len"]
-    bad = np.nonzero(clean & (gl != ol))[0]
-    assert bad.size == 0, f"accept_len differs at {bad[:10]}: gpu {gl[bad[:10]]} oracle {ol[bad[:10]]}"
     gt, ot = sel(g["tokens"]), o["tokens"]
-    bad = np.nonzero(clean & (gt != ot).any(axis=1))[0]
-    assert bad.size == 0, f"tokens differ at {bad[:5]}: gpu {gt[bad[:5]]} oracle {ot[bad[:5]]}"
+    same_path = gl == ol
     if "nodes" in g and o["nodes"].shape[1]:
         gn = sel(g["nodes"])[:, : o["nodes"].shape[1]]
-        bad = np.nonzero(clean & (gn != o["nodes"]).any(axis=1))[0]
-        assert bad.size == 0, f"nodes differ at {bad[:5]}"
+        same_path &= (gn == o["nodes"]).all(axis=1)
     if "rejects" in g:
-        gr = sel(g["rejects"])
-        ok = clean & ~errs
-        bad = np.nonzero(ok & (gr != o["rejects"]))[0]
-        assert bad.size == 0, f"rejects differ at {bad[:5]}: {gr[bad[:5]]} vs {o['rejects'][bad[:5]]}"
+        same_path &= errs | (sel(g["rejects"]) == o["rejects"])
+    differs = ~same_path | (gt != ot).any(axis=1)
+    bad = np.nonzero(differs & ~near)[0]
+    assert bad.size == 0, (f"{bad.size} sequences differ without a near tie, e.g. {bad[:5]}: "
+                           f"gpu len {gl[bad[:5]]} tokens {gt[bad[:3]]}; "
+                           f"oracle len {ol[bad[:5]]} tokens {ot[bad[:3]]}; "
+                           f"margins {o['accept_margin'][bad[:5]]} {o['sample_margin'][bad[:5]]}")
     if check_dist and "dist" in g and "dist" in o:
         gd = sel(g["dist"]).astype(np.float64)
-        ok = clean & ~errs
+        ok = same_path & ~errs
         if ok.any():
             diff = np.abs(gd[ok] - o["dist"][ok])
             scale = np.maximum(1.0, o["cond"][ok])
@@ -110,4 +112,4 @@ def compare(g, o, rows=None, check_dist=True):
             sums = gd[ok].sum(axis=1)
             assert np.abs(sums - 1).max() <= 1e-6, f"residual sum off by {np.abs(sums - 1).max():.3e}"
             assert (gd[ok] >= 0).all()
-    return int(clean.sum()), int(near.sum())
+    return int(len(idx)), int((differs & near).sum())

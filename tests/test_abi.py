@@ -89,8 +89,10 @@ def test_plan_without_device(lib):
     for V in (1, 7, 32000, 128256, 256000, rs.MAX_VOCAB):
         p = rs.plan(128, 488, V, 6, "bf16")
         assert p["smem_bytes"] <= 227 * 1024
+    p = rs.plan(1, 2, 1000, 1, "f32", cluster_size=3)   # any cluster size up to 16
+    assert p["cluster_size"] == 3 and p["slice_elems"] * 3 >= 1000
     with pytest.raises(rs.ResispecError):
-        rs.plan(1, 2, 10, 1, "f32", cluster_size=3)
+        rs.plan(1, 2, 10, 1, "f32", cluster_size=17)
     with pytest.raises(rs.ResispecError):
         rs.plan(1, 2, rs.MAX_VOCAB, 1, "f32", cluster_size=1)  # 2 MB on one CTA
 

@@ -28,14 +28,15 @@ def _np_inputs_to_gpu(inp):
             torch.as_tensor(inp["cand"], dtype=torch.int32, device="cuda"))
 
 
-def _check(inp, mode, seed, near_frac=0.01, **kw):
+def _check(inp, mode, seed, **kw):
     zt, zd, pa, ca = _np_inputs_to_gpu(inp)
     D = int(inp["max_depth"])
     g = P.run_gpu(zt, zd, pa, ca, inp["temperature"], seed, D, mode=mode, **kw)
     o = P.run_oracle(inp["target"], inp["draft"], inp["parents"], inp["cand"],
                      inp["temperature"], seed, D, mode)
     n, near = P.compare(g, o)
-    assert near <= max(2, near_frac * len(o["accept_len"])), (near, n)
+    # near-tie differences are allowed but must stay rare
+    assert near <= max(2, 0.002 * n), (near, n)
     assert g["status"][0] & ~rs.INFO_DEGENERATE == 0
     return g, o
 
@@ -100,7 +101,7 @@ def test_parity_ragged_vocab(V, dtype, no_tma):
     base = W.Workload(name="ragged", batch=64, vocab=V, dtype=dtype, gen="gauss", scale=2.0,
                       slope=0.0, rho=0.6, temperature=0.9, tree=("levels", (3, 2, 1)), steps=1)
     inp = W.make_inputs_np(base, seed=V, batch=64)
-    for cluster in (0, 4, 16):
+    for cluster in (0, 4, 11, 16):
         for mode in MODES:
             _check(inp, mode, seed=V + cluster, cluster_size=cluster, no_tma=no_tma)
 
@@ -110,7 +111,7 @@ def test_launch_shapes_agree(threads):
     w = W.WORKLOADS["tree60-v32000"]
     inp = W.make_inputs_np(w, seed=2, batch=64)
     ref = None
-    for cluster in (1, 2, 4, 8, 16):
+    for cluster in (2, 3, 4, 8, 12, 16):   # one CTA cannot hold two V = 32000 fp32 rows
         g, o = _check(inp, rs.MODE_RESISPEC, seed=3, cluster_size=cluster, block_threads=threads)
         clean = (o["accept_margin"] > P.ACCEPT_TIE) & (o["sample_margin"] > P.SAMPLE_TIE)
         if ref is not None:
@@ -167,7 +168,7 @@ def test_shared_rows_seq_stride_zero():
 def test_error_contract_matches_oracle():
     import torch
     parents = W.tree_levels([2, 2])
-    V, B = 1024, 8
+    V, B = 1024, 9
     rng = np.random.default_rng(1)
     zt = rng.normal(0, 1, (B, 7, V)).astype(np.float32)
     zd = zt.copy()
@@ -178,12 +179,15 @@ def test_error_contract_matches_oracle():
     zt[3, 0, :] = -np.inf
     zt[4, 6, 0] = np.nan              # never visited
     zd[6, 0, 100] = np.inf
+    zt[8, 0, :] = -np.inf             # NaN hidden among -inf logits
+    zt[8, 0, 517] = np.nan
     g = P.run_gpu(P.to_device(zt), P.to_device(zd), torch.as_tensor(parents, device="cuda"),
                   torch.as_tensor(cand, device="cuda"), 1.0, 0, 2, want_dist=False)
     o = P.run_oracle(zt, zd, parents, cand, 1.0, 0, 2, rs.MODE_RESISPEC, want_dist=False)
     np.testing.assert_array_equal(g["accept_len"] == -1, o["accept_len"] == -1)
-    assert list(np.nonzero(o["accept_len"] == -1)[0]) == [1, 2, 3, 5, 6]
-    assert (g["tokens"][[1, 2, 3, 5, 6]] == -1).all()
+    assert list(np.nonzero(o["accept_len"] == -1)[0]) == [1, 2, 3, 5, 6, 8]
+    assert o["status"][8] == oracle.ERR_NONFINITE
+    assert (g["tokens"][[1, 2, 3, 5, 6, 8]] == -1).all()
     want = int(np.bitwise_or.reduce(o["status"]))
     assert g["status"][0] & ~rs.INFO_DEGENERATE == want & ~oracle.INFO_DEGENERATE
     # depth overflow and a tree that is not in topological order
@@ -204,7 +208,7 @@ def test_synchronous_errors_on_device():
     with pytest.raises(rs.ResispecError):
         rs.verify(t, t, pa, ca, 0.0, 0, max_depth=1)
     with pytest.raises(rs.ResispecError):
-        rs.verify(t, t, pa, ca, 1.0, 0, max_depth=1, cluster_size=3)
+        rs.verify(t, t, pa, ca, 1.0, 0, max_depth=1, cluster_size=17)
 
 
 def test_nondefault_stream():
@@ -241,7 +245,7 @@ def _sampled_parity(w, seed, call_seed, rows, mode=rs.MODE_RESISPEC, batch=None,
     o = P.run_oracle(th, dh, inp["parents_np"], ch, w.temperature, call_seed, D, mode,
                      seq_ids=np.asarray(rows, np.int32))
     n, near = P.compare(g, o, rows=rows)
-    assert near <= 1
+    assert near <= 1, near
     assert g["status"][0] & ~rs.INFO_DEGENERATE == 0
     assert (g["accept_len"] >= 0).all()
     del inp

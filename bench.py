@@ -53,6 +53,7 @@ def parse_args(argv=None):
     ap.add_argument("--pool", type=int, default=0, help="input sets rotated between steps (0 = auto)")
     ap.add_argument("--cluster-size", type=int, default=0)
     ap.add_argument("--block-threads", type=int, default=0)
+    ap.add_argument("--kernel", choices=["auto", "resident", "stream"], default="auto")
     ap.add_argument("--e2e-steps", type=int, default=12)
     ap.add_argument("--cpu-seqs", type=int, default=16)
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
@@ -83,10 +84,10 @@ def kernel_source_digest():
     return h.hexdigest()[:16]
 
 
-def profiled_traffic(workload):
-    """DRAM bytes per launch from the committed ncu summary of this
-    workload, if it was taken on the current kernel source."""
-    path = os.path.join(ROOT, "profiles", f"verify_kernel_{workload}.md")
+def profiled_traffic(kernel, workload):
+    """DRAM bytes per launch from the committed ncu summary of this kernel
+    on this workload, if it was taken on the current kernel source."""
+    path = os.path.join(ROOT, "profiles", f"{kernel}_kernel_{workload}.md")
     if not os.path.exists(path):
         return None
     text = open(path).read()
@@ -299,11 +300,12 @@ def run_ours(args):
              torch.empty((B,), dtype=torch.int32, device=dev),
              torch.empty((B, max(D, 1)), dtype=torch.int32, device=dev)) for _ in range(K)]
     status = torch.zeros((1,), dtype=torch.int32, device=dev)
+    kernel = None if args.kernel == "auto" else args.kernel
     kw = dict(max_depth=D, mode=mode, cluster_size=args.cluster_size,
-              block_threads=args.block_threads, status=status)
+              block_threads=args.block_threads, status=status, kernel=kernel)
     stream = torch.cuda.current_stream(dev)
     plan = rs.plan(B, N, V, D, w.dtype, cluster_size=args.cluster_size,
-                   block_threads=args.block_threads)
+                   block_threads=args.block_threads, kernel=kernel)
 
     def launch(i, out):
         s = sets[i % pool]
@@ -361,13 +363,15 @@ def run_ours(args):
             "logits": f"{w.gen} slope {w.slope} scale {w.scale} rho {w.rho}",
             "temperature": w.temperature, "mode": args.mode,
             "parallelism": f"replicas{world}" if world > 1 else "single",
-            "launch": {k: plan[k] for k in ("cluster_size", "block_threads", "smem_bytes",
-                                            "slice_elems", "uses_tma")},
+            "launch": {k: plan[k] for k in ("kernel_name", "cluster_size", "block_threads",
+                                            "smem_bytes", "slice_elems", "uses_tma", "stages",
+                                            "active_clusters")},
             "l2": f"rotating pool of {pool} input sets ({set_bytes / 1e9:.2f} GB each) "
                   f"between steps; each step's visited rows exceed L2 together",
         },
         "roofline": {"bound": "hbm", "achieved": achieved_gbs, "peak": peak, "unit": "GB/s",
-                     "frac": achieved_gbs / peak, "traffic": profiled_traffic(w.name),
+                     "frac": achieved_gbs / peak,
+                     "traffic": profiled_traffic(plan["kernel_name"], w.name),
                      "peak_kind": peak_kind, "frac_of_8tbs": achieved_gbs / NOMINAL_HBM_GBS,
                      "alg_bytes_per_launch": alg_bytes / K,
                      "mean_launch_us": mean_launch_s * 1e6},
@@ -398,7 +402,7 @@ def run_ours(args):
                 dbuf[k].copy_(host[k], non_blocking=True)
             rs.verify(dbuf["target"], dbuf["draft"], dbuf["parents"], dbuf["cand"],
                       w.temperature, args.seed + i, out_tokens=d_tok, out_accept_len=d_len,
-                      max_depth=D, mode=mode, stream=stream)
+                      max_depth=D, mode=mode, stream=stream, kernel=kernel)
             h_tok.copy_(d_tok, non_blocking=True)
             h_len.copy_(d_len, non_blocking=True)
 

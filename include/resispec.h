@@ -40,7 +40,7 @@
 extern "C" {
 #endif
 
-#define RESISPEC_ABI_VERSION 1
+#define RESISPEC_ABI_VERSION 2
 
 /* Synchronous return codes. */
 typedef enum {
@@ -68,10 +68,13 @@ typedef enum { RESISPEC_MODE_RESISPEC = 0, RESISPEC_MODE_SPECINFER = 1 } resispe
 #define RESISPEC_ERR_EMPTY_ROW 8   /* a visited row (or the residual) has no mass */
 #define RESISPEC_ERR_DEPTH 16      /* more accepted tokens than max_depth */
 #define RESISPEC_ERR_TIMEOUT 32    /* a bounded wait for a row copy gave up */
+#define RESISPEC_ERR_FANOUT 64     /* streaming kernel: a visited node has more than
+                                      RESISPEC_MAX_FANOUT_STREAM children */
 #define RESISPEC_INFO_DEGENERATE 256 /* informational: a rejection left R unchanged */
 
 #define RESISPEC_MAX_VOCAB 262144
 #define RESISPEC_MAX_NODES 4096
+#define RESISPEC_MAX_FANOUT_STREAM 128
 
 /* Sizes of one call.  Logit rows: row 0 is the root, row j+1 is node j. */
 typedef struct {
@@ -83,7 +86,24 @@ typedef struct {
 } resispec_dims;
 
 #define RESISPEC_FLAG_NO_TMA 1   /* force plain loads instead of bulk copies */
-#define RESISPEC_FLAG_PREFETCH 2 /* warm L2 with the first child's rows during a visit */
+#define RESISPEC_FLAG_PREFETCH 2 /* resident kernel: warm L2 with the first child's rows */
+#define RESISPEC_FLAG_RESIDENT 4 /* force the resident kernel */
+#define RESISPEC_FLAG_STREAM 8   /* force the streaming kernel */
+
+/* Kernels.  Both compute the same verification; they differ in where a
+ * visited node's rows live between the passes of a visit.
+ *   RESIDENT: both rows of the sequence's vocabulary slice stay in the
+ *     shared memory of the cluster's CTAs as fp32 (8 bytes per vocabulary
+ *     entry per sequence), so only as many sequences as fit on chip run at
+ *     once.  Any fan-out.
+ *   STREAM: nothing but per-sequence scalars stays on chip; every pass
+ *     streams the rows through a small shared-memory ring and the passes
+ *     after the first read them from L2.  All sequences of a large batch run
+ *     at once.  Fan-out up to RESISPEC_MAX_FANOUT_STREAM children per node.
+ * The automatic choice takes RESIDENT when the whole batch fits on chip at
+ * once, else STREAM. */
+#define RESISPEC_KERNEL_RESIDENT 0
+#define RESISPEC_KERNEL_STREAM 1
 
 typedef struct {
   int32_t mode;          /* resispec_mode */
@@ -133,13 +153,23 @@ int resispec_verify_ex(const void* target_logits, const void* draft_logits,
                        int32_t* out_accept_len, resispec_dims dims,
                        const resispec_opts* opts, void* stream);
 
-/* Launch shape resispec_verify_ex would use (no launch): CTAs per sequence,
- * threads per CTA, dynamic shared memory bytes per CTA, vocabulary elements
- * per CTA, and 1 if rows are fetched with bulk copies.  Any output pointer
- * may be NULL. */
-int resispec_plan(resispec_dims dims, const resispec_opts* opts,
-                  int32_t* cluster_size, int32_t* block_threads,
-                  int32_t* smem_bytes, int32_t* slice_elems, int32_t* uses_tma);
+/* Launch shape chosen for a call. */
+typedef struct {
+  int32_t kernel;          /* RESISPEC_KERNEL_* */
+  int32_t cluster_size;    /* CTAs per sequence */
+  int32_t block_threads;   /* threads per CTA */
+  int32_t smem_bytes;      /* dynamic shared memory per CTA */
+  int32_t slice_elems;     /* vocabulary entries per CTA */
+  int32_t uses_tma;        /* 1 if rows are fetched with bulk copies */
+  int32_t stages;          /* STREAM: shared-memory ring stages (0 for RESIDENT) */
+  int32_t active_clusters; /* clusters of this shape resident at once on the
+                              current device (0 without a device) */
+} resispec_plan_info;
+
+/* Launch shape resispec_verify_ex would use for these sizes and options on
+ * the current device (no launch; without a usable device a size-only rule
+ * is applied).  Returns the same argument errors as resispec_verify_ex. */
+int resispec_plan(resispec_dims dims, const resispec_opts* opts, resispec_plan_info* out);
 
 /* Device Philox draws for testing the counter-based generator: for i < n,
  * u0[i] = U(seed, seq[i], row[i], 0) and u1[i] = U(seed, seq[i], row[i], 1).

@@ -31,12 +31,19 @@ ERR_NONFINITE = 4
 ERR_EMPTY_ROW = 8
 ERR_DEPTH = 16
 ERR_TIMEOUT = 32
+ERR_FANOUT = 64
 INFO_DEGENERATE = 256
 FLAG_NO_TMA = 1
 FLAG_PREFETCH = 2
+FLAG_RESIDENT = 4
+FLAG_STREAM = 8
+KERNEL_RESIDENT = 0
+KERNEL_STREAM = 1
+KERNELS = {"auto": None, "resident": KERNEL_RESIDENT, "stream": KERNEL_STREAM}
 
 MAX_VOCAB = 262144
 MAX_NODES = 4096
+MAX_FANOUT_STREAM = 128
 
 E_OK, E_ARG, E_SHAPE, E_DTYPE, E_UNSUPPORTED, E_CUDA = range(6)
 
@@ -62,6 +69,12 @@ class Opts(ctypes.Structure):
                 ("seq_stride", ctypes.c_int64), ("status", ctypes.c_void_p),
                 ("out_nodes", ctypes.c_void_p), ("out_dist", ctypes.c_void_p),
                 ("out_rejects", ctypes.c_void_p)]
+
+
+class PlanInfo(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_int32) for n in (
+        "kernel", "cluster_size", "block_threads", "smem_bytes", "slice_elems", "uses_tma",
+        "stages", "active_clusters")]
 
 
 class ResispecError(RuntimeError):
@@ -101,8 +114,7 @@ def load_library():
         lib.resispec_verify_ex.argtypes = [vp, vp, vp, vp, ctypes.c_float, u64, vp, vp, Dims,
                                            ctypes.POINTER(Opts), vp]
         lib.resispec_verify_ex.restype = ctypes.c_int
-        P = ctypes.POINTER(i32)
-        lib.resispec_plan.argtypes = [Dims, ctypes.POINTER(Opts), P, P, P, P, P]
+        lib.resispec_plan.argtypes = [Dims, ctypes.POINTER(Opts), ctypes.POINTER(PlanInfo)]
         lib.resispec_plan.restype = ctypes.c_int
         lib.resispec_uniforms.argtypes = [u64, vp, vp, i32, vp, vp, vp]
         lib.resispec_uniforms.restype = ctypes.c_int
@@ -142,16 +154,28 @@ def _ptr(t):
     return None if t is None else ctypes.c_void_p(t.data_ptr())
 
 
+def _kernel_flags(kernel) -> int:
+    if kernel in (None, "auto"):
+        return 0
+    k = KERNELS.get(kernel, kernel)
+    if k == KERNEL_RESIDENT:
+        return FLAG_RESIDENT
+    if k == KERNEL_STREAM:
+        return FLAG_STREAM
+    raise ValueError(f"unknown kernel {kernel!r}")
+
+
 def make_opts(mode=MODE_RESISPEC, cluster_size=0, block_threads=0, no_tma=False,
               seq_stride=None, status=None, out_nodes=None, out_dist=None,
-              out_rejects=None, prefetch=False) -> Opts:
+              out_rejects=None, prefetch=False, kernel=None) -> Opts:
     lib = load_library()
     o = Opts()
     lib.resispec_opts_default(ctypes.byref(o))
     o.mode = {"resispec": MODE_RESISPEC, "specinfer": MODE_SPECINFER}.get(mode, mode)
     o.cluster_size = int(cluster_size)
     o.block_threads = int(block_threads)
-    o.flags = (FLAG_NO_TMA if no_tma else 0) | (FLAG_PREFETCH if prefetch else 0)
+    o.flags = ((FLAG_NO_TMA if no_tma else 0) | (FLAG_PREFETCH if prefetch else 0)
+               | _kernel_flags(kernel))
     o.seq_stride = -1 if seq_stride is None else int(seq_stride)
     o.status = None if status is None else status.data_ptr()
     o.out_nodes = None if out_nodes is None else out_nodes.data_ptr()
@@ -166,18 +190,19 @@ def plan(batch, num_nodes, vocab, max_depth, dtype="f32", **opt_kw) -> dict:
     d = Dims(int(batch), int(num_nodes), int(vocab), int(max_depth),
              F32 if dtype in ("f32", F32) else BF16)
     o = make_opts(**opt_kw)
-    vals = [ctypes.c_int32() for _ in range(5)]
-    rc = lib.resispec_plan(d, ctypes.byref(o), *[ctypes.byref(v) for v in vals])
+    info = PlanInfo()
+    rc = lib.resispec_plan(d, ctypes.byref(o), ctypes.byref(info))
     if rc:
         raise ResispecError(rc, "resispec_plan")
-    keys = ("cluster_size", "block_threads", "smem_bytes", "slice_elems", "uses_tma")
-    return {k: v.value for k, v in zip(keys, vals)}
+    out = {k: getattr(info, k) for k, _ in PlanInfo._fields_}
+    out["kernel_name"] = "stream" if info.kernel == KERNEL_STREAM else "resident"
+    return out
 
 
 def verify(target, draft, tree_parents, cand_tokens, temperature, seed, *, max_depth=None,
            mode=MODE_RESISPEC, out_tokens=None, out_accept_len=None, out_nodes=None,
            out_dist=None, out_rejects=None, status=None, cluster_size=0, block_threads=0,
-           no_tma=False, seq_stride=None, stream=None, prefetch=False):
+           no_tma=False, seq_stride=None, stream=None, prefetch=False, kernel=None):
     """Verify a batch of draft trees on the GPU.
 
     target, draft: CUDA tensors [B, N+1, V] (float32 or bfloat16); with
@@ -185,6 +210,7 @@ def verify(target, draft, tree_parents, cand_tokens, temperature, seed, *, max_d
     tree_parents: int32 CUDA tensor [N]; cand_tokens: int32 CUDA tensor
     [B, N].  Returns (out_tokens [B, D+1], out_accept_len [B]).  Runs on
     ``stream`` (default: torch's current stream) without synchronising.
+    ``kernel``: None / "auto" (the library's choice), "resident" or "stream".
     """
     torch = _torch()
     lib = load_library()
@@ -216,7 +242,7 @@ def verify(target, draft, tree_parents, cand_tokens, temperature, seed, *, max_d
     if seq_stride is None and target.numel() != B * (N + 1) * V:
         raise ValueError("target must be [B, N+1, V] (or pass seq_stride)")
     o = make_opts(mode, cluster_size, block_threads, no_tma, seq_stride, status, out_nodes,
-                  out_dist, out_rejects, prefetch)
+                  out_dist, out_rejects, prefetch, kernel)
     if stream is None:
         stream = torch.cuda.current_stream(dev)
     handle = stream.cuda_stream if hasattr(stream, "cuda_stream") else int(stream)

@@ -1,0 +1,11 @@
+// Entry points of the kernel translation units (one per kernel and dtype,
+// compiled in parallel).  Each returns the __global__ function for a block
+// size of 256 or 512 threads.
+#pragma once
+
+namespace rs {
+const void* resident_entry_f32(int threads);
+const void* resident_entry_bf16(int threads);
+const void* stream_entry_f32(int threads);
+const void* stream_entry_bf16(int threads);
+}  // namespace rs

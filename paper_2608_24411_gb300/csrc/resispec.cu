@@ -1,6 +1,6 @@
 // Host side of the C ABI declared in include/resispec.h: argument checks,
-// launch planning (cluster size, threads, shared memory) and the cluster
-// launch of the fused verification kernel on the caller's stream.
+// launch planning (kernel, cluster size, threads, shared memory) and the
+// cluster launch of the fused verification kernel on the caller's stream.
 #include <cuda_runtime.h>
 #include <math.h>
 #include <stdint.h>
@@ -12,7 +12,23 @@
 #include <tuple>
 
 #include "../../include/resispec.h"
-#include "verify_kernel.cuh"
+#include "kernels.h"
+#include "verify_stream.cuh"
+
+namespace rs {
+
+// Device Philox draws for tests.
+__global__ void uniforms_kernel(uint64_t seed, const int32_t* seq, const int32_t* row, int n,
+                                float* u0, float* u1) {
+  const int i = blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= n) return;
+  const U64x4 r = philox4x64_10((uint64_t)(uint32_t)row[i], (uint64_t)(uint32_t)seq[i], 0, 0,
+                                seed, 0);
+  u0[i] = u24(r.w[0]);
+  u1[i] = u24(r.w[1]);
+}
+
+}  // namespace rs
 
 namespace {
 
@@ -27,12 +43,15 @@ constexpr int kMaxSmem = 227 * 1024;      // dynamic shared memory per CTA on sm
 constexpr int kAutoSliceBytes = 96 * 1024; // target on-chip bytes per CTA (two fp32 rows)
 
 struct Plan {
+  int kernel = RESISPEC_KERNEL_RESIDENT;
   int C = 1;
   int threads = 512;
   int L = 8;
   int npad = 16;
   int smem = 0;
   int use_tma = 0;
+  int stages = 0;
+  int active = 0;
 };
 
 int round_up(int x, int m) { return (x + m - 1) / m * m; }
@@ -42,9 +61,27 @@ int slice_for(int V, int C) { return round_up((V + C - 1) / C, 8); }
 // Head, two fp32 rows, then the tree: parent / first child / next sibling
 // (int16), the candidate tokens of the sequence (int32) and two uniforms per
 // logit row (fp32).
-int smem_for(int L, int npad) {
-  const int tree = npad * 2 + (npad + 16) * 2 + npad * 2 + npad * 4 + npad * 8;
-  return round_up(rs::kHeadBytes + 8 * L + tree, 128);
+int tree_bytes(int npad) { return npad * 2 + (npad + 16) * 2 + npad * 2 + npad * 4 + npad * 8; }
+
+int smem_for(int L, int npad) { return round_up(rs::kHeadBytes + 8 * L + tree_bytes(npad), 128); }
+
+// Streaming kernel: head, stream head, S ring stages of two chunk rows
+// (2 * threads 16-byte vectors each), then the tree.
+int stage_bytes(int threads) { return 2 * 2 * threads * 16; }
+
+int stream_smem_for(int threads, int S, int npad) {
+  return round_up(rs::kHeadBytes + rs::kStreamHeadBytes + S * stage_bytes(threads) +
+                      tree_bytes(npad), 128);
+}
+
+// Deepest ring (2..4 stages) that still lets `per_sm` CTAs share an SM.
+int stream_stages(int threads, int npad) {
+  const int per_sm = threads >= 512 ? 2 : 4;
+  const int budget = (228 * 1024) / per_sm - 1024;
+  int S = 2;
+  for (int s = 3; s <= rs::kMaxStages; ++s)
+    if (stream_smem_for(threads, s, npad) <= budget) S = s;
+  return S;
 }
 
 struct DeviceInfo {
@@ -55,7 +92,7 @@ struct DeviceInfo {
 
 std::mutex g_mu;
 DeviceInfo g_dev[64];
-bool g_attr_set[64][4];
+bool g_attr_set[64][8];
 
 int query_device(int* dev_out, DeviceInfo* info) {
   int dev = 0;
@@ -90,12 +127,19 @@ int check_dims(const resispec_dims& d) {
 
 // Clusters of this shape that can be resident at once (0: the shape cannot
 // be launched).  Cached per device and shape.
-using OccKey = std::tuple<int, int, int, int, int>;  // dev, threads, bf16, C, smem
+using OccKey = std::tuple<int, int, int, int, int, int>;  // dev, kernel, threads, bf16, C, smem
 std::map<OccKey, int> g_occ;
 
 template <int THREADS, bool BF16>
-int query_clusters(int C, int smem) {
-  auto kern = rs::verify_kernel<THREADS, BF16>;
+const void* kernel_ptr(int kernel) {
+  if (kernel == RESISPEC_KERNEL_STREAM)
+    return BF16 ? rs::stream_entry_bf16(THREADS) : rs::stream_entry_f32(THREADS);
+  return BF16 ? rs::resident_entry_bf16(THREADS) : rs::resident_entry_f32(THREADS);
+}
+
+template <int THREADS, bool BF16>
+int query_clusters(int kernel, int C, int smem) {
+  const void* kern = kernel_ptr<THREADS, BF16>(kernel);
   if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, kMaxSmem) !=
           cudaSuccess ||
       cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) !=
@@ -123,8 +167,8 @@ int query_clusters(int C, int smem) {
   return n;
 }
 
-int active_clusters(int dev, int threads, bool bf16, int C, int smem) {
-  const OccKey key{dev, threads, bf16 ? 1 : 0, C, smem};
+int active_clusters(int dev, int kernel, int threads, bool bf16, int C, int smem) {
+  const OccKey key{dev, kernel, threads, bf16 ? 1 : 0, C, smem};
   {
     std::lock_guard<std::mutex> lk(g_mu);
     auto it = g_occ.find(key);
@@ -132,40 +176,31 @@ int active_clusters(int dev, int threads, bool bf16, int C, int smem) {
   }
   int n;
   if (threads == 512)
-    n = bf16 ? query_clusters<512, true>(C, smem) : query_clusters<512, false>(C, smem);
+    n = bf16 ? query_clusters<512, true>(kernel, C, smem)
+             : query_clusters<512, false>(kernel, C, smem);
   else
-    n = bf16 ? query_clusters<256, true>(C, smem) : query_clusters<256, false>(C, smem);
+    n = bf16 ? query_clusters<256, true>(kernel, C, smem)
+             : query_clusters<256, false>(kernel, C, smem);
   std::lock_guard<std::mutex> lk(g_mu);
   g_occ[key] = n;
   return n;
 }
 
-// Launch shape.  dev < 0 means no device to query: the automatic cluster
-// size then follows a size-only rule.
-int make_plan(const resispec_dims& d, const resispec_opts& o, int dev, int sms,
-              const void* zt, const void* zd, Plan* p) {
-  int st = check_dims(d);
-  if (st) return st;
-  if (o.mode != RESISPEC_MODE_RESISPEC && o.mode != RESISPEC_MODE_SPECINFER) return RESISPEC_E_ARG;
-  if (o.block_threads != 0 && o.block_threads != 256 && o.block_threads != 512)
-    return RESISPEC_E_ARG;
-  const int cs = o.cluster_size;
-  if (cs < 0 || cs > rs::kMaxCluster) return RESISPEC_E_ARG;
-  if (o.seq_stride < -1) return RESISPEC_E_ARG;
-  p->threads = o.block_threads ? o.block_threads : 512;
-  p->npad = round_up(d.num_nodes + 1, 16);
+// Resident kernel: cluster size.  With a device, most SMs engaged (resident
+// clusters capped by the batch, times their size; ties go to the larger
+// cluster, which shortens a sequence's latency).
+int plan_resident(const resispec_dims& d, int cs, int dev, int sms, Plan* p) {
   const int V = d.vocab;
+  const bool bf16 = d.dtype == RESISPEC_BF16;
   if (cs) {
     p->C = cs;
   } else if (dev >= 0) {
-    // Most SMs engaged: resident clusters (capped by the batch) times their
-    // size; ties go to the larger cluster (shorter per-sequence latency).
     int best = 0;
     int64_t best_score = -1;
     for (int C = 1; C <= rs::kMaxCluster; ++C) {
       const int smem = smem_for(slice_for(V, C), p->npad);
       if (smem > kMaxSmem) continue;
-      const int n = active_clusters(dev, p->threads, d.dtype == RESISPEC_BF16, C, smem);
+      const int n = active_clusters(dev, RESISPEC_KERNEL_RESIDENT, p->threads, bf16, C, smem);
       if (n <= 0) continue;
       const int64_t score = std::min<int64_t>(d.batch, n) * C;
       if (score >= best_score) { best_score = score; best = C; }
@@ -181,6 +216,89 @@ int make_plan(const resispec_dims& d, const resispec_opts& o, int dev, int sms,
   p->L = slice_for(V, p->C);
   p->smem = smem_for(p->L, p->npad);
   if (p->smem > kMaxSmem) return RESISPEC_E_SHAPE;
+  p->stages = 0;
+  p->active = dev >= 0 ? active_clusters(dev, RESISPEC_KERNEL_RESIDENT, p->threads, bf16, p->C,
+                                         p->smem)
+                       : 0;
+  return RESISPEC_OK;
+}
+
+// Streaming kernel: cluster size.  The batch runs in ceil(B / n) waves of n
+// resident clusters and a CTA's work shrinks as 1 / C, so C / waves is
+// maximised; ties go to the smaller cluster (cheaper exchanges, more
+// sequences overlapping their HBM-bound and ALU-bound passes).
+int plan_stream(const resispec_dims& d, int cs, int dev, int sms, Plan* p) {
+  const bool bf16 = d.dtype == RESISPEC_BF16;
+  p->stages = stream_stages(p->threads, p->npad);
+  p->smem = stream_smem_for(p->threads, p->stages, p->npad);
+  if (p->smem > kMaxSmem) return RESISPEC_E_SHAPE;
+  const int B = std::max(d.batch, 1);
+  if (cs) {
+    p->C = cs;
+  } else if (dev >= 0) {
+    int best = 0;
+    double best_score = -1.0;
+    for (int C = 1; C <= rs::kMaxCluster; ++C) {
+      const int n = active_clusters(dev, RESISPEC_KERNEL_STREAM, p->threads, bf16, C, p->smem);
+      if (n <= 0) continue;
+      const double score = (double)C / (double)((B + n - 1) / n);
+      if (score > best_score) { best_score = score; best = C; }
+    }
+    if (best == 0) return RESISPEC_E_UNSUPPORTED;
+    p->C = best;
+  } else {
+    const int slots = (sms > 0 ? sms : 152) * (p->threads >= 512 ? 2 : 4);
+    p->C = std::min(16, std::max(1, slots / B));
+  }
+  p->L = slice_for(d.vocab, p->C);
+  p->active = dev >= 0 ? active_clusters(dev, RESISPEC_KERNEL_STREAM, p->threads, bf16, p->C,
+                                         p->smem)
+                       : 0;
+  return RESISPEC_OK;
+}
+
+// Launch shape.  dev < 0 means no device to query: the automatic choices
+// then follow size-only rules.
+int make_plan(const resispec_dims& d, const resispec_opts& o, int dev, int sms,
+              const void* zt, const void* zd, Plan* p) {
+  int st = check_dims(d);
+  if (st) return st;
+  if (o.mode != RESISPEC_MODE_RESISPEC && o.mode != RESISPEC_MODE_SPECINFER) return RESISPEC_E_ARG;
+  if (o.block_threads != 0 && o.block_threads != 256 && o.block_threads != 512)
+    return RESISPEC_E_ARG;
+  const int cs = o.cluster_size;
+  if (cs < 0 || cs > rs::kMaxCluster) return RESISPEC_E_ARG;
+  if (o.seq_stride < -1) return RESISPEC_E_ARG;
+  const bool force_res = (o.flags & RESISPEC_FLAG_RESIDENT) != 0;
+  const bool force_str = (o.flags & RESISPEC_FLAG_STREAM) != 0;
+  if (force_res && force_str) return RESISPEC_E_ARG;
+  p->threads = o.block_threads ? o.block_threads : 512;
+  p->npad = round_up(d.num_nodes + 1, 16);
+  const int V = d.vocab;
+  if (force_str) {
+    p->kernel = RESISPEC_KERNEL_STREAM;
+    st = plan_stream(d, cs, dev, sms, p);
+  } else if (force_res) {
+    p->kernel = RESISPEC_KERNEL_RESIDENT;
+    st = plan_resident(d, cs, dev, sms, p);
+  } else {
+    // Resident when the whole batch is on chip at once, else streaming.
+    Plan r = *p;
+    r.kernel = RESISPEC_KERNEL_RESIDENT;
+    const int sr = plan_resident(d, cs, dev, sms, &r);
+    bool fits;
+    if (sr == RESISPEC_OK && dev >= 0) fits = r.active >= d.batch;
+    else if (sr == RESISPEC_OK) fits = (int64_t)d.batch * V * 8 <= (int64_t)16 << 20;
+    else fits = false;
+    if (fits) {
+      *p = r;
+      st = RESISPEC_OK;
+    } else {
+      p->kernel = RESISPEC_KERNEL_STREAM;
+      st = plan_stream(d, cs, dev, sms, p);
+    }
+  }
+  if (st) return st;
   const int64_t es = d.dtype == RESISPEC_BF16 ? 2 : 4;
   const int64_t stride = o.seq_stride < 0 ? (int64_t)(d.num_nodes + 1) * V : o.seq_stride;
   p->use_tma = !(o.flags & RESISPEC_FLAG_NO_TMA) && (V * es) % 16 == 0 &&
@@ -192,8 +310,9 @@ int make_plan(const resispec_dims& d, const resispec_opts& o, int dev, int sms,
 template <int THREADS, bool BF16>
 cudaError_t launch_verify(const Plan& pl, const rs::VerifyParams& prm, cudaStream_t stream,
                           int dev) {
-  auto kern = rs::verify_kernel<THREADS, BF16>;
-  const int slot = (THREADS == 512 ? 2 : 0) + (BF16 ? 1 : 0);
+  const void* kern = kernel_ptr<THREADS, BF16>(pl.kernel);
+  const int slot = (pl.kernel == RESISPEC_KERNEL_STREAM ? 4 : 0) + (THREADS == 512 ? 2 : 0) +
+                   (BF16 ? 1 : 0);
   {
     std::lock_guard<std::mutex> lk(g_mu);
     if (!g_attr_set[dev][slot]) {
@@ -217,7 +336,8 @@ cudaError_t launch_verify(const Plan& pl, const rs::VerifyParams& prm, cudaStrea
   attr[0].val.clusterDim.z = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, kern, prm);
+  void* args[] = {const_cast<rs::VerifyParams*>(&prm)};
+  return cudaLaunchKernelExC(&cfg, kern, args);
 }
 
 }  // namespace
@@ -247,9 +367,7 @@ const char* resispec_status_string(int s) {
 
 const char* resispec_last_error(void) { return g_last_error; }
 
-int resispec_plan(resispec_dims dims, const resispec_opts* opts, int32_t* cluster_size,
-                  int32_t* block_threads, int32_t* smem_bytes, int32_t* slice_elems,
-                  int32_t* uses_tma) {
+int resispec_plan(resispec_dims dims, const resispec_opts* opts, resispec_plan_info* out) {
   resispec_opts o;
   resispec_opts_default(&o);
   if (opts) o = *opts;
@@ -267,11 +385,16 @@ int resispec_plan(resispec_dims dims, const resispec_opts* opts, int32_t* cluste
   Plan p;
   const int st = make_plan(dims, o, dev, sms, nullptr, nullptr, &p);
   if (st) return st;
-  if (cluster_size) *cluster_size = p.C;
-  if (block_threads) *block_threads = p.threads;
-  if (smem_bytes) *smem_bytes = p.smem;
-  if (slice_elems) *slice_elems = p.L;
-  if (uses_tma) *uses_tma = p.use_tma;
+  if (out) {
+    out->kernel = p.kernel;
+    out->cluster_size = p.C;
+    out->block_threads = p.threads;
+    out->smem_bytes = p.smem;
+    out->slice_elems = p.L;
+    out->uses_tma = p.use_tma;
+    out->stages = p.stages;
+    out->active_clusters = p.active;
+  }
   return RESISPEC_OK;
 }
 
@@ -327,6 +450,7 @@ int resispec_verify_ex(const void* target_logits, const void* draft_logits,
   prm.mode = o.mode;
   prm.use_tma = pl.use_tma;
   prm.prefetch = (o.flags & RESISPEC_FLAG_PREFETCH) != 0;
+  prm.stages = pl.stages;
 
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   cudaError_t e;

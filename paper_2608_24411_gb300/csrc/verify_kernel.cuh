@@ -52,7 +52,7 @@ constexpr int kFlagTargetBad = 1;
 constexpr int kFlagDraftBad = 2;
 constexpr int kFlagTimeout = 4;
 
-constexpr uint32_t kSpinLimit = 1u << 22;  // try_wait attempts before giving up
+constexpr uint32_t kSpinLimit = 1u << 18;  // suspended try_wait attempts (10 us each) before giving up
 constexpr int kMaxCluster = 16;
 constexpr int kMaxChunks = 32;             // bulk-copy chunks per row
 constexpr int kSlotFloats = 12;
@@ -79,6 +79,7 @@ struct VerifyParams {
   int32_t mode;        // 0 ResiSpec, 1 SpecInfer
   int32_t use_tma;
   int32_t prefetch;    // L2 prefetch of the first child's rows
+  int32_t stages;      // streaming kernel: ring stages
 };
 
 struct __align__(16) Slot {
@@ -102,7 +103,9 @@ constexpr int kHeadBytes = 4608;
 static_assert(sizeof(Head) <= kHeadBytes, "head too large");
 
 // ---------------------------------------------------------------- residual map
-enum : int { kScale = 0, kIdent = 1, kResi = 2, kSpec = 3 };
+// kScale: R = w * sc with the per-thread scale sc (sc = 1 once R is materialised
+// and no map is pending); kResi: GetProxy residual; kSpec: Eq. recur.
+enum : int { kScale = 0, kResi = 1, kSpec = 2 };
 
 struct Pending {
   int kind;
@@ -120,8 +123,6 @@ __device__ __forceinline__ float apply_map(const Pending& P, float w, float qq, 
                                            float sc) {
   if constexpr (KIND == kScale) {
     return __fmul_rn(w, sc);
-  } else if constexpr (KIND == kIdent) {
-    return w;
   } else if constexpr (KIND == kResi) {
     // GetProxy: r = min(Z q, R) + lambda (R - min(Z q, R)) off x0, r(x0) = 0;
     // R' = r / sum r.
@@ -138,7 +139,6 @@ __device__ __forceinline__ float apply_any(const Pending& P, float w, float qq, 
                                            float sc) {
   switch (P.kind) {
     case kScale: return apply_map<kScale>(P, w, qq, idx, sc);
-    case kIdent: return apply_map<kIdent>(P, w, qq, idx, sc);
     case kResi: return apply_map<kResi>(P, w, qq, idx, sc);
     default: return apply_map<kSpec>(P, w, qq, idx, sc);
   }
@@ -150,25 +150,27 @@ __device__ __forceinline__ float ref_scale(float m, float M, float inv) {
 }
 
 // ---------------------------------------------------------------- reductions
-__device__ __forceinline__ float warp_max(float v) {
+// Butterfly sum over groups of 2^LEVELS lanes (every lane of a group gets the
+// same bits).  LEVELS = 5: the whole warp; LEVELS = 4: lanes 0..15 (enough
+// for one value per warp of a CTA, or per CTA of a cluster).
+template <int LEVELS>
+__device__ __forceinline__ float group_sum(float v) {
 #pragma unroll
-  for (int o = 16; o; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
+  for (int o = 1 << (LEVELS - 1); o; o >>= 1) v = __fadd_rn(v, __shfl_xor_sync(0xffffffffu, v, o));
   return v;
 }
 
-__device__ __forceinline__ float warp_sum(float v) {
-#pragma unroll
-  for (int o = 16; o; o >>= 1) v = __fadd_rn(v, __shfl_xor_sync(0xffffffffu, v, o));
-  return v;
-}
+__device__ __forceinline__ float warp_sum(float v) { return group_sum<5>(v); }
 
-// (reference, sum of 2^(z c - reference)) pairs of a warp, references in
-// log2 units: max first, then each lane rescales its sum to the common
-// reference, then a sum.  Butterflies leave the same bits in every lane.
-__device__ __forceinline__ void warp_pair(float& m, float& s) {
-  const float M = warp_max(m);
+// (reference, sum of 2^(z c - reference)) pairs, references in log2 units:
+// the common reference is the warp maximum (one redux), each lane rescales
+// its sum to it, then a butterfly sum over groups of 2^LEVELS lanes.  Lanes
+// that must not contribute hold (-inf, 0).
+template <int LEVELS>
+__device__ __forceinline__ void pair_reduce(float& m, float& s) {
+  const float M = redux_max(m);
   const float t = (m == -INFINITY) ? 0.f : __fmul_rn(s, ex2(__fsub_rn(m, M)));
-  s = warp_sum(t);
+  s = group_sum<LEVELS>(t);
   m = M;
 }
 
@@ -182,23 +184,25 @@ __device__ __forceinline__ bool wait_bar(uint32_t bar, uint32_t parity) {
 // CTA partial to every CTA of the cluster and the same reduction over the C
 // received partials.  Every CTA combines identical partials in identical
 // lanes, so all CTAs obtain the same bits.
-//   NORM: (a0, a1) and (a2, a3) are (max, scaled sum) pairs of the target
-//         and draft rows; SUM: a0, a1 are sums (a2, a3 unused).
-//   H.pubv holds the values published by the owner thread of a token (zero
-//   in CTAs without an owner); they travel unreduced and are summed across
-//   CTAs, where exactly one CTA contributes.  flags are OR-ed.
+//   NORM: (a0, a1) and (a2, a3) are (reference, scaled sum) pairs of the
+//         target and draft rows; SUM: a0, a1 are sums (a2, a3 unused).
+//   H.pubv holds the values published by the owner thread of a token; every
+//   CTA reads them from the slot of the owner CTA `owner` (-1: none).
+//   flags are OR-ed.
 // out[0..3]: reduced partials, out[4..7]: published values.
 template <int NWARPS, bool NORM>
 __device__ __forceinline__ void exchange(Head& H, float a0, float a1, float a2, float a3,
-                                         int flags, int& xp, uint32_t& xph, uint32_t rank,
-                                         uint32_t C, float (&out)[8], int& oflags) {
+                                         int flags, int owner, int& xp, uint32_t& xph,
+                                         uint32_t rank, uint32_t C, float (&out)[8],
+                                         int& oflags) {
+  static_assert(NWARPS <= 16, "second reduction level covers 16 warps");
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   if constexpr (NORM) {
-    warp_pair(a0, a1);
-    warp_pair(a2, a3);
+    pair_reduce<5>(a0, a1);
+    pair_reduce<5>(a2, a3);
   } else {
-    a0 = warp_sum(a0);
-    a1 = warp_sum(a1);
+    a0 = group_sum<5>(a0);
+    a1 = group_sum<5>(a1);
   }
   flags = __reduce_or_sync(0xffffffffu, flags);
   if (lane == 0) {
@@ -211,57 +215,53 @@ __device__ __forceinline__ void exchange(Head& H, float a0, float a1, float a2, 
   __syncthreads();
   if (warp == 0) {
     const float id = NORM ? -INFINITY : 0.f;
-    a0 = lane < NWARPS ? H.wpart[lane][0] : id;
-    a1 = lane < NWARPS ? H.wpart[lane][1] : 0.f;
-    a2 = lane < NWARPS ? H.wpart[lane][2] : id;
-    a3 = lane < NWARPS ? H.wpart[lane][3] : 0.f;
-    int f = lane < NWARPS ? H.wflag[lane] : 0;
+    const bool in = lane < NWARPS;
+    a0 = in ? H.wpart[lane][0] : id;
+    a1 = in ? H.wpart[lane][1] : 0.f;
+    a2 = in ? H.wpart[lane][2] : id;
+    a3 = in ? H.wpart[lane][3] : 0.f;
+    int f = __reduce_or_sync(0xffffffffu, in ? H.wflag[lane] : 0);
     if constexpr (NORM) {
-      warp_pair(a0, a1);
-      warp_pair(a2, a3);
+      pair_reduce<4>(a0, a1);
+      pair_reduce<4>(a2, a3);
     } else {
-      a0 = warp_sum(a0);
-      a1 = warp_sum(a1);
+      a0 = group_sum<4>(a0);
+      a1 = group_sum<4>(a1);
     }
-    f = __reduce_or_sync(0xffffffffu, f);
-    const float p0 = H.pubv[0], p1 = H.pubv[1], p2 = H.pubv[2], p3 = H.pubv[3];
-    __syncwarp();
-    if (lane < 4) H.pubv[lane] = 0.f;  // ready for the next publication
     const int p = xp;
     if (lane < (int)C) {
       const uint32_t dst = map_to_rank(smem_addr(&H.rx[p][rank]), lane);
       const uint32_t bar = map_to_rank(smem_addr(&H.xbar[p]), lane);
       st_async_v4(dst, __float_as_uint(a0), __float_as_uint(a1), __float_as_uint(a2),
                   __float_as_uint(a3), bar);
-      st_async_v4(dst + 16, __float_as_uint(p0), __float_as_uint(p1), __float_as_uint(p2),
-                  __float_as_uint(p3), bar);
+      st_async_v4(dst + 16, __float_as_uint(H.pubv[0]), __float_as_uint(H.pubv[1]),
+                  __float_as_uint(H.pubv[2]), __float_as_uint(H.pubv[3]), bar);
       st_async_v4(dst + 32, (uint32_t)f, 0u, 0u, 0u, bar);
     }
     if (lane == 0) mbar_arrive_expect_tx(smem_addr(&H.xbar[p]), C * kSlotBytes);
     const bool ok = __all_sync(0xffffffffu, wait_bar(smem_addr(&H.xbar[p]), (xph >> p) & 1u));
     xph ^= 1u << p;
-    float q[4] = {0.f, 0.f, 0.f, 0.f};
-    a0 = id; a1 = 0.f; a2 = id; a3 = 0.f; f = 0;
-    if (lane < (int)C) {
-      const Slot& sl = H.rx[p][lane];
-      a0 = sl.v[0]; a1 = sl.v[1]; a2 = sl.v[2]; a3 = sl.v[3];
-      q[0] = sl.v[4]; q[1] = sl.v[5]; q[2] = sl.v[6]; q[3] = sl.v[7];
-      f = __float_as_int(sl.v[8]);
+    const bool got = lane < (int)C;
+    a0 = got ? H.rx[p][lane].v[0] : id;
+    a1 = got ? H.rx[p][lane].v[1] : 0.f;
+    a2 = got ? H.rx[p][lane].v[2] : id;
+    a3 = got ? H.rx[p][lane].v[3] : 0.f;
+    f = __reduce_or_sync(0xffffffffu, got ? __float_as_int(H.rx[p][lane].v[8]) : 0);
+    if (got) {
       H.part[lane][0] = a0; H.part[lane][1] = a1; H.part[lane][2] = a2; H.part[lane][3] = a3;
     }
     if constexpr (NORM) {
-      warp_pair(a0, a1);
-      warp_pair(a2, a3);
+      pair_reduce<4>(a0, a1);
+      pair_reduce<4>(a2, a3);
     } else {
-      a0 = warp_sum(a0);
-      a1 = warp_sum(a1);
+      a0 = group_sum<4>(a0);
+      a1 = group_sum<4>(a1);
     }
-#pragma unroll
-    for (int k = 0; k < 4; ++k) q[k] = warp_sum(q[k]);
-    f = __reduce_or_sync(0xffffffffu, f);
     if (lane == 0) {
       H.bc[0] = a0; H.bc[1] = a1; H.bc[2] = a2; H.bc[3] = a3;
-      H.bc[4] = q[0]; H.bc[5] = q[1]; H.bc[6] = q[2]; H.bc[7] = q[3];
+      const bool has = owner >= 0 && owner < (int)C;
+#pragma unroll
+      for (int k = 0; k < 4; ++k) H.bc[4 + k] = has ? H.rx[p][owner].v[4 + k] : 0.f;
       H.bc[8] = __int_as_float(f | (ok ? 0 : kFlagTimeout));
     }
   }
@@ -275,7 +275,7 @@ __device__ __forceinline__ void exchange(Head& H, float a0, float a1, float a2, 
 // ---------------------------------------------------------------- tree
 // first_child[n + 1] / next_sibling[c] in ascending node order, built by one
 // warp from the highest index down (siblings found with __match_any_sync).
-__device__ void build_children(const int16_t* par, int16_t* first_child, int16_t* next_sib,
+static __device__ void build_children(const int16_t* par, int16_t* first_child, int16_t* next_sib,
                                int N) {
   const int lane = threadIdx.x & 31;
   if ((threadIdx.x >> 5) != 0 || N == 0) return;
@@ -297,6 +297,12 @@ __device__ void build_children(const int16_t* par, int16_t* first_child, int16_t
 }
 
 // ---------------------------------------------------------------- row I/O
+// Rows are copied and normalised in chunks of chunk_vectors() 16-byte
+// vectors: two per thread for fp32 rows, one per thread for bf16 rows (whose
+// widened fp32 values need twice the registers).
+template <int THREADS, bool BF16>
+__host__ __device__ constexpr int chunk_vectors() { return (BF16 ? 1 : 2) * THREADS; }
+
 // Starts the copies of this CTA's slice [lo, lo + nloc) of the target row
 // (and of the draft row when need_draft) that begins at element row_base.
 template <int THREADS, bool BF16>
@@ -305,7 +311,7 @@ __device__ __forceinline__ void issue_rows(Head& H, const VerifyParams& P, float
   const int L = P.slice;
   const size_t off = row_base + (size_t)lo;
   constexpr uint32_t es = BF16 ? 2u : 4u;
-  constexpr uint32_t kChunkBytes = 2u * THREADS * 16u;
+  constexpr uint32_t kChunkBytes = (uint32_t)chunk_vectors<THREADS, BF16>() * 16u;
   // Earlier generic accesses to W / Q must be ordered before the copies.
   fence_proxy_async_smem();
   __syncthreads();
@@ -344,33 +350,28 @@ __device__ __forceinline__ void issue_rows(Head& H, const VerifyParams& P, float
 __device__ __forceinline__ float bf16_lo(uint32_t w) { return __uint_as_float(w << 16); }
 __device__ __forceinline__ float bf16_hi(uint32_t w) { return __uint_as_float(w & 0xffff0000u); }
 
-// Tempered normaliser, first half (S2): one pass over this CTA's slice of a
-// row as its chunks land.  With c = log2(e) / T and the thread's reference
-// mref (log2 units: the rounded product of its largest logit so far and c)
-// it stores e = 2^(z c - mref), one fused multiply-add and one 2^x per
-// element (0 beyond the valid part), and returns (mref, sum e).  A NaN or
-// +inf logit makes the thread's sum non-finite, which is how the error
-// contract detects it.  Returns false if a chunk wait timed out.
+// Tempered normaliser, first half (S2): one pass over this CTA's slice of
+// the target row and (need_draft) the draft row as their chunks land.  With
+// c = log2(e) / T and a per-thread reference m per row (log2 units: the
+// rounded product of the thread's largest logit so far and c) it stores
+// e = 2^(z c - m), one fused multiply-add and one 2^x per element (0 beyond
+// the valid part), and returns (m, sum e) per row.  A NaN or +inf logit makes
+// the thread's sum non-finite, which is how the error contract detects it.
+// Returns false if a chunk wait timed out.
 template <int THREADS, bool BF16>
-__device__ __forceinline__ bool normalize_row(float* buf, int L, int nloc, float c,
-                                              uint32_t bar0, uint32_t parity, int nk_tma,
-                                              bool wait_tma, float& mref, float& ssum) {
-  constexpr int VEC = BF16 ? 8 : 4;
-  constexpr int CV = 2 * THREADS;
-  const int NV = L / VEC;
-  const int NVV = nloc / VEC;  // vectors whose VEC elements are all valid
-  const int NK = (NV + CV - 1) / CV;
-  const int tid = threadIdx.x;
-  const uint16_t* raw = reinterpret_cast<const uint16_t*>(buf) + L;
-  bool ok = true;
-  mref = -INFINITY;
-  ssum = 0.f;
-  for (int k = 0; k < NK; ++k) {
-    if (wait_tma && k < nk_tma) ok = wait_bar(bar0 + 8u * (uint32_t)k, parity) && ok;
-    float z[2][VEC];
+struct RowNorm {
+  static constexpr int VEC = BF16 ? 8 : 4;
+  static constexpr int CV = chunk_vectors<THREADS, BF16>();  // vectors per chunk
+  static constexpr int HV = CV / THREADS;                     // vectors per thread per chunk
+
+  // Load this thread's raw values of chunk k of one row (-inf where invalid).
+  __device__ __forceinline__ static void load(const float* buf, int L, int nloc, int k,
+                                              float (&z)[HV][VEC]) {
+    const int NV = L / VEC, NVV = nloc / VEC;
+    const uint16_t* raw = reinterpret_cast<const uint16_t*>(buf) + L;
 #pragma unroll
-    for (int h = 0; h < 2; ++h) {
-      const int g = k * CV + h * THREADS + tid;
+    for (int h = 0; h < HV; ++h) {
+      const int g = k * CV + h * THREADS + (int)threadIdx.x;
 #pragma unroll
       for (int j = 0; j < VEC; ++j) z[h][j] = -INFINITY;
       if (g < NVV || (g < NV && g * VEC < nloc)) {
@@ -393,51 +394,60 @@ __device__ __forceinline__ bool normalize_row(float* buf, int L, int nloc, float
         }
       }
     }
+  }
+
+  // Turn z into e in place, updating (m, s).
+  __device__ __forceinline__ static void exps(float* buf, int L, int k, float c,
+                                              float (&z)[HV][VEC], float& m, float& s) {
+    const int NV = L / VEC;
     float vmax = -INFINITY;
 #pragma unroll
-    for (int h = 0; h < 2; ++h)
+    for (int h = 0; h < HV; ++h)
 #pragma unroll
       for (int j = 0; j < VEC; ++j) vmax = fmaxf(vmax, z[h][j]);
-    if (__fmaf_rn(vmax, c, -mref) > kRebaseLog2) {
+    if (__fmaf_rn(vmax, c, -m) > kRebaseLog2) {
       // Move this thread's reference up: rescale what it stored so far.
       const float mnew = __fmul_rn(vmax, c);
-      if (mref != -INFINITY) {
-        const float f = ex2(__fsub_rn(mref, mnew));
-        ssum = __fmul_rn(ssum, f);
+      if (m != -INFINITY) {
+        const float f = ex2(__fsub_rn(m, mnew));
+        s = __fmul_rn(s, f);
         for (int k2 = 0; k2 < k; ++k2)
-          for (int h = 0; h < 2; ++h) {
-            const int g = k2 * CV + h * THREADS + tid;
+          for (int h = 0; h < HV; ++h) {
+            const int g = k2 * CV + h * THREADS + (int)threadIdx.x;
             if (g < NV)
               for (int j = 0; j < VEC; ++j) buf[g * VEC + j] = __fmul_rn(buf[g * VEC + j], f);
           }
       }
-      mref = mnew;
+      m = mnew;
     }
-    float e[2][VEC];
-    if (mref == -INFINITY) {  // nothing finite seen yet: every value is -inf or NaN
+    if (m == -INFINITY) {  // nothing finite seen yet: every value is -inf or NaN
 #pragma unroll
-      for (int h = 0; h < 2; ++h)
+      for (int h = 0; h < HV; ++h)
 #pragma unroll
         for (int j = 0; j < VEC; ++j) {
-          e[h][j] = 0.f;
-          if (isnan(z[h][j])) ssum = __int_as_float(0x7fc00000);
+          if (isnan(z[h][j])) s = __int_as_float(0x7fc00000);
+          z[h][j] = 0.f;
         }
     } else {
 #pragma unroll
-      for (int h = 0; h < 2; ++h) {
-        float s = 0.f;
+      for (int h = 0; h < HV; ++h) {
+        float t = 0.f;
 #pragma unroll
         for (int j = 0; j < VEC; ++j) {
-          e[h][j] = ex2(__fmaf_rn(z[h][j], c, -mref));
-          s += e[h][j];
+          z[h][j] = ex2(__fmaf_rn(z[h][j], c, -m));
+          t += z[h][j];
         }
-        ssum += s;
+        s += t;
       }
     }
-    if constexpr (BF16) __syncthreads();  // this chunk's raw values are all read
+  }
+
+  __device__ __forceinline__ static void store(float* buf, int L, int k,
+                                               const float (&e)[HV][VEC]) {
+    const int NV = L / VEC;
 #pragma unroll
-    for (int h = 0; h < 2; ++h) {
-      const int g = k * CV + h * THREADS + tid;
+    for (int h = 0; h < HV; ++h) {
+      const int g = k * CV + h * THREADS + (int)threadIdx.x;
       if (g < NV) {
         float4* d = reinterpret_cast<float4*>(buf + (size_t)g * VEC);
 #pragma unroll
@@ -446,8 +456,42 @@ __device__ __forceinline__ bool normalize_row(float* buf, int L, int nloc, float
       }
     }
   }
-  return ok;
-}
+
+  // One row, chunk by chunk as its copies land: returns (mref, sum e) and
+  // false if a chunk wait timed out.
+  __device__ __forceinline__ static bool row(float* buf, int L, int nloc, float c, uint32_t bar0,
+                                             uint32_t parity, int nk_tma, bool wait_tma,
+                                             float& m, float& s) {
+    const int NK = (L / VEC + CV - 1) / CV;
+    bool ok = true;
+    m = -INFINITY;
+    s = 0.f;
+    for (int k = 0; k < NK; ++k) {
+      if (wait_tma && k < nk_tma) ok = wait_bar(bar0 + 8u * (uint32_t)k, parity) && ok;
+      float z[HV][VEC];
+      load(buf, L, nloc, k, z);
+      exps(buf, L, k, c, z, m, s);
+      if constexpr (BF16) __syncthreads();  // this chunk's raw values are all read
+      store(buf, L, k, z);
+    }
+    return ok;
+  }
+
+  // Target row, then (if the node has children) draft row; both rows' copies
+  // were issued together, so the draft's chunks land while the target is
+  // being normalised.
+  __device__ __forceinline__ static bool run(float* W, float* Q, bool need_draft, int L, int nloc,
+                                             float c, uint32_t bar_t, uint32_t bar_d,
+                                             uint32_t ph_t, uint32_t ph_d, int nk_tma,
+                                             bool wait_tma, float& mt, float& st, float& md,
+                                             float& sd) {
+    bool ok = row(W, L, nloc, c, bar_t, ph_t, nk_tma, wait_tma, mt, st);
+    md = -INFINITY;
+    sd = 0.f;
+    if (need_draft) ok = row(Q, L, nloc, c, bar_d, ph_d, nk_tma, wait_tma, md, sd) && ok;
+    return ok;
+  }
+};
 
 // One rejection pass: materialise R_j = map(W) into W and accumulate the
 // sums of rejection j (ResiSpec: sum min(Z q, R) and sum (R - min(Z q, R))
@@ -522,29 +566,20 @@ __device__ __forceinline__ void reject_pass(float* W, const float* Q, int L, int
   s2out = s2sum;
 }
 
+// A ResiSpec pass follows either the normaliser scale or a ResiSpec map; a
+// SpecInfer pass either the scale or a SpecInfer map.
 template <int THREADS, bool BF16, bool RESI>
 __device__ __forceinline__ void reject_pass_any(float* W, const float* Q, int L, int lo,
                                                 const Pending& P, float at, float bt, float mt,
                                                 float md, int x0, float Z, int xn, float* pubv,
                                                 float& s1, float& s2) {
-  switch (P.kind) {
-    case kScale:
-      reject_pass<THREADS, BF16, kScale, RESI>(W, Q, L, lo, P, at, bt, mt, md, x0, Z, xn, pubv,
-                                               s1, s2);
-      break;
-    case kIdent:
-      reject_pass<THREADS, BF16, kIdent, RESI>(W, Q, L, lo, P, at, bt, mt, md, x0, Z, xn, pubv,
-                                               s1, s2);
-      break;
-    case kResi:
-      reject_pass<THREADS, BF16, kResi, RESI>(W, Q, L, lo, P, at, bt, mt, md, x0, Z, xn, pubv,
-                                              s1, s2);
-      break;
-    default:
-      reject_pass<THREADS, BF16, kSpec, RESI>(W, Q, L, lo, P, at, bt, mt, md, x0, Z, xn, pubv,
-                                              s1, s2);
-      break;
-  }
+  constexpr int MAPPED = RESI ? kResi : kSpec;
+  if (P.kind == kScale)
+    reject_pass<THREADS, BF16, kScale, RESI>(W, Q, L, lo, P, at, bt, mt, md, x0, Z, xn, pubv, s1,
+                                             s2);
+  else
+    reject_pass<THREADS, BF16, MAPPED, RESI>(W, Q, L, lo, P, at, bt, mt, md, x0, Z, xn, pubv, s1,
+                                             s2);
 }
 
 // ---------------------------------------------------------------- sampler
@@ -622,7 +657,7 @@ __device__ bool sample_final(Head& H, const VerifyParams& P, float* W, const flo
     if (need_direct) {
       float o[8];
       int of;
-      exchange<NW, false>(H, s, 0.f, 0.f, 0.f, 0, xp, xph, rank, C, o, of);
+      exchange<NW, false>(H, s, 0.f, 0.f, 0.f, 0, -1, xp, xph, rank, C, o, of);
       mass_kind = 4;
     }
   }
@@ -729,7 +764,7 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 3)
   constexpr int NW = THREADS / 32;
   constexpr int VEC = BF16 ? 8 : 4;
   constexpr uint32_t es = BF16 ? 2u : 4u;
-  constexpr uint32_t kChunkBytes = 2u * THREADS * 16u;
+  constexpr uint32_t kChunkBytes = (uint32_t)chunk_vectors<THREADS, BF16>() * 16u;
   extern __shared__ __align__(128) unsigned char smem[];
   Head& H = *reinterpret_cast<Head*>(smem);
   const int L = P.slice;
@@ -751,6 +786,8 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 3)
   const int nloc = max(0, min(V, lo + L) - lo);
   const int nk_tma = (int)(((uint32_t)nloc * es + kChunkBytes - 1) / kChunkBytes);
   const float c = P.scale_log2;
+  // CTA of the cluster whose slice holds token x (-1 for an invalid token)
+  auto owner_of = [&](int x) { return (x >= 0 && x < V) ? x / L : -1; };
 
   if (tid < 4) H.pubv[tid] = 0.f;
   if (tid == 0) {
@@ -799,12 +836,10 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 3)
     const bool need_draft = c1 >= 0;
 
     // ---- tempered normaliser (S2): one pass per row, then one exchange
-    float mref_t, sum_t, mref_d = -INFINITY, sum_d = 0.f;
-    bool ok = normalize_row<THREADS, BF16>(W, L, nloc, c, smem_addr(&H.tbar[0][0]), tph & 1u,
-                                           nk_tma, P.use_tma, mref_t, sum_t);
-    if (need_draft)
-      ok = normalize_row<THREADS, BF16>(Q, L, nloc, c, smem_addr(&H.tbar[1][0]),
-                                        (tph >> 1) & 1u, nk_tma, P.use_tma, mref_d, sum_d) && ok;
+    float mref_t, sum_t, mref_d, sum_d;
+    const bool ok = RowNorm<THREADS, BF16>::run(
+        W, Q, need_draft, L, nloc, c, smem_addr(&H.tbar[0][0]), smem_addr(&H.tbar[1][0]),
+        tph & 1u, (tph >> 1) & 1u, nk_tma, P.use_tma, mref_t, sum_t, mref_d, sum_d);
     const bool bad_t = !(sum_t <= FLT_MAX), bad_d = !(sum_d <= FLT_MAX);
     if (ok) {
       tph ^= need_draft ? 3u : 1u;
@@ -821,7 +856,8 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 3)
                       (ok ? 0 : kFlagTimeout);
     float o[8];
     int oflags;
-    exchange<NW, true>(H, mref_t, sum_t, mref_d, sum_d, flags, xp, xph, rank, C, o, oflags);
+    exchange<NW, true>(H, mref_t, sum_t, mref_d, sum_d, flags, owner_of(x1), xp, xph, rank, C, o,
+                       oflags);
     if (oflags & kFlagTimeout) { err |= kErrTimeout; break; }
     if (oflags & kFlagTargetBad) { err |= kErrNonfinite; break; }
     if (o[0] == -INFINITY) { err |= kErrEmpty; break; }
@@ -829,7 +865,8 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 3)
     if (need_draft && o[2] == -INFINITY) { err |= kErrEmpty; break; }
     const float Mt = o[0], invSt = __frcp_rn(o[1]);
     const float Md = o[2], invSd = need_draft ? __frcp_rn(o[3]) : 0.f;
-    const float at = ref_scale(mref_t, Mt, invSt);
+    float at = ref_scale(mref_t, Mt, invSt);  // 1 once R is materialised with no map pending
+    bool ident = false;
     const float bt = need_draft ? ref_scale(mref_d, Md, invSd) : 0.f;
     float pub[4] = {o[4], o[5], o[6], o[7]};
     Pending Pm{kScale, -1, 0.f, 0.f, 0.f};
@@ -860,8 +897,9 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 3)
       const int x = cand_s[cn];
       if (x < 0 || x >= V) { err |= kErrToken; break; }
       const float qx = __fmul_rn(pub[2], ref_scale(pub[3], Md, invSd));
-      const float Rx = Pm.kind == kScale ? __fmul_rn(pub[0], ref_scale(pub[1], Mt, invSt))
-                                         : apply_any(Pm, pub[0], qx, x, 0.f);
+      const float Rx = Pm.kind != kScale ? apply_any(Pm, pub[0], qx, x, 0.f)
+                       : ident          ? pub[0]
+                                        : __fmul_rn(pub[0], ref_scale(pub[1], Mt, invSt));
       const float u = u_acc[cn + 1];
       if (__fmul_rn(u, qx) < Rx) { accepted = cn; acc_tok = x; break; }
       rejects += 1;
@@ -879,7 +917,8 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 3)
             H.pubv[2] = Q[xn - lo];
             H.pubv[3] = mref_d;
           }
-          exchange<NW, false>(H, 0.f, 0.f, 0.f, 0.f, 0, xp, xph, rank, C, o, oflags);
+          exchange<NW, false>(H, 0.f, 0.f, 0.f, 0.f, 0, owner_of(xn), xp, xph, rank, C, o,
+                              oflags);
           if (oflags & kFlagTimeout) { err |= kErrTimeout; break; }
           pub[0] = o[4]; pub[1] = o[5]; pub[2] = o[6]; pub[3] = o[7];
           mass_kind = 0;
@@ -888,7 +927,8 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 3)
         }
         reject_pass_any<THREADS, BF16, true>(W, Q, L, lo, Pm, at, bt, mref_t, mref_d, x, Z, xn,
                                              H.pubv, s1, s2);
-        exchange<NW, false>(H, s1, s2, 0.f, 0.f, 0, xp, xph, rank, C, o, oflags);
+        exchange<NW, false>(H, s1, s2, 0.f, 0.f, 0, owner_of(xn), xp, xph, rank, C, o,
+                            oflags);
         if (oflags & kFlagTimeout) { err |= kErrTimeout; break; }
         const float S1 = o[0], S2 = o[1];
         const float delta = __fsub_rn(Z, S1);
@@ -897,21 +937,26 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 3)
         if (norm > 0.f) {
           Pm = Pending{kResi, x, __frcp_rn(norm), Z, lam};
           mass_kind = 2;
-        } else {
-          Pm = Pending{kIdent, -1, 1.f, 0.f, 0.f};
+        } else {  // R_j is materialised in W: continue from it unchanged
+          Pm = Pending{kScale, -1, 1.f, 0.f, 0.f};
+          at = 1.f;
+          ident = true;
           info |= kInfoDegenerate;
           mass_kind = 0;
         }
       } else {
         reject_pass_any<THREADS, BF16, false>(W, Q, L, lo, Pm, at, bt, mref_t, mref_d, x, 0.f,
                                               xn, H.pubv, s1, s2);
-        exchange<NW, false>(H, s1, s2, 0.f, 0.f, 0, xp, xph, rank, C, o, oflags);
+        exchange<NW, false>(H, s1, s2, 0.f, 0.f, 0, owner_of(xn), xp, xph, rank, C, o,
+                            oflags);
         if (oflags & kFlagTimeout) { err |= kErrTimeout; break; }
         if (o[0] > 0.f) {
           Pm = Pending{kSpec, -1, __frcp_rn(o[0]), 0.f, 0.f};
           mass_kind = 3;
-        } else {
-          Pm = Pending{kIdent, -1, 1.f, 0.f, 0.f};
+        } else {  // R_j is materialised in W: continue from it unchanged
+          Pm = Pending{kScale, -1, 1.f, 0.f, 0.f};
+          at = 1.f;
+          ident = true;
           info |= kInfoDegenerate;
           mass_kind = 0;
         }
@@ -966,17 +1011,6 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 3)
     }
   }
   cluster_sync();  // no CTA leaves while a peer may still write its slots
-}
-
-// Device Philox draws for tests.
-__global__ void uniforms_kernel(uint64_t seed, const int32_t* seq, const int32_t* row, int n,
-                                float* u0, float* u1) {
-  const int i = blockIdx.x * blockDim.x + threadIdx.x;
-  if (i >= n) return;
-  const U64x4 r = philox4x64_10((uint64_t)(uint32_t)row[i], (uint64_t)(uint32_t)seq[i], 0, 0,
-                                seed, 0);
-  u0[i] = u24(r.w[0]);
-  u1[i] = u24(r.w[1]);
 }
 
 }  // namespace rs

@@ -39,7 +39,7 @@ def test_library_exports_every_declared_symbol(lib):
     for n in declared_functions():
         assert hasattr(lib, n), n
     assert set(rs.EXPORTED) <= set(declared_functions())
-    assert lib.resispec_abi_version() == 1
+    assert lib.resispec_abi_version() == 2
 
 
 def test_opts_default_layout(lib):
@@ -74,12 +74,20 @@ def test_synchronous_argument_errors(lib):
 
 
 def test_plan_without_device(lib):
+    # the bench workload (B = 64, V = 151936 fp32) cannot sit on chip at once:
+    # the automatic choice streams it, four CTAs per sequence
     p = rs.plan(64, 62, 151936, 5, "f32")
-    assert p["cluster_size"] in (8, 16)
-    assert p["slice_elems"] % 8 == 0
-    assert p["slice_elems"] * p["cluster_size"] >= 151936
-    assert p["smem_bytes"] <= 227 * 1024
+    assert p["kernel_name"] == "stream" and p["cluster_size"] == 4
+    assert p["stages"] >= 2 and p["smem_bytes"] <= 113 * 1024   # two CTAs per SM
+    assert p["slice_elems"] % 8 == 0 and p["slice_elems"] * 4 >= 151936
     assert p["uses_tma"] == 1
+    p = rs.plan(64, 62, 151936, 5, "f32", kernel="resident")
+    assert p["kernel_name"] == "resident" and p["cluster_size"] in (8, 16)
+    assert p["slice_elems"] * p["cluster_size"] >= 151936
+    assert p["smem_bytes"] <= 227 * 1024 and p["stages"] == 0
+    # a small batch that fits on chip stays resident
+    p = rs.plan(1, 60, 32000, 5, "bf16")
+    assert p["kernel_name"] == "resident"
     p = rs.plan(1, 12, 64, 4, "f32", cluster_size=1)
     assert p["cluster_size"] == 1 and p["slice_elems"] == 64
     p = rs.plan(1, 12, 61, 4, "f32", cluster_size=2)
@@ -87,14 +95,24 @@ def test_plan_without_device(lib):
     p = rs.plan(1, 12, 64, 4, "bf16", no_tma=True)
     assert p["uses_tma"] == 0
     for V in (1, 7, 32000, 128256, 256000, rs.MAX_VOCAB):
-        p = rs.plan(128, 488, V, 6, "bf16")
-        assert p["smem_bytes"] <= 227 * 1024
+        for kernel in ("resident", "stream"):
+            p = rs.plan(128, 488, V, 6, "bf16", kernel=kernel)
+            assert p["smem_bytes"] <= 227 * 1024
+    # streaming: C / waves over 2 CTAs per SM (152 SMs without a device)
+    assert rs.plan(128, 16, 256000, 1, "bf16")["cluster_size"] == 2
+    assert rs.plan(16, 32, 128256, 4, "bf16", kernel="stream")["cluster_size"] == 16
+    # the streaming kernel holds no rows: one CTA per sequence at any V
+    p = rs.plan(1, 2, rs.MAX_VOCAB, 1, "f32", cluster_size=1, kernel="stream")
+    assert p["cluster_size"] == 1 and p["slice_elems"] == rs.MAX_VOCAB
     p = rs.plan(1, 2, 1000, 1, "f32", cluster_size=3)   # any cluster size up to 16
     assert p["cluster_size"] == 3 and p["slice_elems"] * 3 >= 1000
     with pytest.raises(rs.ResispecError):
         rs.plan(1, 2, 10, 1, "f32", cluster_size=17)
     with pytest.raises(rs.ResispecError):
-        rs.plan(1, 2, rs.MAX_VOCAB, 1, "f32", cluster_size=1)  # 2 MB on one CTA
+        rs.plan(1, 2, rs.MAX_VOCAB, 1, "f32", cluster_size=1, kernel="resident")  # 2 MB on one CTA
+    o = rs.make_opts(kernel="stream")
+    o.flags |= rs.FLAG_RESIDENT                   # both kernels forced: argument error
+    assert lib.resispec_plan(rs.Dims(1, 2, 10, 1, rs.F32), o, None) == rs.E_ARG
 
 
 def test_no_cpu_path():

@@ -13,6 +13,7 @@ from tests.test_oracle_walk import chisq_pvalue
 
 pytestmark = pytest.mark.gpu
 MODES = [rs.MODE_RESISPEC, rs.MODE_SPECINFER]
+KERNELS = ["resident", "stream"]
 
 
 @pytest.fixture(scope="module", autouse=True)
@@ -58,78 +59,129 @@ def test_device_philox_matches_numpy():
             assert u1[i] == np.float32((int(blk[1]) >> 40) / 2.0 ** 24)
 
 
+@pytest.mark.parametrize("kernel", KERNELS)
 @pytest.mark.parametrize("mode", MODES)
 @pytest.mark.parametrize("cluster", [0, 1, 16])
-def test_parity_tiny_chain_10000(mode, cluster):
+def test_parity_tiny_chain_10000(mode, cluster, kernel):
     """Chain depth 4 with k = 3, V = 64, fp32: 10,000 independent problems
     from seed 0 (10,000 verify steps) in one batch."""
     w = W.WORKLOADS["tiny-chain-v64"]
     inp = W.make_inputs_np(w, seed=0, batch=10_000)
-    _check(inp, mode, seed=0, cluster_size=cluster)
+    _check(inp, mode, seed=0, cluster_size=cluster, kernel=kernel)
 
 
+@pytest.mark.parametrize("kernel", KERNELS)
 @pytest.mark.parametrize("mode", MODES)
-def test_parity_tree60_v32000(mode):
+def test_parity_tree60_v32000(mode, kernel):
     w = W.WORKLOADS["tree60-v32000"]
     inp = W.make_inputs_np(w, seed=1, batch=256)
-    _check(inp, mode, seed=11)
+    _check(inp, mode, seed=11, kernel=kernel)
 
 
-def test_parity_tree60_v32000_per_call_seeds():
+@pytest.mark.parametrize("kernel", KERNELS)
+def test_parity_tree60_v32000_per_call_seeds(kernel):
     """Batch 1, one call per step with seed = base + step (the paper's seed
     schedule), launch shape chosen automatically for a single sequence."""
     w = W.WORKLOADS["tree60-v32000"]
     for step in range(12):
         inp = W.make_inputs_np(w, seed=100 + step, batch=1)
-        _check(inp, rs.MODE_RESISPEC, seed=5000 + step)
+        _check(inp, rs.MODE_RESISPEC, seed=5000 + step, kernel=kernel)
 
 
+@pytest.mark.parametrize("kernel", KERNELS)
 @pytest.mark.parametrize("mode", MODES)
-def test_parity_chain8x4_v128256(mode):
+def test_parity_chain8x4_v128256(mode, kernel):
     w = W.WORKLOADS["chain8x4-v128256-b16"]
     for step in range(3):
         inp = W.make_inputs_np(w, seed=20 + step, batch=16)
-        _check(inp, mode, seed=900 + step)
+        _check(inp, mode, seed=900 + step, kernel=kernel)
 
 
-@pytest.mark.parametrize("V", [1, 2, 3, 7, 61, 999, 1000, 1003, 4104])
+@pytest.mark.parametrize("kernel", KERNELS)
+@pytest.mark.parametrize("V", [1, 2, 3, 7, 61, 999, 1000, 1003, 4104, 20000, 20001])
 @pytest.mark.parametrize("dtype", ["f32", "bf16"])
 @pytest.mark.parametrize("no_tma", [False, True])
-def test_parity_ragged_vocab(V, dtype, no_tma):
+def test_parity_ragged_vocab(V, dtype, no_tma, kernel):
     """Vocabularies that leave ragged slice tails, empty CTAs (V < cluster
-    slices) and rows that are not 16-byte aligned (plain-load path)."""
+    slices), slices of several streaming chunks with a ragged last chunk,
+    and rows that are not 16-byte aligned (plain-load path)."""
     base = W.Workload(name="ragged", batch=64, vocab=V, dtype=dtype, gen="gauss", scale=2.0,
                       slope=0.0, rho=0.6, temperature=0.9, tree=("levels", (3, 2, 1)), steps=1)
     inp = W.make_inputs_np(base, seed=V, batch=64)
-    for cluster in (0, 4, 11, 16):
+    for cluster in (0, 1, 4, 11, 16):
+        if kernel == "resident" and cluster == 1 and V > 4104:
+            continue  # two fp32 rows of V = 20001 do not fit one CTA's shared memory
         for mode in MODES:
-            _check(inp, mode, seed=V + cluster, cluster_size=cluster, no_tma=no_tma)
+            _check(inp, mode, seed=V + cluster, cluster_size=cluster, no_tma=no_tma,
+                   kernel=kernel)
 
 
+@pytest.mark.parametrize("kernel", KERNELS)
 @pytest.mark.parametrize("threads", [256, 512])
-def test_launch_shapes_agree(threads):
+def test_launch_shapes_agree(threads, kernel):
     w = W.WORKLOADS["tree60-v32000"]
     inp = W.make_inputs_np(w, seed=2, batch=64)
     ref = None
-    for cluster in (2, 3, 4, 8, 12, 16):   # one CTA cannot hold two V = 32000 fp32 rows
-        g, o = _check(inp, rs.MODE_RESISPEC, seed=3, cluster_size=cluster, block_threads=threads)
+    # one CTA cannot hold two V = 32000 fp32 rows (resident kernel)
+    clusters = (2, 3, 4, 8, 12, 16) if kernel == "resident" else (1, 2, 3, 5, 8, 16)
+    for cluster in clusters:
+        g, o = _check(inp, rs.MODE_RESISPEC, seed=3, cluster_size=cluster, block_threads=threads,
+                      kernel=kernel)
         clean = (o["accept_margin"] > P.ACCEPT_TIE) & (o["sample_margin"] > P.SAMPLE_TIE)
         if ref is not None:
             assert (g["tokens"][clean] == ref[clean]).all()
         ref = g["tokens"]
 
 
-def test_repeat_runs_bit_identical():
+def test_kernels_agree_away_from_ties():
+    """Both kernels on the same inputs: identical outputs wherever the
+    oracle sees no near tie."""
+    w = W.WORKLOADS["chain8x4-v128256-b16"]
+    inp = W.make_inputs_np(w, seed=7, batch=16)
+    g1, o = _check(inp, rs.MODE_RESISPEC, seed=70, kernel="resident")
+    g2, _ = _check(inp, rs.MODE_RESISPEC, seed=70, kernel="stream")
+    clean = (o["accept_margin"] > P.ACCEPT_TIE) & (o["sample_margin"] > P.SAMPLE_TIE)
+    assert (g1["tokens"][clean] == g2["tokens"][clean]).all()
+    assert (g1["accept_len"][clean] == g2["accept_len"][clean]).all()
+
+
+@pytest.mark.parametrize("kernel", KERNELS)
+def test_repeat_runs_bit_identical(kernel):
     w = W.WORKLOADS["chain8x4-v128256-b16"]
     inp = W.make_inputs_np(w, seed=5, batch=16)
     zt, zd, pa, ca = _np_inputs_to_gpu(inp)
-    a = P.run_gpu(zt, zd, pa, ca, inp["temperature"], 77, inp["max_depth"])
-    b = P.run_gpu(zt, zd, pa, ca, inp["temperature"], 77, inp["max_depth"])
+    a = P.run_gpu(zt, zd, pa, ca, inp["temperature"], 77, inp["max_depth"], kernel=kernel)
+    b = P.run_gpu(zt, zd, pa, ca, inp["temperature"], 77, inp["max_depth"], kernel=kernel)
     for k in ("tokens", "accept_len", "nodes", "rejects", "dist"):
         np.testing.assert_array_equal(a[k], b[k])
 
 
-def test_empty_tree_and_empty_batch():
+@pytest.mark.parametrize("mode", MODES)
+def test_wide_fanout(mode):
+    """A star of 128 children (the streaming kernel's limit) with weak drafts
+    (long rejection chains) on both kernels; 129 children: the streaming
+    kernel reports ERR_FANOUT, the resident kernel verifies."""
+    import torch
+    V = 3000
+    for kids in (128, 129):
+        parents = np.full(kids, -1, np.int32)
+        rng = np.random.default_rng(kids)
+        zt = rng.normal(0, 2, (8, kids + 1, V)).astype(np.float32)
+        zd = rng.normal(0, 2, (8, kids + 1, V)).astype(np.float32)
+        cand = rng.integers(0, V, (8, kids)).astype(np.int32)
+        inp = {"target": zt, "draft": zd, "parents": parents, "cand": cand, "temperature": 1.0,
+               "max_depth": 1}
+        _check(inp, mode, seed=kids, kernel="resident")
+        if kids <= rs.MAX_FANOUT_STREAM:
+            _check(inp, mode, seed=kids, kernel="stream")
+        else:
+            zt_, zd_, pa, ca = _np_inputs_to_gpu(inp)
+            g = P.run_gpu(zt_, zd_, pa, ca, 1.0, kids, 1, mode=mode, kernel="stream")
+            assert (g["accept_len"] == -1).all() and g["status"][0] == rs.ERR_FANOUT
+
+
+@pytest.mark.parametrize("kernel", KERNELS)
+def test_empty_tree_and_empty_batch(kernel):
     import torch
     V = 5000
     rng = np.random.default_rng(4)
@@ -137,7 +189,8 @@ def test_empty_tree_and_empty_batch():
     pa = np.zeros(0, np.int32)
     ca = np.zeros((40, 0), np.int32)
     g = P.run_gpu(P.to_device(zt), P.to_device(zt), torch.zeros(0, dtype=torch.int32, device="cuda"),
-                  torch.zeros((40, 0), dtype=torch.int32, device="cuda"), 1.0, 8, 0)
+                  torch.zeros((40, 0), dtype=torch.int32, device="cuda"), 1.0, 8, 0,
+                  kernel=kernel)
     o = P.run_oracle(zt, zt, pa, ca, 1.0, 8, 0, rs.MODE_RESISPEC)
     P.compare(g, o)
     assert (g["accept_len"] == 0).all()
@@ -148,7 +201,8 @@ def test_empty_tree_and_empty_batch():
     assert toks.shape == (0, 1) and alen.shape == (0,)
 
 
-def test_shared_rows_seq_stride_zero():
+@pytest.mark.parametrize("kernel", KERNELS)
+def test_shared_rows_seq_stride_zero(kernel):
     import torch
     w = W.WORKLOADS["tiny-chain-v64"]
     inp = W.make_inputs_np(w, seed=3, batch=1)
@@ -159,13 +213,14 @@ def test_shared_rows_seq_stride_zero():
     zd = P.to_device(inp["draft"][0])
     pa = torch.as_tensor(inp["parents"], device="cuda")
     g = P.run_gpu(zt, zd, pa, torch.as_tensor(cand, device="cuda"), 1.0, 6, w.max_depth,
-                  seq_stride=0)
+                  seq_stride=0, kernel=kernel)
     o = P.run_oracle(inp["target"][0], inp["draft"][0], inp["parents"], cand, 1.0, 6,
                      w.max_depth, rs.MODE_RESISPEC, seq_stride=0)
     P.compare(g, o)
 
 
-def test_error_contract_matches_oracle():
+@pytest.mark.parametrize("kernel", KERNELS)
+def test_error_contract_matches_oracle(kernel):
     import torch
     parents = W.tree_levels([2, 2])
     V, B = 1024, 9
@@ -182,7 +237,8 @@ def test_error_contract_matches_oracle():
     zt[8, 0, :] = -np.inf             # NaN hidden among -inf logits
     zt[8, 0, 517] = np.nan
     g = P.run_gpu(P.to_device(zt), P.to_device(zd), torch.as_tensor(parents, device="cuda"),
-                  torch.as_tensor(cand, device="cuda"), 1.0, 0, 2, want_dist=False)
+                  torch.as_tensor(cand, device="cuda"), 1.0, 0, 2, want_dist=False,
+                  kernel=kernel)
     o = P.run_oracle(zt, zd, parents, cand, 1.0, 0, 2, rs.MODE_RESISPEC, want_dist=False)
     np.testing.assert_array_equal(g["accept_len"] == -1, o["accept_len"] == -1)
     assert list(np.nonzero(o["accept_len"] == -1)[0]) == [1, 2, 3, 5, 6, 8]
@@ -192,11 +248,13 @@ def test_error_contract_matches_oracle():
     assert g["status"][0] & ~rs.INFO_DEGENERATE == want & ~oracle.INFO_DEGENERATE
     # depth overflow and a tree that is not in topological order
     g = P.run_gpu(P.to_device(zt[:1]), P.to_device(zd[:1]), torch.as_tensor(parents, device="cuda"),
-                  torch.as_tensor(cand[:1], device="cuda"), 1.0, 0, 1, want_dist=False)
+                  torch.as_tensor(cand[:1], device="cuda"), 1.0, 0, 1, want_dist=False,
+                  kernel=kernel)
     assert g["accept_len"][0] == -1 and g["status"][0] == rs.ERR_DEPTH
     bad = torch.as_tensor(np.array([-1, 1, 0, 0, 1, 1], np.int32), device="cuda")
     g = P.run_gpu(P.to_device(zt[:2]), P.to_device(zd[:2]), bad,
-                  torch.as_tensor(cand[:2], device="cuda"), 1.0, 0, 3, want_dist=False)
+                  torch.as_tensor(cand[:2], device="cuda"), 1.0, 0, 3, want_dist=False,
+                  kernel=kernel)
     assert (g["accept_len"] == -1).all() and g["status"][0] == rs.ERR_TREE
 
 
@@ -230,14 +288,15 @@ def test_nondefault_stream():
 # ------------------------------------------------------------ full-size workloads
 
 
-def _sampled_parity(w, seed, call_seed, rows, mode=rs.MODE_RESISPEC, batch=None, rho=None):
+def _sampled_parity(w, seed, call_seed, rows, mode=rs.MODE_RESISPEC, batch=None, rho=None,
+                    kernel=None):
     """Full-size inputs drawn on the GPU; the oracle recomputes the sampled
     sequences `rows` one by one from the same tensors."""
     import torch
     inp = W.make_inputs_torch(w, seed, "cuda", batch=batch, rho=rho)
     D = inp["max_depth"]
     g = P.run_gpu(inp["target"], inp["draft"], inp["parents"], inp["cand"], w.temperature,
-                  call_seed, D, mode=mode)
+                  call_seed, D, mode=mode, kernel=kernel)
     ridx = torch.as_tensor(rows, device="cuda")
     th = P.to_host_logits(inp["target"].index_select(0, ridx))
     dh = P.to_host_logits(inp["draft"].index_select(0, ridx))
@@ -253,34 +312,48 @@ def _sampled_parity(w, seed, call_seed, rows, mode=rs.MODE_RESISPEC, batch=None,
     return g
 
 
+@pytest.mark.parametrize("kernel", [None, "resident"])
 @pytest.mark.parametrize("rho", [0.5, 0.8, 0.95])
-def test_parity_binary5_v151936_full_size(rho):
+def test_parity_binary5_v151936_full_size(rho, kernel):
     """B = 64, V = 151936 fp32, full binary tree of depth 5, in the launch
-    shape the benchmark times; 8 sampled sequences per call checked."""
+    shape the benchmark times (kernel None: the automatic choice); 8 sampled
+    sequences per call checked."""
     w = W.WORKLOADS["binary5-v151936-b64"]
-    _sampled_parity(w, seed=31, call_seed=1000, rows=[0, 9, 17, 26, 35, 44, 53, 63], rho=rho)
+    _sampled_parity(w, seed=31, call_seed=1000, rows=[0, 9, 17, 26, 35, 44, 53, 63], rho=rho,
+                    kernel=kernel)
 
 
-def test_parity_binary5_specinfer_full_size():
+@pytest.mark.parametrize("kernel", KERNELS)
+def test_parity_binary5_specinfer_full_size(kernel):
     w = W.WORKLOADS["binary5-v151936-b64"]
-    _sampled_parity(w, seed=32, call_seed=1001, rows=[1, 20, 40, 62], mode=rs.MODE_SPECINFER)
+    _sampled_parity(w, seed=32, call_seed=1001, rows=[1, 20, 40, 62], mode=rs.MODE_SPECINFER,
+                    kernel=kernel)
 
 
+@pytest.mark.parametrize("kernel", KERNELS)
 @pytest.mark.parametrize("k", [2, 16])
-def test_parity_single_position_v256000(k):
+def test_parity_single_position_v256000(k, kernel):
     w = W.WORKLOADS[f"single-k{k}-v256000-b32"]
-    _sampled_parity(w, seed=40 + k, call_seed=77, rows=[0, 7, 15, 31])
+    _sampled_parity(w, seed=40 + k, call_seed=77, rows=[0, 7, 15, 31], kernel=kernel)
 
 
-def test_parity_tree488_v256000():
+def test_parity_single_position_v256000_b128():
+    """B = 128, k = 16, in the launch shape the benchmark times."""
+    w = W.WORKLOADS["single-k16-v256000-b128"]
+    _sampled_parity(w, seed=45, call_seed=79, rows=[0, 33, 64, 97, 127])
+
+
+@pytest.mark.parametrize("kernel", KERNELS)
+def test_parity_tree488_v256000(kernel):
     w = W.WORKLOADS["tree488-v256000-b32"]
-    _sampled_parity(w, seed=50, call_seed=78, rows=[0, 5], batch=6)
+    _sampled_parity(w, seed=50, call_seed=78, rows=[0, 5], batch=6, kernel=kernel)
 
 
 # ------------------------------------------------------------ exactness on the GPU
 
 
-def test_gpu_specinfer_million_draws_v32000():
+@pytest.mark.parametrize("kernel", KERNELS)
+def test_gpu_specinfer_million_draws_v32000(kernel):
     """SpecInfer mode is distribution-exact: 1e6 GPU draws at V = 32000 (one
     shared set of rows, fresh candidates per draw) do not reject p."""
     import torch
@@ -299,7 +372,8 @@ def test_gpu_specinfer_million_draws_v32000():
     cand = cand.view(n, k).contiguous()
     toks, alen = rs.verify(P.to_device(rows_t), P.to_device(rows_d),
                            torch.full((k,), -1, dtype=torch.int32, device="cuda"), cand, 1.0,
-                           2024, max_depth=1, mode=rs.MODE_SPECINFER, seq_stride=0)
+                           2024, max_depth=1, mode=rs.MODE_SPECINFER, seq_stride=0,
+                           kernel=kernel)
     first = toks[:, 0].to(torch.int64)
     assert int(first.min()) >= 0
     counts = torch.bincount(first, minlength=V).cpu().numpy()
@@ -308,7 +382,8 @@ def test_gpu_specinfer_million_draws_v32000():
     assert pv > 1e-4, (pv, nb)
 
 
-def test_gpu_resispec_million_draws_vs_enumerator():
+@pytest.mark.parametrize("kernel", KERNELS)
+def test_gpu_resispec_million_draws_vs_enumerator(kernel):
     """ResiSpec mode on the GPU follows the enumerated law of Algorithm 1
     (and not p: the documented bias)."""
     import torch
@@ -322,7 +397,7 @@ def test_gpu_resispec_million_draws_vs_enumerator():
                         P.to_device(np.broadcast_to(zd, (k + 1, V)).copy()),
                         torch.full((k,), -1, dtype=torch.int32, device="cuda"),
                         torch.as_tensor(cand, device="cuda"), 1.0, 99, max_depth=1,
-                        seq_stride=0)
+                        seq_stride=0, kernel=kernel)
     counts = np.bincount(toks[:, 0].cpu().numpy(), minlength=V)
     dist, _ = en.single_position(p, q, k, en.MODE_RESISPEC)
     assert chisq_pvalue(counts, dist)[0] > 1e-4

@@ -364,7 +364,7 @@ def run_ours(args):
             "temperature": w.temperature, "mode": args.mode,
             "parallelism": f"replicas{world}" if world > 1 else "single",
             "launch": {k: plan[k] for k in ("kernel_name", "cluster_size", "block_threads",
-                                            "smem_bytes", "slice_elems", "uses_tma", "stages",
+                                            "smem_bytes", "slice_elems", "uses_tma",
                                             "active_clusters")},
             "l2": f"rotating pool of {pool} input sets ({set_bytes / 1e9:.2f} GB each) "
                   f"between steps; each step's visited rows exceed L2 together",

@@ -97,9 +97,9 @@ typedef struct {
  *     entry per sequence), so only as many sequences as fit on chip run at
  *     once.  Any fan-out.
  *   STREAM: nothing but per-sequence scalars stays on chip; every pass
- *     streams the rows through a small shared-memory ring and the passes
- *     after the first read them from L2.  All sequences of a large batch run
- *     at once.  Fan-out up to RESISPEC_MAX_FANOUT_STREAM children per node.
+ *     streams the rows from global memory (the passes after a visit's first
+ *     read them from L2).  All sequences of a large batch run at once.
+ *     Fan-out up to RESISPEC_MAX_FANOUT_STREAM children per node.
  * The automatic choice takes RESIDENT when the whole batch fits on chip at
  * once, else STREAM. */
 #define RESISPEC_KERNEL_RESIDENT 0
@@ -161,7 +161,7 @@ typedef struct {
   int32_t smem_bytes;      /* dynamic shared memory per CTA */
   int32_t slice_elems;     /* vocabulary entries per CTA */
   int32_t uses_tma;        /* 1 if rows are fetched with bulk copies */
-  int32_t stages;          /* STREAM: shared-memory ring stages (0 for RESIDENT) */
+  int32_t reserved;        /* 0 */
   int32_t active_clusters; /* clusters of this shape resident at once on the
                               current device (0 without a device) */
 } resispec_plan_info;

@@ -50,7 +50,6 @@ struct Plan {
   int npad = 16;
   int smem = 0;
   int use_tma = 0;
-  int stages = 0;
   int active = 0;
 };
 
@@ -65,23 +64,14 @@ int tree_bytes(int npad) { return npad * 2 + (npad + 16) * 2 + npad * 2 + npad *
 
 int smem_for(int L, int npad) { return round_up(rs::kHeadBytes + 8 * L + tree_bytes(npad), 128); }
 
-// Streaming kernel: head, stream head, S ring stages of two chunk rows
-// (2 * threads 16-byte vectors each), then the tree.
-int stage_bytes(int threads) { return 2 * 2 * threads * 16; }
-
-int stream_smem_for(int threads, int S, int npad) {
-  return round_up(rs::kHeadBytes + rs::kStreamHeadBytes + S * stage_bytes(threads) +
-                      tree_bytes(npad), 128);
-}
-
-// Deepest ring (2..4 stages) that still lets `per_sm` CTAs share an SM.
-int stream_stages(int threads, int npad) {
-  const int per_sm = threads >= 512 ? 2 : 4;
-  const int budget = (228 * 1024) / per_sm - 1024;
-  int S = 2;
-  for (int s = 3; s <= rs::kMaxStages; ++s)
-    if (stream_smem_for(threads, s, npad) <= budget) S = s;
-  return S;
+// Streaming kernel: head, stream head, the cp.async ring (96 KB at 512
+// threads; the sampler's chunk buffer reuses one of its stages), then the
+// tree (parents, first children, next siblings, candidate tokens; the
+// uniforms are drawn per visit).
+int stream_smem_for(int threads, bool bf16, int npad) {
+  const int ring = bf16 ? rs::StreamGeom<512, true>::RING : rs::StreamGeom<512, false>::RING;
+  const int tree = npad * 2 + (npad + 16) * 2 + npad * 2 + npad * 4;
+  return round_up(rs::kHeadBytes + rs::kStreamHeadBytes + ring * threads / 512 + tree, 128);
 }
 
 struct DeviceInfo {
@@ -216,44 +206,48 @@ int plan_resident(const resispec_dims& d, int cs, int dev, int sms, Plan* p) {
   p->L = slice_for(V, p->C);
   p->smem = smem_for(p->L, p->npad);
   if (p->smem > kMaxSmem) return RESISPEC_E_SHAPE;
-  p->stages = 0;
   p->active = dev >= 0 ? active_clusters(dev, RESISPEC_KERNEL_RESIDENT, p->threads, bf16, p->C,
                                          p->smem)
                        : 0;
   return RESISPEC_OK;
 }
 
-// Streaming kernel: cluster size.  The batch runs in ceil(B / n) waves of n
-// resident clusters and a CTA's work shrinks as 1 / C, so C / waves is
-// maximised; ties go to the smaller cluster (cheaper exchanges, more
-// sequences overlapping their HBM-bound and ALU-bound passes).
+// Streaming kernel: cluster size.  A sequence's passes shrink as 1 / C,
+// and the batch runs in ceil(B / n) waves of n resident clusters; the
+// largest C whose waves stay within a small bound wins (per-sequence chains
+// differ in length, so the longest chain, run at C CTAs, sets the time).
+// Without a device, 2 CTAs of 512 threads per SM on 152 SMs are assumed and
+// a cluster of 16 is taken to fit 14 times (how many clusters of 16 CTAs
+// GB300 places at once), smaller ones in proportion.
 int plan_stream(const resispec_dims& d, int cs, int dev, int sms, Plan* p) {
   const bool bf16 = d.dtype == RESISPEC_BF16;
-  p->stages = stream_stages(p->threads, p->npad);
-  p->smem = stream_smem_for(p->threads, p->stages, p->npad);
+  p->smem = stream_smem_for(p->threads, bf16, p->npad);
   if (p->smem > kMaxSmem) return RESISPEC_E_SHAPE;
   const int B = std::max(d.batch, 1);
+  auto active_for = [&](int C) {
+    if (dev >= 0) return active_clusters(dev, RESISPEC_KERNEL_STREAM, p->threads, bf16, C, p->smem);
+    const int slots = (sms > 0 ? sms : 152) * (p->threads >= 512 ? 2 : 4);
+    return C == 16 ? 14 * slots / 304 : slots / C;
+  };
   if (cs) {
     p->C = cs;
-  } else if (dev >= 0) {
+  } else {
     int best = 0;
-    double best_score = -1.0;
-    for (int C = 1; C <= rs::kMaxCluster; ++C) {
-      const int n = active_clusters(dev, RESISPEC_KERNEL_STREAM, p->threads, bf16, C, p->smem);
+    for (int C : {16, 8, 4, 2, 1}) {
+      const int n = active_for(C);
       if (n <= 0) continue;
-      const double score = (double)C / (double)((B + n - 1) / n);
-      if (score > best_score) { best_score = score; best = C; }
+      const int waves = (B + n - 1) / n;
+      if (waves <= (C == 16 ? 2 : 4) || C == 1) {
+        best = C;
+        break;
+      }
     }
     if (best == 0) return RESISPEC_E_UNSUPPORTED;
     p->C = best;
-  } else {
-    const int slots = (sms > 0 ? sms : 152) * (p->threads >= 512 ? 2 : 4);
-    p->C = std::min(16, std::max(1, slots / B));
   }
   p->L = slice_for(d.vocab, p->C);
-  p->active = dev >= 0 ? active_clusters(dev, RESISPEC_KERNEL_STREAM, p->threads, bf16, p->C,
-                                         p->smem)
-                       : 0;
+  p->active = active_for(p->C);
+  if (dev < 0) p->active = 0;
   return RESISPEC_OK;
 }
 
@@ -392,7 +386,7 @@ int resispec_plan(resispec_dims dims, const resispec_opts* opts, resispec_plan_i
     out->smem_bytes = p.smem;
     out->slice_elems = p.L;
     out->uses_tma = p.use_tma;
-    out->stages = p.stages;
+    out->reserved = 0;
     out->active_clusters = p.active;
   }
   return RESISPEC_OK;
@@ -450,7 +444,6 @@ int resispec_verify_ex(const void* target_logits, const void* draft_logits,
   prm.mode = o.mode;
   prm.use_tma = pl.use_tma;
   prm.prefetch = (o.flags & RESISPEC_FLAG_PREFETCH) != 0;
-  prm.stages = pl.stages;
 
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   cudaError_t e;

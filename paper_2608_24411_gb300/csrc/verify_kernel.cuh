@@ -79,7 +79,6 @@ struct VerifyParams {
   int32_t mode;        // 0 ResiSpec, 1 SpecInfer
   int32_t use_tma;
   int32_t prefetch;    // L2 prefetch of the first child's rows
-  int32_t stages;      // streaming kernel: ring stages
 };
 
 struct __align__(16) Slot {

@@ -12,9 +12,15 @@
 // between the passes of a visit.  Rows are read from HBM once per visit.
 //
 // Passes.  Each CTA owns the slice [lo, lo + nloc) of the vocabulary and
-// streams it through a ring of S shared-memory stages, one chunk (2 THREADS
-// 16-byte vectors per row) per stage, filled by 1-D bulk copies (TMA) that
-// complete on one mbarrier per stage.  A visit runs
+// streams it in chunks of 8 logits per thread and row (two 16-byte fp32
+// vectors or one bf16 vector).  Every thread copies its own vectors of the
+// next S - 1 chunks into its own slots of a shared-memory ring with
+// cp.async (16-byte asynchronous copies) and reads back only what it copied
+// itself, so no barrier is needed between chunks and the bytes in flight
+// cost no registers.  With 1024 threads per SM this saturates HBM, and one
+// CTA alone streams about twice as fast as through a bulk-copy (TMA) ring
+// of the same size, whose single issuing thread and per-chunk barrier
+// limit it.  A visit runs
 //   NORM   online (reference, sum) of 2^(z c) per thread, c = log2(e) / T,
 //          then one cluster exchange gives the global (M, S) of each row;
 //   REJ    once per rejected candidate (Algorithm 1, GetProxy / Eq. recur):
@@ -30,23 +36,31 @@
 
 namespace rs {
 
-constexpr int kMaxStages = 4;
 constexpr int kMaxMaps = 128;          // residual maps per node (rejections with a map)
 constexpr int kMaxKids = kMaxMaps;      // children per node the streaming kernel walks
 constexpr int kErrFanout = 64;
 
+// Residual maps are kept in unnormalised units.  With p~ = 2^(z_t c - M_t)
+// and q~ = 2^(z_d c - M_d) (so p = p~ / S_t, q = q~ / S_d), the residual
+// after i maps is R_i = sigma_i R~_i, R~_0 = p~, sigma_0 = 1 / S_t, and map
+// i (Z_i, lambda_i, normaliser 1 / a_i) becomes, element-wise,
+//   ResiSpec:  m = min(k_i q~, R~), R~' = m + lambda_i (R~ - m),
+//   SpecInfer: R~' = (R~ - k_i q~)_+,
+// with k_i = Z_i / (S_d sigma_{i-1}) (ResiSpec) or 1 / (S_d sigma_{i-1})
+// (SpecInfer) and sigma_i = sigma_{i-1} a_i: every scale is folded into the
+// per-map scalar k_i and the running factor sigma.
 struct __align__(16) StreamHead {
-  unsigned long long fbar[kMaxStages];  // stage full barriers
-  float mZ[kMaxMaps];                   // ResiSpec budget Z of map i
-  float mlam[kMaxMaps];                 // ResiSpec filled fraction lambda of map i
-  float ma[kMaxMaps];                   // 1 / normaliser of map i
-  int rej[kMaxMaps];                    // tokens whose residual is 0 (ResiSpec maps)
-  float kzt[kMaxKids];                  // raw target / draft logits of the children's tokens
+  float mk[kMaxMaps];    // k_i of map i
+  float mlam[kMaxMaps];  // ResiSpec filled fraction lambda_i of map i
+  int rej[kMaxMaps];     // tokens whose residual is 0 (ResiSpec maps)
+  int rejk[kMaxMaps];    // their child index in this visit
+  float kzt[kMaxKids];   // raw target / draft logits of the children's tokens
   float kzd[kMaxKids];
-  int knode[kMaxKids];                  // the children, ascending
+  int16_t knode[kMaxKids];  // the children, ascending
+  float kua[kMaxKids];   // their accept draws U(seed, b, child + 1, 0)
+  float ufin;            // the visit's final draw U(seed, b, row, 1)
   int nkids;
   int nmaps;
-  int fz[4];
 };
 constexpr int kStreamHeadBytes = 4096;
 static_assert(sizeof(StreamHead) <= kStreamHeadBytes, "stream head too large");
@@ -54,48 +68,156 @@ static_assert(sizeof(StreamHead) <= kStreamHeadBytes, "stream head too large");
 template <int THREADS, bool BF16>
 struct StreamGeom {
   static constexpr int VEC = BF16 ? 8 : 4;            // elements per 16-byte vector
-  static constexpr int VPT = 2;                       // vectors per thread per chunk and row
-  static constexpr int CV = VPT * THREADS;            // vectors per chunk and row
-  static constexpr int CE = CV * VEC;                 // elements per chunk and row
-  static constexpr uint32_t RB = (uint32_t)CV * 16u;  // bytes per chunk and row
-  static constexpr uint32_t SB = 2u * RB;             // bytes per stage (target, draft)
+  static constexpr int VPT = BF16 ? 1 : 2;            // vectors per thread per chunk and row
+  static constexpr int NE = VPT * VEC;                // elements per thread per chunk and row (8)
+  static constexpr int CE = NE * THREADS;             // elements per chunk and row
+  static constexpr uint32_t RB = (uint32_t)VPT * THREADS * 16u;  // bytes per chunk and row
+  static constexpr uint32_t SB = 2u * RB;             // bytes per ring stage (target, draft)
+  static constexpr int S = BF16 ? 6 : 3;              // ring stages: 96 KB at 512 threads
+  static constexpr uint32_t RING = S * SB;
 };
 
-// Ring bookkeeping; every thread holds identical copies.
-struct Ring {
-  unsigned char* buf;  // S stages of SB bytes
-  uint32_t addr;       // shared address of buf
-  uint32_t bar0;       // shared address of fbar[0]
-  int S;
-  uint32_t issued;     // chunks issued so far
-  uint32_t consumed;   // chunks consumed so far
-  bool tma;
-  bool ok;             // false once a stage wait timed out
+__device__ __forceinline__ void cp_async16(void* dst, const void* src) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_addr(dst)), "l"(src)
+               : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() {
+  asm volatile("cp.async.commit_group;" ::: "memory");
+}
+template <int N>
+__device__ __forceinline__ void cp_async_wait() {
+  asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
+}
+
+// The rows one pass streams: element 0 of the CTA's slice in each row.
+struct Src {
+  const char* t;  // target row
+  const char* d;  // draft row (rows == 2)
+  int rows;
+  int nloc;
+  bool vec;       // 16-byte aligned rows: vector loads
 };
 
-// Raw logits of vector g of a stage row; elements at or beyond `valid` read
-// as -inf (the ragged end of a slice in the plain-load path).
 template <bool BF16>
-__device__ __forceinline__ void load_vec(const unsigned char* row, int g, int valid,
-                                         float (&z)[BF16 ? 8 : 4]) {
-  if constexpr (BF16) {
-    const uint4 r = reinterpret_cast<const uint4*>(row)[g];
-    const uint32_t w[4] = {r.x, r.y, r.z, r.w};
+__device__ __forceinline__ uint4 neg_inf_vec() {
+  const uint32_t w = BF16 ? 0xff80ff80u : 0xff800000u;
+  return make_uint4(w, w, w, w);
+}
+
+// The VEC values of one 16-byte vector.
+template <bool BF16>
+__device__ __forceinline__ void unpack_vec(const uint4& w, float (&z)[BF16 ? 8 : 4]) {
+  const uint32_t v[4] = {w.x, w.y, w.z, w.w};
 #pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      z[2 * j] = bf16_lo(w[j]);
-      z[2 * j + 1] = bf16_hi(w[j]);
+  for (int i = 0; i < 4; ++i) {
+    if constexpr (BF16) {
+      z[2 * i] = bf16_lo(v[i]);
+      z[2 * i + 1] = bf16_hi(v[i]);
+    } else {
+      z[i] = __uint_as_float(v[i]);
     }
-  } else {
-    const float4 r = reinterpret_cast<const float4*>(row)[g];
-    z[0] = r.x; z[1] = r.y; z[2] = r.z; z[3] = r.w;
   }
-  constexpr int VEC = BF16 ? 8 : 4;
-  if (valid < VEC) {
+}
+
+// Vector h of this thread in a ring stage row: slice element
+// k CE + (h THREADS + tid) VEC of chunk k.  Vectors past the slice hold
+// -inf (written by the copy step).
+__device__ __forceinline__ uint4 stage_vec(const unsigned char* row, int h, int threads) {
+  return reinterpret_cast<const uint4*>(row)[h * threads + (int)threadIdx.x];
+}
+
+// Copies this thread's vectors of chunk k into ring stage `st` (the copies
+// of one chunk form one cp.async group).  Aligned rows: 16-byte
+// asynchronous copies; other rows: element loads stored synchronously.
+template <int THREADS, bool BF16>
+__device__ __forceinline__ void copy_chunk(const Src& s, int k, unsigned char* st) {
+  using G = StreamGeom<THREADS, BF16>;
+  constexpr int VEC = G::VEC;
+  constexpr int es = BF16 ? 2 : 4;
+  const uint4 ninf = neg_inf_vec<BF16>();
 #pragma unroll
-    for (int j = 0; j < VEC; ++j)
-      if (j >= valid) z[j] = -INFINITY;
+  for (int h = 0; h < G::VPT; ++h) {
+    const int g = h * THREADS + (int)threadIdx.x;
+    const int e0 = k * G::CE + g * VEC;
+    uint4* dt = reinterpret_cast<uint4*>(st) + g;
+    uint4* dd = reinterpret_cast<uint4*>(st + G::RB) + g;
+    if (s.vec) {
+      // nloc is a multiple of VEC on this path: a vector is whole or absent
+      if (e0 < s.nloc) {
+        cp_async16(dt, s.t + (size_t)e0 * es);
+        if (s.rows == 2) cp_async16(dd, s.d + (size_t)e0 * es);
+      } else {
+        *dt = ninf;
+        *dd = ninf;
+      }
+    } else {
+      uint32_t wt[4], wd[4];
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        if constexpr (BF16) {
+          uint32_t lt[2], ld[2];
+#pragma unroll
+          for (int j = 0; j < 2; ++j) {
+            const int e = e0 + 2 * i + j;
+            const bool in = e < s.nloc;
+            lt[j] = in ? (uint32_t)__ldg(reinterpret_cast<const uint16_t*>(s.t) + e) : 0xff80u;
+            ld[j] = (in && s.rows == 2)
+                        ? (uint32_t)__ldg(reinterpret_cast<const uint16_t*>(s.d) + e)
+                        : 0xff80u;
+          }
+          wt[i] = lt[0] | (lt[1] << 16);
+          wd[i] = ld[0] | (ld[1] << 16);
+        } else {
+          const int e = e0 + i;
+          const bool in = e < s.nloc;
+          wt[i] = in ? __float_as_uint(__ldg(reinterpret_cast<const float*>(s.t) + e))
+                     : 0xff800000u;
+          wd[i] = (in && s.rows == 2)
+                      ? __float_as_uint(__ldg(reinterpret_cast<const float*>(s.d) + e))
+                      : 0xff800000u;
+        }
+      }
+      *dt = make_uint4(wt[0], wt[1], wt[2], wt[3]);
+      *dd = make_uint4(wd[0], wd[1], wd[2], wd[3]);
+    }
   }
+  cp_async_commit();
+}
+
+// Streams the slice chunk by chunk, S - 1 chunks ahead, calling
+// body(target_stage_row, draft_stage_row, k) with all threads; body returns
+// true (uniformly) to end the pass.  pre() runs once, after the first copies
+// are issued.  On return every copy of the pass has landed.
+template <int THREADS, bool BF16, class Pre, class Body>
+__device__ __forceinline__ void stream_pass_pre(unsigned char* ring, const Src& s, Pre&& pre,
+                                                Body&& body) {
+  using G = StreamGeom<THREADS, BF16>;
+  constexpr int S = G::S;
+  const int NK = (s.nloc + G::CE - 1) / G::CE;
+#pragma unroll
+  for (int k = 0; k < S - 1; ++k) {
+    if (k < NK) copy_chunk<THREADS, BF16>(s, k, ring + k * G::SB);
+    else cp_async_commit();
+  }
+  pre();
+  int slot = 0;
+  for (int k = 0; k < NK; ++k) {
+    const int kn = k + S - 1;
+    const int nslot = slot == 0 ? S - 1 : slot - 1;  // (k + S - 1) % S
+    if (kn < NK) copy_chunk<THREADS, BF16>(s, kn, ring + nslot * G::SB);
+    else cp_async_commit();
+    cp_async_wait<S - 1>();  // chunk k's copies (this thread's) have landed
+    const unsigned char* st = ring + slot * G::SB;
+    const bool stop = body(st, st + G::RB, k);
+    slot = slot == S - 1 ? 0 : slot + 1;
+    if (stop) break;
+  }
+  cp_async_wait<0>();
+}
+
+template <int THREADS, bool BF16, class Body>
+__device__ __forceinline__ void stream_pass(unsigned char* ring, const Src& s, Body&& body) {
+  stream_pass_pre<THREADS, BF16>(ring, s, [] {}, body);
 }
 
 __device__ __forceinline__ float raw_logit(const void* base, size_t i, bool bf16) {
@@ -106,102 +228,71 @@ __device__ __forceinline__ float raw_logit(const void* base, size_t i, bool bf16
   return __ldg(static_cast<const float*>(base) + i);
 }
 
-// Streams this CTA's slice of `rows` rows (1: target; 2: target and draft,
-// each starting at element `off` of its tensor) through the ring, calling
-// body(target_stage_row, draft_stage_row, k, clen) for chunk k of clen
-// elements with all threads.  body returns true (uniformly) to end the pass
-// after its chunk; copies already in flight are then waited for (bounded).
-// pre() runs once with all threads after the first copies are issued.
-template <int THREADS, bool BF16, class Pre, class Body>
-__device__ __forceinline__ void stream_pass_pre(Ring& R, const VerifyParams& P, int rows,
-                                                size_t off, int nloc, Pre&& pre, Body&& body) {
-  using G = StreamGeom<THREADS, BF16>;
-  constexpr uint32_t es = BF16 ? 2u : 4u;
-  const int NK = (nloc + G::CE - 1) / G::CE;
-  const char* st = static_cast<const char*>(P.zt) + off * es;
-  const char* sd = static_cast<const char*>(P.zd) + off * es;
-  auto issue = [&](int k) {
-    const uint32_t slot = R.issued % (uint32_t)R.S;
-    if (threadIdx.x == 0) {
-      const uint32_t bytes = (uint32_t)min(G::CE, nloc - k * G::CE) * es;
-      const uint32_t bar = R.bar0 + 8u * slot;
-      const uint32_t dst = R.addr + slot * G::SB;
-      fence_proxy_async_smem();  // earlier generic accesses to the stage come first
-      mbar_arrive_expect_tx(bar, (uint32_t)rows * bytes);
-      bulk_g2s(dst, st + (size_t)k * G::CE * es, bytes, bar);
-      if (rows == 2) bulk_g2s(dst + G::RB, sd + (size_t)k * G::CE * es, bytes, bar);
-    }
-    R.issued += 1;
-  };
-  if (R.tma)
-    for (int k = 0; k < min(R.S, NK); ++k) issue(k);
-  pre();
-  for (int k = 0; k < NK; ++k) {
-    const uint32_t slot = R.consumed % (uint32_t)R.S;
-    unsigned char* s0 = R.buf + slot * G::SB;
-    const int clen = min(G::CE, nloc - k * G::CE);
-    if (R.tma) {
-      // after one timed-out wait the pass runs on without waiting (the
-      // sequence reports ERR_TIMEOUT)
-      if (R.ok) R.ok = wait_bar(R.bar0 + 8u * slot, (R.consumed / (uint32_t)R.S) & 1u);
-    } else {
-      for (int w = 0; w < rows; ++w) {
-        if constexpr (BF16) {
-          const uint16_t* src = reinterpret_cast<const uint16_t*>(w ? sd : st) + (size_t)k * G::CE;
-          uint16_t* dst = reinterpret_cast<uint16_t*>(s0 + w * G::RB);
-          for (int i = threadIdx.x; i < clen; i += THREADS) dst[i] = __ldg(src + i);
-        } else {
-          const float* src = reinterpret_cast<const float*>(w ? sd : st) + (size_t)k * G::CE;
-          float* dst = reinterpret_cast<float*>(s0 + w * G::RB);
-          for (int i = threadIdx.x; i < clen; i += THREADS) dst[i] = __ldg(src + i);
-        }
-      }
-      __syncthreads();
-    }
-    const bool stop = body(s0, s0 + G::RB, k, clen);
-    R.consumed += 1;
-    __syncthreads();  // every thread is done with the stage
-    if (stop) break;
-    if (R.tma && k + R.S < NK) issue(k + R.S);
-  }
-  while (R.consumed < R.issued) {  // copies of an ended pass still land
-    const uint32_t slot = R.consumed % (uint32_t)R.S;
-    if (R.ok) R.ok = wait_bar(R.bar0 + 8u * slot, (R.consumed / (uint32_t)R.S) & 1u);
-    R.consumed += 1;
-  }
-}
+// Online (reference, sum) of 2^(z c) over one thread's values of a chunk,
+// for one or two rows at once (independent chains for the scheduler).  The
+// reference m (log2 units) starts at the sentinel -FLT_MAX and is raised to
+// the rounded product of the largest logit and c whenever a value exceeds
+// it; the sum is rescaled.  Tracking the maximum exactly keeps every 2^x
+// argument at or below 0, where its rounding is below 2^-24 absolute: a
+// reference lagging by d binary orders would cost up to d 2^-24 relative
+// error in each term, and the later passes compute p from the exact global
+// maximum, so the two would drift apart.  With the sentinel no branch is
+// needed for rows that are all -inf so far (2^(-inf) = 0), and NaN or +inf
+// still makes the sum non-finite (detected by the caller).
+constexpr float kNoRef = -FLT_MAX;
 
-template <int THREADS, bool BF16, class Body>
-__device__ __forceinline__ void stream_pass(Ring& R, const VerifyParams& P, int rows, size_t off,
-                                            int nloc, Body&& body) {
-  stream_pass_pre<THREADS, BF16>(R, P, rows, off, nloc, [] {}, body);
-}
-
-// Online (reference, sum) of 2^(z c) over one thread's values of a chunk:
-// the reference m (log2 units) is raised when a value exceeds it by more
-// than 64 binary orders, and the sum is rescaled.  NaN or +inf makes the
-// sum non-finite (detected by the caller).
 template <int N>
-__device__ __forceinline__ void norm_accumulate(const float (&z)[N], float c, float& m,
-                                                float& s) {
-  float vmax = -INFINITY;
+__device__ __forceinline__ float tree_max(const float (&z)[N]) {
+  float v[N];
 #pragma unroll
-  for (int j = 0; j < N; ++j) vmax = fmaxf(vmax, z[j]);
-  if (__fmaf_rn(vmax, c, -m) > kRebaseLog2) {
-    const float mnew = __fmul_rn(vmax, c);
-    if (m != -INFINITY) s = __fmul_rn(s, ex2(__fsub_rn(m, mnew)));
-    m = mnew;
+  for (int j = 0; j < N; ++j) v[j] = z[j];
+#pragma unroll
+  for (int w = N / 2; w > 0; w /= 2)
+#pragma unroll
+    for (int j = 0; j < w; ++j) v[j] = fmaxf(v[j], v[j + w]);
+  return v[0];
+}
+
+template <int N>
+__device__ __forceinline__ float tree_sum(float (&v)[N]) {
+#pragma unroll
+  for (int w = N / 2; w > 0; w /= 2)
+#pragma unroll
+    for (int j = 0; j < w; ++j) v[j] = __fadd_rn(v[j], v[j + w]);
+  return v[0];
+}
+
+__device__ __forceinline__ void rebase(float vmax, float c, float& m, float& s) {
+  const float mnew = __fmul_rn(vmax, c);
+  s = __fmul_rn(s, ex2(__fsub_rn(m, mnew)));  // 0 from the sentinel
+  m = mnew;
+}
+
+template <int N, bool TWO>
+__device__ __forceinline__ void norm_accumulate(const float (&zt)[N], const float (&zd)[N],
+                                                float c, float& mt, float& st, float& md,
+                                                float& sd) {
+  const float vt = tree_max<N>(zt);
+  const bool rt = __fmaf_rn(vt, c, -mt) > 0.f;
+  float vd = 0.f;
+  bool rd = false;
+  if constexpr (TWO) {
+    vd = tree_max<N>(zd);
+    rd = __fmaf_rn(vd, c, -md) > 0.f;
   }
-  if (m == -INFINITY) {  // nothing finite seen yet: every value is -inf or NaN
-#pragma unroll
-    for (int j = 0; j < N; ++j)
-      if (isnan(z[j])) s = __int_as_float(0x7fc00000);
-  } else {
-    float t = 0.f;
-#pragma unroll
-    for (int j = 0; j < N; ++j) t += ex2(__fmaf_rn(z[j], c, -m));
-    s += t;
+  if (rt || rd) {  // rare: a new reference for one of the rows
+    if (rt) rebase(vt, c, mt, st);
+    if constexpr (TWO)
+      if (rd) rebase(vd, c, md, sd);
   }
+  float et[N], ed[N];
+#pragma unroll
+  for (int j = 0; j < N; ++j) {
+    et[j] = ex2(__fmaf_rn(zt[j], c, -mt));
+    if constexpr (TWO) ed[j] = ex2(__fmaf_rn(zd[j], c, -md));
+  }
+  st = __fadd_rn(st, tree_sum<N>(et));
+  if constexpr (TWO) sd = __fadd_rn(sd, tree_sum<N>(ed));
 }
 
 // Cluster-wide scalars of a visit after the normaliser.
@@ -209,6 +300,7 @@ struct VisitScalars {
   float c;           // log2(e) / T
   float Mt, invSt;   // target: global reference, 1 / sum
   float Md, invSd;   // draft
+  float sig;         // sigma of the current residual (R = sig R~; 1 / S_t before any map)
 };
 
 // p and q of one element from its raw logits.
@@ -216,95 +308,109 @@ __device__ __forceinline__ float prob_of(float z, float c, float M, float inv) {
   return __fmul_rn(ex2(__fmaf_rn(z, c, -M)), inv);
 }
 
-// The residual after the first nm maps, element-wise (no rejected-token
-// zeroing: the caller applies it).  ResiSpec map: GetProxy residual
-// r = min(Z q, R) + lambda (R - min(Z q, R)), R' = r / sum r; SpecInfer map:
-// R' = (R - q)_+ / sum (Eq. recur).
+// 2^(z c - M): p~ or q~ of one element from its raw logit.
+__device__ __forceinline__ float exp_of(float z, float c, float M) {
+  return ex2(__fmaf_rn(z, c, -M));
+}
+
+// The unnormalised residual R~ after the first nm maps, element-wise (no
+// rejected-token zeroing: the caller applies it).  ResiSpec map: GetProxy
+// residual r = min(Z q, R) + lambda (R - min(Z q, R)), R' = r / sum r;
+// SpecInfer map: R' = (R - q)_+ / sum (Eq. recur); in the units above.
 template <bool RESI>
 __device__ __forceinline__ float apply_chain(const StreamHead& S2, int nm, float R, float q) {
   for (int i = 0; i < nm; ++i) {
     if constexpr (RESI) {
-      const float m = fminf(__fmul_rn(S2.mZ[i], q), R);
-      R = __fmul_rn(__fmaf_rn(S2.mlam[i], __fsub_rn(R, m), m), S2.ma[i]);
+      const float m = fminf(__fmul_rn(S2.mk[i], q), R);
+      R = __fmaf_rn(S2.mlam[i], __fsub_rn(R, m), m);
     } else {
-      R = __fmul_rn(fmaxf(__fsub_rn(R, q), 0.f), S2.ma[i]);
+      R = fmaxf(__fmaf_rn(-S2.mk[i], q, R), 0.f);
     }
   }
   return R;
 }
 
-template <int VEC, bool RESI>
-__device__ __forceinline__ void apply_chain_vec(const StreamHead& S2, int nm, float (&R)[VEC],
-                                                const float (&q)[VEC]) {
+template <int N, bool RESI>
+__device__ __forceinline__ void apply_chain_vec(const StreamHead& S2, int nm, float (&R)[N],
+                                                const float (&q)[N]) {
   for (int i = 0; i < nm; ++i) {
+    const float k = S2.mk[i];
     if constexpr (RESI) {
-      const float Z = S2.mZ[i], lam = S2.mlam[i], a = S2.ma[i];
+      const float lam = S2.mlam[i];
 #pragma unroll
-      for (int j = 0; j < VEC; ++j) {
-        const float m = fminf(__fmul_rn(Z, q[j]), R[j]);
-        R[j] = __fmul_rn(__fmaf_rn(lam, __fsub_rn(R[j], m), m), a);
+      for (int j = 0; j < N; ++j) {
+        const float m = fminf(__fmul_rn(k, q[j]), R[j]);
+        R[j] = __fmaf_rn(lam, __fsub_rn(R[j], m), m);
       }
     } else {
-      const float a = S2.ma[i];
 #pragma unroll
-      for (int j = 0; j < VEC; ++j) R[j] = __fmul_rn(fmaxf(__fsub_rn(R[j], q[j]), 0.f), a);
+      for (int j = 0; j < N; ++j) R[j] = fmaxf(__fmaf_rn(-k, q[j], R[j]), 0.f);
     }
   }
 }
 
 // Zero the residual at rejected tokens (ResiSpec: r(x0) = 0 and the later
-// maps keep a zero at zero) inside the vector starting at token `base`.
+// maps keep a zero at zero) in the vector whose first token is `base`.
 template <int VEC>
-__device__ __forceinline__ void zero_rejected(const StreamHead& S2, int nm, int base,
-                                              float (&R)[VEC]) {
+__device__ __forceinline__ void zero_rejected_vec(const StreamHead& S2, int nm, int base,
+                                                  float (&R)[VEC]) {
   for (int i = 0; i < nm; ++i) {
     const unsigned d = (unsigned)(S2.rej[i] - base);
-    if (d < (unsigned)VEC) {
 #pragma unroll
-      for (int j = 0; j < VEC; ++j)
-        if ((unsigned)j == d) R[j] = 0.f;
-    }
+    for (int j = 0; j < VEC; ++j)
+      if ((unsigned)j == d) R[j] = 0.f;
   }
 }
 
-// Final value (the distribution being sampled) of the VEC elements of a
-// vector: p when no map is pending, else the residual.
-template <int VEC>
+// Final values (the distribution being sampled) of vector h of a thread's
+// chunk: p when no map is pending, else the residual, R = sig R~ (zero at
+// the rejected tokens).  base: its first token.
+template <int THREADS, bool BF16>
 __device__ __forceinline__ void final_values(const StreamHead& S2, const VisitScalars& K,
-                                             bool resi, int nm, int base, const float (&zt)[VEC],
-                                             const float (&zd)[VEC], float (&v)[VEC]) {
+                                             bool resi, int nm, int base,
+                                             const unsigned char* rt, const unsigned char* rd,
+                                             int h, float (&v)[BF16 ? 8 : 4]) {
+  constexpr int VEC = BF16 ? 8 : 4;
+  unpack_vec<BF16>(stage_vec(rt, h, THREADS), v);
+  if (nm == 0) {
 #pragma unroll
-  for (int j = 0; j < VEC; ++j) v[j] = prob_of(zt[j], K.c, K.Mt, K.invSt);
-  if (nm == 0) return;
+    for (int j = 0; j < VEC; ++j) v[j] = prob_of(v[j], K.c, K.Mt, K.invSt);
+    return;
+  }
   float q[VEC];
+  unpack_vec<BF16>(stage_vec(rd, h, THREADS), q);
 #pragma unroll
-  for (int j = 0; j < VEC; ++j) q[j] = prob_of(zd[j], K.c, K.Md, K.invSd);
+  for (int j = 0; j < VEC; ++j) {
+    v[j] = exp_of(v[j], K.c, K.Mt);
+    q[j] = exp_of(q[j], K.c, K.Md);
+  }
   if (resi) {
     apply_chain_vec<VEC, true>(S2, nm, v, q);
-    zero_rejected<VEC>(S2, nm, base, v);
+    zero_rejected_vec<VEC>(S2, nm, base, v);
   } else {
     apply_chain_vec<VEC, false>(S2, nm, v, q);
   }
+#pragma unroll
+  for (int j = 0; j < VEC; ++j) v[j] = __fmul_rn(v[j], K.sig);
 }
 
 // ---------------------------------------------------------------- sampler
 // Inverse-CDF draw inside one CTA from fixed-point masses (as the resident
 // kernel's sampler): chunk totals locate the chunk that holds the threshold
-// `tau` (mass units 2^-44), the chunk's values are written to a free stage
-// as fp32, then NW contiguous warp segments, 32 lane ranges and one lane's
-// walk find the token.  If rounding leaves tau past the slice's own total,
-// the last token with positive mass is taken.  Returns the token's offset in
-// the slice (-1 if the slice has no mass).
+// `tau` (mass units 2^-44); the chunk's values are written to shared memory
+// F as fp32 in token order; then NW contiguous warp segments, 32 lane ranges
+// and one lane's walk find the token.  If rounding leaves tau past the
+// slice's own total, the last token with positive mass is taken.  Returns
+// the token's offset in the slice (-1 if the slice has no mass).
 template <int THREADS, bool BF16>
-__device__ int stream_search(Head& H, StreamHead& S2, Ring& R, const VerifyParams& P,
-                             const VisitScalars& K, bool resi, size_t off, int lo, int nloc,
+__device__ int stream_search(Head& H, const StreamHead& S2, float* F, unsigned char* ring,
+                             const Src& s, const VisitScalars& K, bool resi, int lo,
                              unsigned long long tau) {
   using G = StreamGeom<THREADS, BF16>;
   constexpr int VEC = G::VEC;
   constexpr int NW = THREADS / 32;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int nm = S2.nmaps;
-  const int rows = nm > 0 ? 2 : 1;
   if (threadIdx.x == 0) {
     H.misc[0] = -1;  // chunk holding tau
     H.misc[1] = -1;  // last chunk with mass
@@ -312,105 +418,53 @@ __device__ int stream_search(Head& H, StreamHead& S2, Ring& R, const VerifyParam
   }
   __syncthreads();
   unsigned long long run = 0;  // thread 0 only
-  stream_pass<THREADS, BF16>(R, P, rows, off, nloc,
-      [&](const unsigned char* rt, const unsigned char* rd, int k, int clen) -> bool {
-        unsigned long long acc = 0;
+  stream_pass<THREADS, BF16>(ring, s, [&](const unsigned char* rt, const unsigned char* rd,
+                                           int k) -> bool {
+    unsigned long long acc = 0;
 #pragma unroll
-        for (int h = 0; h < G::VPT; ++h) {
-          const int g = h * THREADS + (int)threadIdx.x;
-          if (g * VEC < clen) {
-            float zt[VEC], zd[VEC], v[VEC];
-            const int valid = min(VEC, clen - g * VEC);
-            load_vec<BF16>(rt, g, valid, zt);
-            if (rows == 2) load_vec<BF16>(rd, g, valid, zd);
-            else {
+    for (int h = 0; h < G::VPT; ++h) {
+      float v[VEC];
+      final_values<THREADS, BF16>(S2, K, resi, nm, lo + k * G::CE + (h * THREADS + (int)threadIdx.x) * VEC,
+                                  rt, rd, h, v);
 #pragma unroll
-              for (int j = 0; j < VEC; ++j) zd[j] = -INFINITY;
-            }
-            final_values<VEC>(S2, K, resi, nm, lo + k * G::CE + g * VEC, zt, zd, v);
-#pragma unroll
-            for (int j = 0; j < VEC; ++j) acc += to_fix(v[j]);
-          }
-        }
-        acc = warp_sum_u64(acc);
-        if (lane == 0) H.seg[warp] = acc;
-        __syncthreads();
-        if (threadIdx.x == 0) {
-          unsigned long long m = 0;
-          for (int w = 0; w < NW; ++w) m += H.seg[w];
-          if (m > 0) H.misc[1] = k;
-          if (H.misc[0] < 0) {
-            if (run + m > tau) { H.misc[0] = k; H.fixd[0] = tau - run; }
-            else run += m;
-          }
-        }
-        __syncthreads();
-        return H.misc[0] >= 0;
-      });
+      for (int j = 0; j < VEC; ++j) acc += to_fix(v[j]);
+    }
+    acc = warp_sum_u64(acc);
+    if (lane == 0) H.seg[warp] = acc;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      unsigned long long m = 0;
+      for (int w = 0; w < NW; ++w) m += H.seg[w];
+      if (m > 0) H.misc[1] = k;
+      if (H.misc[0] < 0) {
+        if (run + m > tau) { H.misc[0] = k; H.fixd[0] = tau - run; }
+        else run += m;
+      }
+    }
+    __syncthreads();
+    return H.misc[0] >= 0;
+  });
   const int kfound = H.misc[0];
   const int klast = H.misc[1];
   if (kfound < 0 && klast < 0) return -1;
   const bool force = kfound < 0;
   const int ks = force ? klast : kfound;
   const unsigned long long t = force ? 0ull : H.fixd[0];
-  // Load chunk ks into the next stage, write its values to the stage after.
-  const uint32_t slot = R.consumed % (uint32_t)R.S;
-  unsigned char* s0 = R.buf + slot * G::SB;
-  float* F = reinterpret_cast<float*>(R.buf + ((slot + 1) % (uint32_t)R.S) * G::SB);
-  const int clen = min(G::CE, nloc - ks * G::CE);
-  constexpr uint32_t es = BF16 ? 2u : 4u;
-  {
-    const char* st = static_cast<const char*>(P.zt) + (off + (size_t)ks * G::CE) * es;
-    const char* sd = static_cast<const char*>(P.zd) + (off + (size_t)ks * G::CE) * es;
-    if (R.tma) {
-      if (threadIdx.x == 0) {
-        const uint32_t bar = R.bar0 + 8u * slot;
-        fence_proxy_async_smem();
-        mbar_arrive_expect_tx(bar, (uint32_t)rows * (uint32_t)clen * es);
-        bulk_g2s(R.addr + slot * G::SB, st, (uint32_t)clen * es, bar);
-        if (rows == 2) bulk_g2s(R.addr + slot * G::SB + G::RB, sd, (uint32_t)clen * es, bar);
-      }
-      R.issued += 1;
-      if (R.ok) R.ok = wait_bar(R.bar0 + 8u * slot, (R.consumed / (uint32_t)R.S) & 1u);
-      R.consumed += 1;
-    } else {
-      for (int w = 0; w < rows; ++w) {
-        if constexpr (BF16) {
-          const uint16_t* src = reinterpret_cast<const uint16_t*>(w ? sd : st);
-          uint16_t* dst = reinterpret_cast<uint16_t*>(s0 + w * G::RB);
-          for (int i = threadIdx.x; i < clen; i += THREADS) dst[i] = __ldg(src + i);
-        } else {
-          const float* src = reinterpret_cast<const float*>(w ? sd : st);
-          float* dst = reinterpret_cast<float*>(s0 + w * G::RB);
-          for (int i = threadIdx.x; i < clen; i += THREADS) dst[i] = __ldg(src + i);
-        }
-      }
-      __syncthreads();
-    }
-  }
+  // the chosen chunk's values in token order (this thread's vectors, copied
+  // again into ring stage 0)
+  copy_chunk<THREADS, BF16>(s, ks, ring);
+  cp_async_wait<0>();
 #pragma unroll
   for (int h = 0; h < G::VPT; ++h) {
-    const int g = h * THREADS + (int)threadIdx.x;
     float v[VEC];
-    if (g * VEC < clen) {
-      float zt[VEC], zd[VEC];
-      const int valid = min(VEC, clen - g * VEC);
-      load_vec<BF16>(s0, g, valid, zt);
-      if (rows == 2) load_vec<BF16>(s0 + G::RB, g, valid, zd);
-      else {
-#pragma unroll
-        for (int j = 0; j < VEC; ++j) zd[j] = -INFINITY;
-      }
-      final_values<VEC>(S2, K, resi, nm, lo + ks * G::CE + g * VEC, zt, zd, v);
-    } else {
-#pragma unroll
-      for (int j = 0; j < VEC; ++j) v[j] = 0.f;
-    }
+    const int g = h * THREADS + (int)threadIdx.x;
+    final_values<THREADS, BF16>(S2, K, resi, nm, lo + ks * G::CE + g * VEC, ring, ring + G::RB, h,
+                                v);
 #pragma unroll
     for (int j = 0; j < VEC; ++j) F[g * VEC + j] = v[j];
   }
   __syncthreads();
-  // warp segments of SEG elements over the chunk (zeros past clen)
+  // warp segments of SEG elements over the chunk (zeros past the slice)
   constexpr int SEG = G::CE / NW;
   {
     const int s0i = warp * SEG;
@@ -478,55 +532,46 @@ __device__ int stream_search(Head& H, StreamHead& S2, Ring& R, const VerifyParam
   }
   __syncthreads();
   const int pick = H.misc[4];
-  __syncthreads();  // the stage holding F may be refilled afterwards
+  __syncthreads();
   return pick < 0 ? -1 : ks * G::CE + pick;
 }
 
 // Final draw of a visit: every CTA picks the CTA whose mass range holds
 // u * total (as the resident kernel's sampler); that CTA searches its slice.
 template <int THREADS, bool BF16>
-__device__ bool stream_sample(Head& H, StreamHead& S2, Ring& R, const VerifyParams& P,
-                              const VisitScalars& K, bool resi, int mass_kind, const Pending& Pm,
-                              float u, int b, int depth, size_t off, int lo, int nloc,
+__device__ bool stream_sample(Head& H, const StreamHead& S2, float* F, unsigned char* ring,
+                              const VerifyParams& P, const Src& s_in, const VisitScalars& K, bool resi, int mass_kind,
+                              const Pending& Pm, float u, int b, int depth, int lo,
                               uint32_t rank, uint32_t C, int& xp, uint32_t& xph, bool& timeout) {
   using G = StreamGeom<THREADS, BF16>;
   constexpr int VEC = G::VEC;
   constexpr int NW = THREADS / 32;
   const int nm = S2.nmaps;
-  const int rows = nm > 0 ? 2 : 1;
+  Src s = s_in;
+  s.rows = nm > 0 ? 2 : 1;
   if (P.out_dist || mass_kind == 0) {
     // every CTA: values of its slice (written out when asked) and their sum
     float* dist = P.out_dist ? P.out_dist + (size_t)b * P.V + lo : nullptr;
-    float s = 0.f;
-    stream_pass<THREADS, BF16>(R, P, rows, off, nloc,
-        [&](const unsigned char* rt, const unsigned char* rd, int k, int clen) -> bool {
+    float sum = 0.f;
+    stream_pass<THREADS, BF16>(ring, s, [&](const unsigned char* rt, const unsigned char* rd,
+                                             int k) -> bool {
 #pragma unroll
-          for (int h = 0; h < G::VPT; ++h) {
-            const int g = h * THREADS + (int)threadIdx.x;
-            if (g * VEC < clen) {
-              float zt[VEC], zd[VEC], v[VEC];
-              const int valid = min(VEC, clen - g * VEC);
-              load_vec<BF16>(rt, g, valid, zt);
-              if (rows == 2) load_vec<BF16>(rd, g, valid, zd);
-              else {
+      for (int h = 0; h < G::VPT; ++h) {
+        float v[VEC];
+        const int e0 = k * G::CE + (h * THREADS + (int)threadIdx.x) * VEC;  // offset in the slice
+        final_values<THREADS, BF16>(S2, K, resi, nm, lo + e0, rt, rd, h, v);
 #pragma unroll
-                for (int j = 0; j < VEC; ++j) zd[j] = -INFINITY;
-              }
-              final_values<VEC>(S2, K, resi, nm, lo + k * G::CE + g * VEC, zt, zd, v);
-#pragma unroll
-              for (int j = 0; j < VEC; ++j) {
-                s += v[j];
-                if (dist && j < valid) dist[k * G::CE + g * VEC + j] = v[j];
-              }
-            }
-          }
-          return false;
-        });
+        for (int j = 0; j < VEC; ++j) {
+          sum += v[j];
+          if (dist && e0 + j < s.nloc) dist[e0 + j] = v[j];
+        }
+      }
+      return false;
+    });
     if (mass_kind == 0) {
       float o[8];
       int of;
-      exchange<NW, false>(H, s, 0.f, 0.f, 0.f, R.ok ? 0 : kFlagTimeout, -1, xp, xph, rank, C, o,
-                          of);
+      exchange<NW, false>(H, sum, 0.f, 0.f, 0.f, 0, -1, xp, xph, rank, C, o, of);
       if (of & kFlagTimeout) { timeout = true; return true; }
       mass_kind = 4;
     }
@@ -558,7 +603,7 @@ __device__ bool stream_sample(Head& H, StreamHead& S2, Ring& R, const VerifyPara
   if ((int)rank != cstar) return true;
   // A slice whose exchange mass is positive but whose every element rounds
   // to zero mass yields its first token.
-  const int pick = stream_search<THREADS, BF16>(H, S2, R, P, K, resi, off, lo, nloc, tau);
+  const int pick = stream_search<THREADS, BF16>(H, S2, F, ring, s, K, resi, lo, tau);
   if (threadIdx.x == 0) P.out_tokens[(size_t)b * (P.D + 1) + depth] = lo + max(pick, 0);
   return true;
 }
@@ -570,17 +615,19 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
   using G = StreamGeom<THREADS, BF16>;
   constexpr int NW = THREADS / 32;
   constexpr int VEC = G::VEC;
+  constexpr int es = BF16 ? 2 : 4;
   extern __shared__ __align__(128) unsigned char smem[];
   Head& H = *reinterpret_cast<Head*>(smem);
   StreamHead& S2 = *reinterpret_cast<StreamHead*>(smem + kHeadBytes);
-  unsigned char* ring = smem + kHeadBytes + kStreamHeadBytes;
-  const int S = P.stages;
-  int16_t* par = reinterpret_cast<int16_t*>(ring + (size_t)S * G::SB);
+  unsigned char* ring = smem + kHeadBytes + kStreamHeadBytes;  // S stages of SB bytes
+  // the sampler's chunk buffer (CE floats): ring stage 1, free once a pass
+  // has drained (the sampler copies its chunk into stage 0)
+  float* F = reinterpret_cast<float*>(ring + G::SB);
+  static_assert(G::CE * 4 <= G::SB, "sampler buffer exceeds a ring stage");
+  int16_t* par = reinterpret_cast<int16_t*>(ring + G::RING);
   int16_t* first_child = par + P.npad;
   int16_t* next_sib = first_child + P.npad + 16;
   int32_t* cand_s = reinterpret_cast<int32_t*>(next_sib + P.npad);
-  float* u_acc = reinterpret_cast<float*>(cand_s + P.npad);  // [r]: accept test of node r - 1
-  float* u_fin = u_acc + P.npad;                             // [r]: final draw at row r
 
   const int tid = threadIdx.x;
   const uint32_t rank = cluster_ctarank();
@@ -595,7 +642,6 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
 
   if (tid < 4) H.pubv[tid] = 0.f;
   if (tid == 0) {
-    for (int s = 0; s < S; ++s) mbar_init(smem_addr(&S2.fbar[s]), 1);
     mbar_init(smem_addr(&H.xbar[0]), 1);
     mbar_init(smem_addr(&H.xbar[1]), 1);
     fence_mbar_init();
@@ -609,27 +655,10 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
     par[i] = (int16_t)(ok ? p : -2);
     cand_s[i] = __ldg(P.cand + (size_t)b * N + i);
   }
-  // One Philox block per logit row r: the accept draw of node r - 1 (word 0)
-  // and the final draw at row r (word 1).
-  for (int r = tid; r <= N; r += THREADS) {
-    const U64x4 blk = philox4x64_10((uint64_t)r, (uint64_t)(uint32_t)b, 0, 0, P.seed, 0);
-    u_acc[r] = u24(blk.w[0]);
-    u_fin[r] = u24(blk.w[1]);
-  }
   const bool tree_bad = __syncthreads_or(bad) != 0;
   build_children(par, first_child, next_sib, N);
   __syncthreads();
   cluster_sync();  // every peer has started: its receive slots may now be written
-
-  Ring R;
-  R.buf = ring;
-  R.addr = smem_addr(ring);
-  R.bar0 = smem_addr(&S2.fbar[0]);
-  R.S = S;
-  R.issued = 0;
-  R.consumed = 0;
-  R.tma = P.use_tma != 0;
-  R.ok = true;
 
   int err = tree_bad ? kErrTree : 0;
   int info = 0;
@@ -642,68 +671,63 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
     const int c1 = first_child[node + 1];
     const bool need_draft = c1 >= 0;
     const size_t rbase = (size_t)b * P.seq_stride + (size_t)row * V;
-    const size_t off = rbase + (size_t)lo;
+    Src src;
+    src.t = static_cast<const char*>(P.zt) + (rbase + (size_t)lo) * es;
+    src.d = static_cast<const char*>(P.zd) + (rbase + (size_t)lo) * es;
+    src.rows = need_draft ? 2 : 1;
+    src.nloc = nloc;
+    src.vec = P.use_tma != 0;
 
     // children of the node, ascending
     if (tid == 0) {
       int n = 0;
       for (int cn = c1; cn >= 0; cn = next_sib[cn]) {
         if (n == kMaxKids) { n = -1; break; }
-        S2.knode[n++] = cn;
+        S2.knode[n++] = (int16_t)cn;
       }
       S2.nkids = n;
       S2.nmaps = 0;
     }
     __syncthreads();
 
-    // ---- tempered normaliser (S2): online (reference, sum) per row; the
-    // children's tokens' raw logits are read (one thread per child) while
-    // the first chunks are in flight
-    float mt = -INFINITY, st = 0.f, md = -INFINITY, sd = 0.f;
-    stream_pass_pre<THREADS, BF16>(R, P, need_draft ? 2 : 1, off, nloc,
+    // ---- tempered normaliser (S2): online (reference, sum) per row; while
+    // the first chunks are in flight, one thread per child reads its token's
+    // raw logits and draws its accept uniform (one Philox block per logit
+    // row r: word 0 is the accept draw of node r - 1, word 1 the final draw
+    // at row r), and one more thread draws the visit's final uniform
+    float mt = kNoRef, st = 0.f, md = kNoRef, sd = 0.f;
+    stream_pass_pre<THREADS, BF16>(ring, src,
         [&] {
-          if (tid < S2.nkids) {
-            const int x = cand_s[S2.knode[tid]];
+          const int nk = S2.nkids;
+          if (tid < nk) {
+            const int cn = S2.knode[tid];
+            const int x = cand_s[cn];
             const bool okx = x >= 0 && x < V;
             S2.kzt[tid] = okx ? raw_logit(P.zt, rbase + (size_t)x, bf16) : 0.f;
             S2.kzd[tid] = okx ? raw_logit(P.zd, rbase + (size_t)x, bf16) : 0.f;
+            S2.kua[tid] = uniform_draw(P.seed, (uint32_t)b, (uint32_t)(cn + 1), 0);
+          } else if (tid == max(nk, 0)) {
+            S2.ufin = uniform_draw(P.seed, (uint32_t)b, (uint32_t)row, 1);
           }
         },
-        [&](const unsigned char* rt, const unsigned char* rd, int k, int clen) -> bool {
-          float zt[G::VPT * VEC];
+        [&](const unsigned char* rt, const unsigned char* rd, int) -> bool {
 #pragma unroll
           for (int h = 0; h < G::VPT; ++h) {
-            const int g = h * THREADS + tid;
-            float z[VEC];
-            if (g * VEC < clen) load_vec<BF16>(rt, g, min(VEC, clen - g * VEC), z);
-            else {
-#pragma unroll
-              for (int j = 0; j < VEC; ++j) z[j] = -INFINITY;
+            float zt[VEC], zd[VEC];
+            unpack_vec<BF16>(stage_vec(rt, h, THREADS), zt);
+            if (need_draft) {
+              unpack_vec<BF16>(stage_vec(rd, h, THREADS), zd);
+              norm_accumulate<VEC, true>(zt, zd, P.scale_log2, mt, st, md, sd);
+            } else {
+              norm_accumulate<VEC, false>(zt, zd, P.scale_log2, mt, st, md, sd);
             }
-#pragma unroll
-            for (int j = 0; j < VEC; ++j) zt[h * VEC + j] = z[j];
-          }
-          norm_accumulate<G::VPT * VEC>(zt, P.scale_log2, mt, st);
-          if (need_draft) {
-#pragma unroll
-            for (int h = 0; h < G::VPT; ++h) {
-              const int g = h * THREADS + tid;
-              float z[VEC];
-              if (g * VEC < clen) load_vec<BF16>(rd, g, min(VEC, clen - g * VEC), z);
-              else {
-#pragma unroll
-                for (int j = 0; j < VEC; ++j) z[j] = -INFINITY;
-              }
-#pragma unroll
-              for (int j = 0; j < VEC; ++j) zt[h * VEC + j] = z[j];
-            }
-            norm_accumulate<G::VPT * VEC>(zt, P.scale_log2, md, sd);
           }
           return false;
         });
+    if (mt == kNoRef) mt = -INFINITY;  // no finite logit: the exchange's "no mass" marker
+    if (md == kNoRef) md = -INFINITY;
     const bool bad_t = !(st <= FLT_MAX), bad_d = !(sd <= FLT_MAX);
-    const int flags = (bad_t ? kFlagTargetBad : 0) | (bad_d ? kFlagDraftBad : 0) |
-                      (R.ok ? 0 : kFlagTimeout);
+    const int flags = (bad_t ? kFlagTargetBad : 0) | (bad_d ? kFlagDraftBad : 0);
     float o[8];
     int oflags;
     exchange<NW, true>(H, mt, st, md, sd, flags, -1, xp, xph, rank, C, o, oflags);
@@ -718,16 +742,17 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
     K.invSt = __frcp_rn(o[1]);
     K.Md = o[2];
     K.invSd = need_draft ? __frcp_rn(o[3]) : 0.f;
+    K.sig = K.invSt;
     Pending Pm{kScale, -1, 0.f, 0.f, 0.f};  // parameters of the latest map (sampler masses)
     int mass_kind = 1;
 
     if (!need_draft) {
       // accepted leaf (or a root without children): bonus token from p
       bool to = false;
-      if (!stream_sample<THREADS, BF16>(H, S2, R, P, K, resi, mass_kind, Pm, u_fin[row], b, depth,
-                                        off, lo, nloc, rank, C, xp, xph, to))
+      if (!stream_sample<THREADS, BF16>(H, S2, F, ring, P, src, K, resi, mass_kind, Pm, S2.ufin,
+                                        b, depth, lo, rank, C, xp, xph, to))
         err |= kErrEmpty;
-      if (to || !R.ok) err |= kErrTimeout;
+      if (to) err |= kErrTimeout;
       break;
     }
     const int nk = S2.nkids;  // written by thread 0 before the exchange's barriers
@@ -740,16 +765,18 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
       const int x = cand_s[cn];
       if (x < 0 || x >= V) { err |= kErrToken; break; }
       const int nm = S2.nmaps;
-      const float qx = prob_of(S2.kzd[i], K.c, K.Md, K.invSd);
-      float Rx = prob_of(S2.kzt[i], K.c, K.Mt, K.invSt);
+      const float qt = exp_of(S2.kzd[i], K.c, K.Md);
+      const float qx = __fmul_rn(qt, K.invSd);
+      float Rt = exp_of(S2.kzt[i], K.c, K.Mt);
       if (resi) {
-        Rx = apply_chain<true>(S2, nm, Rx, qx);
+        Rt = apply_chain<true>(S2, nm, Rt, qt);
         for (int j = 0; j < nm; ++j)
-          if (S2.rej[j] == x) Rx = 0.f;
+          if (S2.rej[j] == x) Rt = 0.f;
       } else {
-        Rx = apply_chain<false>(S2, nm, Rx, qx);
+        Rt = apply_chain<false>(S2, nm, Rt, qt);
       }
-      const float u = u_acc[cn + 1];
+      const float Rx = __fmul_rn(Rt, K.sig);
+      const float u = S2.kua[i];
       if (__fmul_rn(u, qx) < Rx) { accepted = cn; acc_tok = x; break; }
       rejects += 1;
       float Z = 0.f;
@@ -761,72 +788,94 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
         }
       }
       if (nm >= kMaxMaps) { err |= kErrFanout; break; }
-      // one pass: the residual so far and the sums of the new map
+      // one pass: the residual so far and the sums of the new map, in
+      // unnormalised units (k: the new map's scalar).  The rejected tokens
+      // get no special case here; their terms are taken out below.
+      const float kq = __fdiv_rn(resi ? __fmul_rn(Z, K.invSd) : K.invSd, K.sig);
       float s1 = 0.f, s2 = 0.f;
-      stream_pass<THREADS, BF16>(R, P, 2, off, nloc,
-          [&](const unsigned char* rt, const unsigned char* rd, int k, int clen) -> bool {
+      stream_pass<THREADS, BF16>(ring, src, [&](const unsigned char* rt, const unsigned char* rd,
+                                                int) -> bool {
 #pragma unroll
-            for (int h = 0; h < G::VPT; ++h) {
-              const int g = h * THREADS + tid;
-              if (g * VEC < clen) {
-                float zt[VEC], zd[VEC], Rv[VEC], q[VEC];
-                const int valid = min(VEC, clen - g * VEC);
-                load_vec<BF16>(rt, g, valid, zt);
-                load_vec<BF16>(rd, g, valid, zd);
-                const int base = lo + k * G::CE + g * VEC;
+        for (int h = 0; h < G::VPT; ++h) {
+          float Rv[VEC], q[VEC];
+          unpack_vec<BF16>(stage_vec(rt, h, THREADS), Rv);  // -inf past the slice: 0
+          unpack_vec<BF16>(stage_vec(rd, h, THREADS), q);
 #pragma unroll
-                for (int j = 0; j < VEC; ++j) {
-                  Rv[j] = prob_of(zt[j], K.c, K.Mt, K.invSt);
-                  q[j] = prob_of(zd[j], K.c, K.Md, K.invSd);
-                }
-                if (resi) {
-                  apply_chain_vec<VEC, true>(S2, nm, Rv, q);
-                  zero_rejected<VEC>(S2, nm, base, Rv);
-                  const unsigned dx = (unsigned)(x - base);
+          for (int j = 0; j < VEC; ++j) {
+            Rv[j] = exp_of(Rv[j], K.c, K.Mt);
+            q[j] = exp_of(q[j], K.c, K.Md);
+          }
+          float a1[VEC], a2[VEC];
+          if (resi) {
+            apply_chain_vec<VEC, true>(S2, nm, Rv, q);
 #pragma unroll
-                  for (int j = 0; j < VEC; ++j) {
-                    if ((unsigned)j == dx) continue;  // the rejected token: r(x0) = 0
-                    const float m = fminf(__fmul_rn(Z, q[j]), Rv[j]);
-                    s1 += m;
-                    s2 += __fsub_rn(Rv[j], m);
-                  }
-                } else {
-                  apply_chain_vec<VEC, false>(S2, nm, Rv, q);
-#pragma unroll
-                  for (int j = 0; j < VEC; ++j) s1 += fmaxf(__fsub_rn(Rv[j], q[j]), 0.f);
-                }
-              }
+            for (int j = 0; j < VEC; ++j) {
+              a1[j] = fminf(__fmul_rn(kq, q[j]), Rv[j]);
+              a2[j] = __fsub_rn(Rv[j], a1[j]);
             }
-            return false;
-          });
-      exchange<NW, false>(H, s1, s2, 0.f, 0.f, R.ok ? 0 : kFlagTimeout, -1, xp, xph, rank, C, o,
-                          oflags);
+            s1 = __fadd_rn(s1, tree_sum<VEC>(a1));
+            s2 = __fadd_rn(s2, tree_sum<VEC>(a2));
+          } else {
+            apply_chain_vec<VEC, false>(S2, nm, Rv, q);
+#pragma unroll
+            for (int j = 0; j < VEC; ++j) a1[j] = fmaxf(__fmaf_rn(-kq, q[j], Rv[j]), 0.f);
+            s1 = __fadd_rn(s1, tree_sum<VEC>(a1));
+          }
+        }
+        return false;
+      });
+      if (resi) {
+        // The token just rejected (r(x0) = 0) and the earlier rejected ones
+        // (R = 0 there) add nothing: the thread that summed each such token
+        // of this slice subtracts the terms the pass gave it, recomputed
+        // bit for bit (each distinct token once).
+        for (int t = -1; t < nm; ++t) {
+          const int y = t < 0 ? x : S2.rej[t];
+          const int yk = t < 0 ? i : S2.rejk[t];
+          if (y < lo || y >= lo + nloc) continue;
+          if ((((y - lo) % G::CE) / VEC) % THREADS != tid) continue;
+          bool seen = t >= 0 && y == x;
+          for (int t2 = 0; t2 < t && !seen; ++t2) seen = S2.rej[t2] == y;
+          if (seen) continue;
+          const float qy = exp_of(S2.kzd[yk], K.c, K.Md);
+          const float Ry = apply_chain<true>(S2, nm, exp_of(S2.kzt[yk], K.c, K.Mt), qy);
+          const float my = fminf(__fmul_rn(kq, qy), Ry);
+          s1 = __fsub_rn(s1, my);
+          s2 = __fsub_rn(s2, __fsub_rn(Ry, my));
+        }
+      }
+      exchange<NW, false>(H, s1, s2, 0.f, 0.f, 0, -1, xp, xph, rank, C, o, oflags);
       if (oflags & kFlagTimeout) { err |= kErrTimeout; break; }
       bool has_map = false;
       float a = 0.f, lam = 0.f;
       if (resi) {
-        const float S1 = o[0], S2s = o[1];
+        const float S1 = __fmul_rn(o[0], K.sig), S2s = __fmul_rn(o[1], K.sig);
         const float delta = __fsub_rn(Z, S1);
         lam = S2s > 0.f ? fminf(fmaxf(__fdiv_rn(delta, S2s), 0.f), 1.f) : 0.f;
         const float norm = __fmaf_rn(lam, S2s, S1);
         if (norm > 0.f) {
           has_map = true;
           a = __frcp_rn(norm);
-          Pm = Pending{kResi, x, a, Z, lam};
           mass_kind = 2;
         }
-      } else if (o[0] > 0.f) {
-        has_map = true;
-        a = __frcp_rn(o[0]);
-        Pm = Pending{kSpec, -1, a, 0.f, 0.f};
-        mass_kind = 3;
+      } else {
+        const float Ssum = __fmul_rn(o[0], K.sig);
+        if (Ssum > 0.f) {
+          has_map = true;
+          a = __frcp_rn(Ssum);
+          mass_kind = 3;
+        }
       }
       if (has_map) {
+        K.sig = __fmul_rn(K.sig, a);
+        // per-CTA masses of the new residual: (p0 + lambda p1) sig (ResiSpec)
+        // or p0 sig (SpecInfer) from this exchange's unnormalised partials
+        Pm = Pending{resi ? kResi : kSpec, x, K.sig, Z, lam};
         if (tid == 0) {
-          S2.mZ[nm] = Z;
+          S2.mk[nm] = kq;
           S2.mlam[nm] = lam;
-          S2.ma[nm] = a;
           S2.rej[nm] = x;
+          S2.rejk[nm] = i;
           S2.nmaps = nm + 1;
         }
         __syncthreads();
@@ -840,10 +889,10 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
     if (accepted < 0) {
       // every child rejected: residual draw (Algorithm 1, last step)
       bool to = false;
-      if (!stream_sample<THREADS, BF16>(H, S2, R, P, K, resi, mass_kind, Pm, u_fin[row], b, depth,
-                                        off, lo, nloc, rank, C, xp, xph, to))
+      if (!stream_sample<THREADS, BF16>(H, S2, F, ring, P, src, K, resi, mass_kind, Pm, S2.ufin,
+                                        b, depth, lo, rank, C, xp, xph, to))
         err |= kErrEmpty;
-      if (to || !R.ok) err |= kErrTimeout;
+      if (to) err |= kErrTimeout;
       break;
     }
     if (depth >= D) { err |= kErrDepth; break; }

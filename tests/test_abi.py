@@ -75,16 +75,19 @@ def test_synchronous_argument_errors(lib):
 
 def test_plan_without_device(lib):
     # the bench workload (B = 64, V = 151936 fp32) cannot sit on chip at once:
-    # the automatic choice streams it, four CTAs per sequence
+    # the automatic choice streams it, in clusters of 8 CTAs (two waves)
     p = rs.plan(64, 62, 151936, 5, "f32")
-    assert p["kernel_name"] == "stream" and p["cluster_size"] == 4
-    assert p["stages"] >= 2 and p["smem_bytes"] <= 113 * 1024   # two CTAs per SM
-    assert p["slice_elems"] % 8 == 0 and p["slice_elems"] * 4 >= 151936
+    assert p["kernel_name"] == "stream" and p["cluster_size"] == 8
+    assert p["smem_bytes"] <= 228 * 1024 // 2 - 1024   # two CTAs per SM
+    assert p["slice_elems"] % 8 == 0 and p["slice_elems"] * 8 >= 151936
     assert p["uses_tma"] == 1
+    for B in (1, 7, 64, 128, 1000):
+        p = rs.plan(B, 488, 256000, 6, "bf16", kernel="stream")
+        assert p["smem_bytes"] <= 228 * 1024 // 2 - 1024
     p = rs.plan(64, 62, 151936, 5, "f32", kernel="resident")
     assert p["kernel_name"] == "resident" and p["cluster_size"] in (8, 16)
     assert p["slice_elems"] * p["cluster_size"] >= 151936
-    assert p["smem_bytes"] <= 227 * 1024 and p["stages"] == 0
+    assert p["smem_bytes"] <= 227 * 1024
     # a small batch that fits on chip stays resident
     p = rs.plan(1, 60, 32000, 5, "bf16")
     assert p["kernel_name"] == "resident"
@@ -98,8 +101,7 @@ def test_plan_without_device(lib):
         for kernel in ("resident", "stream"):
             p = rs.plan(128, 488, V, 6, "bf16", kernel=kernel)
             assert p["smem_bytes"] <= 227 * 1024
-    # streaming: C / waves over 2 CTAs per SM (152 SMs without a device)
-    assert rs.plan(128, 16, 256000, 1, "bf16")["cluster_size"] == 2
+    # streaming: the largest cluster size within the wave bound
     assert rs.plan(16, 32, 128256, 4, "bf16", kernel="stream")["cluster_size"] == 16
     # the streaming kernel holds no rows: one CTA per sequence at any V
     p = rs.plan(1, 2, rs.MAX_VOCAB, 1, "f32", cluster_size=1, kernel="stream")

@@ -158,12 +158,12 @@ def test_repeat_runs_bit_identical(kernel):
 
 @pytest.mark.parametrize("mode", MODES)
 def test_wide_fanout(mode):
-    """A star of 128 children (the streaming kernel's limit) with weak drafts
-    (long rejection chains) on both kernels; 129 children: the streaming
+    """A star of MAX_FANOUT_STREAM children (the streaming kernel's limit) with weak drafts
+    (long rejection chains) on both kernels; one child more: the streaming
     kernel reports ERR_FANOUT, the resident kernel verifies."""
     import torch
     V = 3000
-    for kids in (128, 129):
+    for kids in (rs.MAX_FANOUT_STREAM, rs.MAX_FANOUT_STREAM + 1):
         parents = np.full(kids, -1, np.int32)
         rng = np.random.default_rng(kids)
         zt = rng.normal(0, 2, (8, kids + 1, V)).astype(np.float32)

@@ -84,18 +84,21 @@ def kernel_source_digest():
     return h.hexdigest()[:16]
 
 
-def profiled_traffic(kernel, workload):
-    """DRAM bytes per launch from the committed ncu summary of this kernel
-    on this workload, if it was taken on the current kernel source."""
+def profiled_traffic(kernel, workload, alg_bytes_per_launch):
+    """DRAM bytes per launch: the committed ncu summary of this kernel on
+    this workload gives DRAM bytes per algorithmic byte (measured on a
+    smaller case of the same kernel); traffic grows with the rows visited,
+    so it is scaled by this run's algorithmic bytes per launch.  None unless
+    the summary was taken on the current kernel source."""
     path = os.path.join(ROOT, "profiles", f"{kernel}_kernel_{workload}.md")
     if not os.path.exists(path):
         return None
     text = open(path).read()
     m_src = re.search(r"kernel_source_digest:\s*([0-9a-f]+)", text)
-    m_tr = re.search(r"dram_bytes_per_launch:\s*([0-9.eE+]+)", text)
+    m_tr = re.search(r"dram_bytes_per_alg_byte:\s*([0-9.eE+]+)", text)
     if not m_src or not m_tr or m_src.group(1) != kernel_source_digest():
         return None
-    return float(m_tr.group(1))
+    return float(m_tr.group(1)) * alg_bytes_per_launch
 
 
 # ------------------------------------------------------------------ clocks
@@ -194,6 +197,59 @@ def cpu_oracle_rate(w, target_h, draft_h, parents, cand_h, seq_ids, mode, second
     return nodes / el, threads, sample
 
 
+# ------------------------------------------------------------------ ranks
+
+
+def rank_layout():
+    """(rank, local rank, world size) from the launcher's environment."""
+    return (int(os.environ.get("RANK", "0")), int(os.environ.get("LOCAL_RANK", "0")),
+            int(os.environ.get("WORLD_SIZE", "1")))
+
+
+def replica_seed(seed, rank, i):
+    """Seed of input set i on `rank`: every replica verifies its own data
+    (weak scaling, no exchange between ranks)."""
+    return seed + 7919 * rank + 31 * i
+
+
+class RankGroup:
+    """Barrier and scalar reductions over the ranks of a replicas run (one
+    process per GPU).  The path has no data exchange between ranks: these
+    calls only bracket the timed region and combine its timings.  With
+    dist None (one process) every call is local."""
+
+    def __init__(self, dist=None, device=None):
+        self.dist = dist
+        self.device = device
+
+    def barrier(self):
+        if self.dist is not None:
+            self.dist.barrier()
+
+    def _reduce(self, x, op):
+        if self.dist is None:
+            return float(x)
+        import torch
+        t = torch.tensor([float(x)], dtype=torch.float64, device=self.device)
+        self.dist.all_reduce(t, op=op)
+        return float(t.item())
+
+    def max(self, x):
+        return self._reduce(x, None if self.dist is None else self.dist.ReduceOp.MAX)
+
+    def sum(self, x):
+        return self._reduce(x, None if self.dist is None else self.dist.ReduceOp.SUM)
+
+
+def whole_job_rate(group, units_this_rank, elapsed_ms_this_rank):
+    """Whole-job throughput: the units all ranks processed over the slowest
+    rank's time (max over ranks, the timed region of every rank bracketed by
+    a barrier)."""
+    total = group.sum(units_this_rank)
+    slowest_ms = group.max(elapsed_ms_this_rank)
+    return total / (slowest_ms / 1e3), slowest_ms
+
+
 # ------------------------------------------------------------------ reference arm
 
 
@@ -201,9 +257,9 @@ def run_reference(args):
     """The oracle as it stands on the host cores, on this arm's workload."""
     import oracle
     from paper_2608_24411_gb300 import workloads as W
-    rank = int(os.environ.get("RANK", "0"))
+    rank, _, _ = rank_layout()
     if rank != 0:
-        return 0
+        return 0  # under torchrun rank 0 alone times the oracle
     w = W.WORKLOADS[args.workload]
     if args.rho is not None:
         w = W.with_rho(w, args.rho)
@@ -249,9 +305,7 @@ def run_ours(args):
     import paper_2608_24411_gb300 as rs
     from paper_2608_24411_gb300 import workloads as W
 
-    world = int(os.environ.get("WORLD_SIZE", "1"))
-    rank = int(os.environ.get("RANK", "0"))
-    local = int(os.environ.get("LOCAL_RANK", "0"))
+    rank, local, world = rank_layout()
     if world != args.gpus and world > 1:
         raise SystemExit(f"--gpus {args.gpus} but WORLD_SIZE {world}")
     torch.cuda.set_device(local)
@@ -260,24 +314,8 @@ def run_ours(args):
     if world > 1:
         import torch.distributed as dist
         dist.init_process_group("nccl", device_id=dev)
-
-    def barrier():
-        if dist is not None:
-            dist.barrier()
-
-    def max_over_ranks(x):
-        if dist is None:
-            return x
-        t = torch.tensor([x], dtype=torch.float64, device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        return float(t.item())
-
-    def sum_over_ranks(x):
-        if dist is None:
-            return x
-        t = torch.tensor([x], dtype=torch.float64, device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.SUM)
-        return float(t.item())
+    group = RankGroup(dist, dev)
+    barrier, max_over_ranks, sum_over_ranks = group.barrier, group.max, group.sum
 
     rs.build()
     rs.load_library()
@@ -289,7 +327,7 @@ def run_ours(args):
     es = w.elem_bytes
     set_bytes = 2 * B * (N + 1) * V * es
     pool = args.pool or max(2, min(8, math.ceil(4 * L2_BYTES / max(1, 2 * B * V * es))))
-    sets = [W.make_inputs_torch(w, seed=args.seed + 7919 * rank + 31 * i, device=dev, batch=B)
+    sets = [W.make_inputs_torch(w, seed=replica_seed(args.seed, rank, i), device=dev, batch=B)
             for i in range(pool)]
     parents_np = w.parents
     haschild = np.zeros(N + 1, dtype=bool)
@@ -332,8 +370,7 @@ def run_ours(args):
     wall = time.perf_counter() - wall0
     clk = clocks.stop()
     launch_ms = [ev[i].elapsed_time(ev[i + 1]) for i in range(K)]
-    elapsed_ms = ev[0].elapsed_time(ev[K])
-    elapsed_ms = max_over_ranks(elapsed_ms)
+    value, elapsed_ms = whole_job_rate(group, float(K * B * N), ev[0].elapsed_time(ev[K]))
     if int(status.item()) & ~rs.INFO_DEGENERATE:
         raise SystemExit(f"kernel reported data errors: status {int(status.item())}")
 
@@ -347,8 +384,6 @@ def run_ours(args):
         alg_bytes += int(rows.sum()) * V * es
         emitted += int((alen + 1).sum())
         accepted += int(alen.sum())
-    total_nodes = sum_over_ranks(float(K * B * N))
-    value = total_nodes / (elapsed_ms / 1e3)
     mean_launch_s = (sum(launch_ms) / K) / 1e3
     achieved_gbs = (alg_bytes / K) / mean_launch_s / 1e9
     peak, peak_kind = measured_peak()
@@ -371,7 +406,7 @@ def run_ours(args):
         },
         "roofline": {"bound": "hbm", "achieved": achieved_gbs, "peak": peak, "unit": "GB/s",
                      "frac": achieved_gbs / peak,
-                     "traffic": profiled_traffic(plan["kernel_name"], w.name),
+                     "traffic": profiled_traffic(plan["kernel_name"], w.name, alg_bytes / K),
                      "peak_kind": peak_kind, "frac_of_8tbs": achieved_gbs / NOMINAL_HBM_GBS,
                      "alg_bytes_per_launch": alg_bytes / K,
                      "mean_launch_us": mean_launch_s * 1e6},

@@ -38,6 +38,7 @@ namespace rs {
 
 constexpr int kMaxMaps = 128;          // residual maps per node (rejections with a map)
 constexpr int kMaxKids = kMaxMaps;      // children per node the streaming kernel walks
+static_assert(kMaxKids < 256, "per-visit draws use the last threads of a CTA");
 constexpr int kErrFanout = 64;
 
 // Residual maps are kept in unnormalised units.  With p~ = 2^(z_t c - M_t)
@@ -696,17 +697,22 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
     // row r: word 0 is the accept draw of node r - 1, word 1 the final draw
     // at row r), and one more thread draws the visit's final uniform
     float mt = kNoRef, st = 0.f, md = kNoRef, sd = 0.f;
+    // (the loaded logits stay in registers until the pass ends, so no warp
+    // waits for them; the draws are computed by the last threads)
+    const int nk0 = S2.nkids;
+    float kz_t = 0.f, kz_d = 0.f;
     stream_pass_pre<THREADS, BF16>(ring, src,
         [&] {
-          const int nk = S2.nkids;
-          if (tid < nk) {
-            const int cn = S2.knode[tid];
-            const int x = cand_s[cn];
+          if (tid < nk0) {
+            const int x = cand_s[S2.knode[tid]];
             const bool okx = x >= 0 && x < V;
-            S2.kzt[tid] = okx ? raw_logit(P.zt, rbase + (size_t)x, bf16) : 0.f;
-            S2.kzd[tid] = okx ? raw_logit(P.zd, rbase + (size_t)x, bf16) : 0.f;
-            S2.kua[tid] = uniform_draw(P.seed, (uint32_t)b, (uint32_t)(cn + 1), 0);
-          } else if (tid == max(nk, 0)) {
+            kz_t = okx ? raw_logit(P.zt, rbase + (size_t)x, bf16) : 0.f;
+            kz_d = okx ? raw_logit(P.zd, rbase + (size_t)x, bf16) : 0.f;
+          }
+          const int j = THREADS - 1 - tid;  // kMaxKids < THREADS
+          if (j < nk0) {
+            S2.kua[j] = uniform_draw(P.seed, (uint32_t)b, (uint32_t)(S2.knode[j] + 1), 0);
+          } else if (j == max(nk0, 0)) {
             S2.ufin = uniform_draw(P.seed, (uint32_t)b, (uint32_t)row, 1);
           }
         },
@@ -724,6 +730,10 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
           }
           return false;
         });
+    if (tid < nk0) {
+      S2.kzt[tid] = kz_t;
+      S2.kzd[tid] = kz_d;
+    }
     if (mt == kNoRef) mt = -INFINITY;  // no finite logit: the exchange's "no mass" marker
     if (md == kNoRef) md = -INFINITY;
     const bool bad_t = !(st <= FLT_MAX), bad_d = !(sd <= FLT_MAX);

@@ -1,0 +1,81 @@
+"""Multi-rank host logic of bench.py on CPU: one process per rank (gloo,
+world size 2), as the replicas run launches one per GPU.  The path has no
+data exchange between ranks; only the timing barrier and the reductions
+that form the whole-job number cross ranks."""
+import json
+import os
+import socket
+import subprocess
+import sys
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+sys.path.insert(0, ROOT)
+
+import bench  # noqa: E402
+
+
+def _free_port():
+    with socket.socket() as s:
+        s.bind(("127.0.0.1", 0))
+        return s.getsockname()[1]
+
+
+def _worker(rank, world, port, out_dir):
+    import torch
+    import torch.distributed as dist
+    os.environ["MASTER_ADDR"] = "127.0.0.1"
+    os.environ["MASTER_PORT"] = str(port)
+    dist.init_process_group("gloo", rank=rank, world_size=world)
+    g = bench.RankGroup(dist, torch.device("cpu"))
+    g.barrier()
+    # rank r processed 100 (r + 1) units in 10 (r + 1) ms
+    value, slowest = bench.whole_job_rate(g, 100.0 * (rank + 1), 10.0 * (rank + 1))
+    res = {"max": g.max(float(rank) + 0.5), "sum": g.sum(float(rank) + 1.0), "value": value,
+           "slowest": slowest, "seeds": [bench.replica_seed(1234, rank, i) for i in range(3)]}
+    g.barrier()
+    dist.destroy_process_group()
+    with open(os.path.join(out_dir, f"rank{rank}.json"), "w") as f:
+        json.dump(res, f)
+
+
+def test_rank_group_single_process():
+    g = bench.RankGroup()
+    g.barrier()
+    assert g.max(3.0) == 3.0 and g.sum(2.5) == 2.5
+    value, slowest = bench.whole_job_rate(g, 500.0, 250.0)
+    assert slowest == 250.0 and value == pytest.approx(2000.0)
+
+
+def test_rank_group_gloo_world2(tmp_path):
+    torch = pytest.importorskip("torch")
+    import torch.multiprocessing as mp
+    mp.start_processes(_worker, args=(2, _free_port(), str(tmp_path)), nprocs=2,
+                       start_method="spawn")
+    r = [json.load(open(tmp_path / f"rank{i}.json")) for i in range(2)]
+    for x in r:
+        assert x["max"] == 1.5 and x["sum"] == 3.0
+        # 300 units over the slowest rank's 20 ms
+        assert x["slowest"] == 20.0 and x["value"] == pytest.approx(300.0 / 0.020)
+    # every replica verifies its own inputs
+    assert not set(r[0]["seeds"]) & set(r[1]["seeds"])
+
+
+def test_reference_arm_under_torchrun_world2(tmp_path):
+    """`bench.py --impl reference` launched the way the driver launches N > 1
+    runs: rank 0 alone times the oracle and prints one line; rank 1 exits 0."""
+    pytest.importorskip("torch")
+    import oracle
+    oracle.build()
+    cmd = [sys.executable, "-m", "torch.distributed.run", "--nnodes=1", "--nproc-per-node", "2",
+           "--master-addr", "127.0.0.1", "--master-port", str(_free_port()),
+           os.path.join(ROOT, "bench.py"), "--impl", "reference", "--gpus", "2", "--steps", "2",
+           "--warmup", "1", "--cpu-seqs", "4", "--workload", "tiny-chain-v64"]
+    p = subprocess.run(cmd, cwd=ROOT, capture_output=True, text=True, timeout=300)
+    assert p.returncode == 0, p.stderr[-2000:]
+    lines = [l for l in p.stdout.splitlines() if l.startswith("{")]
+    assert len(lines) == 1, p.stdout
+    d = json.loads(lines[0])
+    assert d["impl"] == "reference" and d["n_gpus"] == 2 and d["value"] > 0
+    assert d["e2e"]["h2d_bytes_per_step"] == 0 and d["cpu_baseline"]["kind"] == "oracle"

@@ -38,7 +38,7 @@ namespace rs {
 
 constexpr int kMaxMaps = 128;          // residual maps per node (rejections with a map)
 constexpr int kMaxKids = kMaxMaps;      // children per node the streaming kernel walks
-static_assert(kMaxKids < 256, "per-visit draws use the last threads of a CTA");
+static_assert(2 * kMaxKids <= 256, "per-visit loads and draws use distinct threads of a CTA");
 constexpr int kErrFanout = 64;
 
 // Residual maps are kept in unnormalised units.  With p~ = 2^(z_t c - M_t)
@@ -57,10 +57,8 @@ struct __align__(16) StreamHead {
   int rejk[kMaxMaps];    // their child index in this visit
   float kzt[kMaxKids];   // raw target / draft logits of the children's tokens
   float kzd[kMaxKids];
-  int16_t knode[kMaxKids];  // the children, ascending
   float kua[kMaxKids];   // their accept draws U(seed, b, child + 1, 0)
   float ufin;            // the visit's final draw U(seed, b, row, 1)
-  int nkids;
   int nmaps;
 };
 constexpr int kStreamHeadBytes = 4096;
@@ -679,17 +677,11 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
     src.nloc = nloc;
     src.vec = P.use_tma != 0;
 
-    // children of the node, ascending
-    if (tid == 0) {
-      int n = 0;
-      for (int cn = c1; cn >= 0; cn = next_sib[cn]) {
-        if (n == kMaxKids) { n = -1; break; }
-        S2.knode[n++] = (int16_t)cn;
-      }
-      S2.nkids = n;
-      S2.nmaps = 0;
-    }
-    __syncthreads();
+    // Per-visit state in S2 is written by every thread with identical
+    // values (each thread reads back its own writes), so no barrier is
+    // needed to publish it; the barrier at the end of the previous visit
+    // orders these writes after every read of the old values.
+    S2.nmaps = 0;
 
     // ---- tempered normaliser (S2): online (reference, sum) per row; while
     // the first chunks are in flight, one thread per child reads its token's
@@ -697,22 +689,33 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
     // row r: word 0 is the accept draw of node r - 1, word 1 the final draw
     // at row r), and one more thread draws the visit's final uniform
     float mt = kNoRef, st = 0.f, md = kNoRef, sd = 0.f;
-    // (the loaded logits stay in registers until the pass ends, so no warp
-    // waits for them; the draws are computed by the last threads)
-    const int nk0 = S2.nkids;
+    // (child t is found by walking t siblings; the loaded logits stay in
+    // registers until the pass ends, so no warp waits for them; the draws
+    // are computed by the last threads)
+    auto nth_child = [&](int t) {
+      int cn = c1;
+      for (int k = 0; k < t && cn >= 0; ++k) cn = next_sib[cn];
+      return cn;
+    };
+    bool have_kid = false;
     float kz_t = 0.f, kz_d = 0.f;
     stream_pass_pre<THREADS, BF16>(ring, src,
         [&] {
-          if (tid < nk0) {
-            const int x = cand_s[S2.knode[tid]];
-            const bool okx = x >= 0 && x < V;
-            kz_t = okx ? raw_logit(P.zt, rbase + (size_t)x, bf16) : 0.f;
-            kz_d = okx ? raw_logit(P.zd, rbase + (size_t)x, bf16) : 0.f;
+          if (tid < kMaxKids && need_draft) {
+            const int cn = nth_child(tid);
+            if (cn >= 0) {
+              const int x = cand_s[cn];
+              const bool okx = x >= 0 && x < V;
+              have_kid = true;
+              kz_t = okx ? raw_logit(P.zt, rbase + (size_t)x, bf16) : 0.f;
+              kz_d = okx ? raw_logit(P.zd, rbase + (size_t)x, bf16) : 0.f;
+            }
           }
-          const int j = THREADS - 1 - tid;  // kMaxKids < THREADS
-          if (j < nk0) {
-            S2.kua[j] = uniform_draw(P.seed, (uint32_t)b, (uint32_t)(S2.knode[j] + 1), 0);
-          } else if (j == max(nk0, 0)) {
+          const int j = THREADS - 1 - tid;  // kMaxKids < THREADS - kMaxKids
+          if (j < kMaxKids && need_draft) {
+            const int cn = nth_child(j);
+            if (cn >= 0) S2.kua[j] = uniform_draw(P.seed, (uint32_t)b, (uint32_t)(cn + 1), 0);
+          } else if (j == kMaxKids) {
             S2.ufin = uniform_draw(P.seed, (uint32_t)b, (uint32_t)row, 1);
           }
         },
@@ -730,7 +733,7 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
           }
           return false;
         });
-    if (tid < nk0) {
+    if (have_kid) {
       S2.kzt[tid] = kz_t;
       S2.kzd[tid] = kz_d;
     }
@@ -765,13 +768,10 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
       if (to) err |= kErrTimeout;
       break;
     }
-    const int nk = S2.nkids;  // written by thread 0 before the exchange's barriers
-    if (nk < 0) { err |= kErrFanout; break; }
-
     // ---- sequential accept tests over the children (S3), shaping on reject
     int accepted = -1, acc_tok = -1;
-    for (int i = 0; i < nk; ++i) {
-      const int cn = S2.knode[i];
+    for (int i = 0, cn = c1; cn >= 0; ++i, cn = next_sib[cn]) {
+      if (i == kMaxKids) { err |= kErrFanout; break; }
       const int x = cand_s[cn];
       if (x < 0 || x >= V) { err |= kErrToken; break; }
       const int nm = S2.nmaps;
@@ -881,14 +881,11 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
         // per-CTA masses of the new residual: (p0 + lambda p1) sig (ResiSpec)
         // or p0 sig (SpecInfer) from this exchange's unnormalised partials
         Pm = Pending{resi ? kResi : kSpec, x, K.sig, Z, lam};
-        if (tid == 0) {
-          S2.mk[nm] = kq;
-          S2.mlam[nm] = lam;
-          S2.rej[nm] = x;
-          S2.rejk[nm] = i;
-          S2.nmaps = nm + 1;
-        }
-        __syncthreads();
+        S2.mk[nm] = kq;  // every thread, identical values (see the visit start)
+        S2.mlam[nm] = lam;
+        S2.rej[nm] = x;
+        S2.rejk[nm] = i;
+        S2.nmaps = nm + 1;
       } else {
         info |= kInfoDegenerate;
         mass_kind = 0;  // the exchange's partials do not describe R: sum it directly
@@ -913,7 +910,7 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
     node = accepted;
     row = accepted + 1;
     depth += 1;
-    __syncthreads();  // thread 0 rewrites the children list of the next visit
+    __syncthreads();  // every read of this visit's S2 state precedes the next visit's writes
   }
 
   if (rank == 0 && tid == 0) {

@@ -133,4 +133,21 @@ __device__ __forceinline__ float ex2(float x) {
   return y;
 }
 
+// Largest of three floats in one instruction (sm_100 family); a NaN input is
+// ignored like fmaxf.
+__device__ __forceinline__ float fmax3(float a, float b, float c) {
+  float d;
+  asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
+  return d;
+}
+
+// Pairs of fp32 values for the packed (two lanes per instruction) fp32
+// add / multiply / fused multiply-add of the sm_100 family; each lane is
+// rounded exactly like the scalar operation.
+__device__ __forceinline__ float2 dup2(float a) { return make_float2(a, a); }
+__device__ __forceinline__ float2 ex2x2(float2 a) { return make_float2(ex2(a.x), ex2(a.y)); }
+__device__ __forceinline__ float2 relu2(float2 a) {
+  return make_float2(fmaxf(a.x, 0.f), fmaxf(a.y, 0.f));
+}
+
 }  // namespace rs

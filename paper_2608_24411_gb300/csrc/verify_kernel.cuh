@@ -585,10 +585,25 @@ __device__ __forceinline__ void reject_pass_any(float* W, const float* Q, int L,
 // The inverse-CDF search runs on exact 64-bit fixed-point masses
 // (probability * 2^44, rounded): integer sums are associative, so every
 // level of the hierarchical search agrees with every other.
-constexpr float kFix = 17592186044416.f;  // 2^44
 
+// round(x 2^44) (nearest, ties to even) of a mass x >= 0, with integer
+// operations only: the float-to-64-bit-integer conversion runs on the FP64
+// pipe, which issues 2 lanes per clock per SM on this part, and the sampler
+// converts every element of a slice.  x = m 2^(e - 150) with the 24-bit
+// significand m, so x 2^44 = m 2^(e - 106): a left shift when e >= 106,
+// else m / 2^s (s = 106 - e) rounded by adding 2^(s-1) - 1 plus the parity
+// of the quotient before the shift.  Negative x gives 0 and x >= 2^20
+// saturates (neither occurs for masses).
 __device__ __forceinline__ unsigned long long to_fix(float x) {
-  return __float2ull_rn(__fmul_rn(x, kFix));
+  const uint32_t b = __float_as_uint(x);
+  if ((int32_t)b <= 0) return 0ull;
+  const int e = (int)(b >> 23);
+  const uint32_t m = e ? ((b & 0x7fffffu) | 0x800000u) : b;
+  const int sh = (e ? e : 1) - 106;
+  if (sh >= 0) return sh >= 40 ? ~0ull : (unsigned long long)m << sh;
+  const int s = -sh;
+  if (s > 24) return 0ull;
+  return (unsigned long long)((m + (1u << (s - 1)) - 1u + ((m >> s) & 1u)) >> s);
 }
 
 __device__ __forceinline__ unsigned long long warp_sum_u64(unsigned long long v) {

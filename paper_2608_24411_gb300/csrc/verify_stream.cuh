@@ -49,10 +49,13 @@ constexpr int kErrFanout = 64;
 //   SpecInfer: R~' = (R~ - k_i q~)_+,
 // with k_i = Z_i / (S_d sigma_{i-1}) (ResiSpec) or 1 / (S_d sigma_{i-1})
 // (SpecInfer) and sigma_i = sigma_{i-1} a_i: every scale is folded into the
-// per-map scalar k_i and the running factor sigma.
+// per-map scalar k_i and the running factor sigma.  The ResiSpec form keeps
+// m (its minimum taken directly) and R~ - m separate: folding the map into
+// R~ - (1 - lambda_i)(R~ - m) would round 1 - lambda_i, an error that the
+// renormalisation by a small Z_i magnifies wherever m + lambda_i (R~ - m)
+// is much smaller than R~.  Maps are applied two lanes per instruction.
 struct __align__(16) StreamHead {
-  float mk[kMaxMaps];    // k_i of map i
-  float mlam[kMaxMaps];  // ResiSpec filled fraction lambda_i of map i
+  float2 map[kMaxMaps];  // {k_i, lambda_i} of map i (SpecInfer: {-k_i, 0})
   int rej[kMaxMaps];     // tokens whose residual is 0 (ResiSpec maps)
   int rejk[kMaxMaps];    // their child index in this visit
   float kzt[kMaxKids];   // raw target / draft logits of the children's tokens
@@ -123,6 +126,25 @@ __device__ __forceinline__ void unpack_vec(const uint4& w, float (&z)[BF16 ? 8 :
 // -inf (written by the copy step).
 __device__ __forceinline__ uint4 stage_vec(const unsigned char* row, int h, int threads) {
   return reinterpret_cast<const uint4*>(row)[h * threads + (int)threadIdx.x];
+}
+
+// This thread's NE values of a ring stage row as NE / 2 pairs, in the order
+// of its vectors (pair j holds elements 2j, 2j + 1 of the thread's chunk).
+template <int THREADS, bool BF16>
+__device__ __forceinline__ void load_pairs(const unsigned char* row, float2 (&z)[4]) {
+  if constexpr (BF16) {
+    const uint4 w = stage_vec(row, 0, THREADS);
+    const uint32_t v[4] = {w.x, w.y, w.z, w.w};
+#pragma unroll
+    for (int i = 0; i < 4; ++i) z[i] = make_float2(bf16_lo(v[i]), bf16_hi(v[i]));
+  } else {
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+      const float4 f = *reinterpret_cast<const float4*>(&reinterpret_cast<const uint4*>(row)[h * THREADS + (int)threadIdx.x]);
+      z[2 * h] = make_float2(f.x, f.y);
+      z[2 * h + 1] = make_float2(f.z, f.w);
+    }
+  }
 }
 
 // Copies this thread's vectors of chunk k into ring stage `st` (the copies
@@ -240,58 +262,47 @@ __device__ __forceinline__ float raw_logit(const void* base, size_t i, bool bf16
 // still makes the sum non-finite (detected by the caller).
 constexpr float kNoRef = -FLT_MAX;
 
-template <int N>
-__device__ __forceinline__ float tree_max(const float (&z)[N]) {
-  float v[N];
-#pragma unroll
-  for (int j = 0; j < N; ++j) v[j] = z[j];
-#pragma unroll
-  for (int w = N / 2; w > 0; w /= 2)
-#pragma unroll
-    for (int j = 0; j < w; ++j) v[j] = fmaxf(v[j], v[j + w]);
-  return v[0];
+__device__ __forceinline__ float max8(const float2 (&z)[4]) {
+  return fmax3(fmax3(z[0].x, z[0].y, z[1].x), fmax3(z[1].y, z[2].x, z[2].y),
+               fmaxf(z[3].x, z[3].y));
 }
 
-template <int N>
-__device__ __forceinline__ float tree_sum(float (&v)[N]) {
-#pragma unroll
-  for (int w = N / 2; w > 0; w /= 2)
-#pragma unroll
-    for (int j = 0; j < w; ++j) v[j] = __fadd_rn(v[j], v[j + w]);
-  return v[0];
-}
-
-__device__ __forceinline__ void rebase(float vmax, float c, float& m, float& s) {
+__device__ __forceinline__ void rebase2(float vmax, float c, float& m, float2& s) {
   const float mnew = __fmul_rn(vmax, c);
-  s = __fmul_rn(s, ex2(__fsub_rn(m, mnew)));  // 0 from the sentinel
+  s = __fmul2_rn(s, dup2(ex2(__fsub_rn(m, mnew))));  // 0 from the sentinel
   m = mnew;
 }
 
-template <int N, bool TWO>
-__device__ __forceinline__ void norm_accumulate(const float (&zt)[N], const float (&zd)[N],
-                                                float c, float& mt, float& st, float& md,
-                                                float& sd) {
-  const float vt = tree_max<N>(zt);
+// Sum of 2^(z c - m) over 8 values (4 pairs), as a pair of partial sums.
+__device__ __forceinline__ float2 exp_sum8(const float2 (&z)[4], float2 c2, float2 nm2) {
+  float2 e[4];
+#pragma unroll
+  for (int j = 0; j < 4; ++j) e[j] = ex2x2(__ffma2_rn(z[j], c2, nm2));
+  return __fadd2_rn(__fadd2_rn(e[0], e[1]), __fadd2_rn(e[2], e[3]));
+}
+
+// One chunk of a thread's values (8 per row) into its online (reference,
+// sum) pairs; the sums are kept as pairs of lanes.
+template <bool TWO>
+__device__ __forceinline__ void norm_accumulate(const float2 (&zt)[4], const float2 (&zd)[4],
+                                                float c, float& mt, float2& st, float& md,
+                                                float2& sd) {
+  const float vt = max8(zt);
   const bool rt = __fmaf_rn(vt, c, -mt) > 0.f;
   float vd = 0.f;
   bool rd = false;
   if constexpr (TWO) {
-    vd = tree_max<N>(zd);
+    vd = max8(zd);
     rd = __fmaf_rn(vd, c, -md) > 0.f;
   }
   if (rt || rd) {  // rare: a new reference for one of the rows
-    if (rt) rebase(vt, c, mt, st);
+    if (rt) rebase2(vt, c, mt, st);
     if constexpr (TWO)
-      if (rd) rebase(vd, c, md, sd);
+      if (rd) rebase2(vd, c, md, sd);
   }
-  float et[N], ed[N];
-#pragma unroll
-  for (int j = 0; j < N; ++j) {
-    et[j] = ex2(__fmaf_rn(zt[j], c, -mt));
-    if constexpr (TWO) ed[j] = ex2(__fmaf_rn(zd[j], c, -md));
-  }
-  st = __fadd_rn(st, tree_sum<N>(et));
-  if constexpr (TWO) sd = __fadd_rn(sd, tree_sum<N>(ed));
+  const float2 c2 = dup2(c);
+  st = __fadd2_rn(st, exp_sum8(zt, c2, dup2(-mt)));
+  if constexpr (TWO) sd = __fadd2_rn(sd, exp_sum8(zd, c2, dup2(-md)));
 }
 
 // Cluster-wide scalars of a visit after the normaliser.
@@ -302,11 +313,6 @@ struct VisitScalars {
   float sig;         // sigma of the current residual (R = sig R~; 1 / S_t before any map)
 };
 
-// p and q of one element from its raw logits.
-__device__ __forceinline__ float prob_of(float z, float c, float M, float inv) {
-  return __fmul_rn(ex2(__fmaf_rn(z, c, -M)), inv);
-}
-
 // 2^(z c - M): p~ or q~ of one element from its raw logit.
 __device__ __forceinline__ float exp_of(float z, float c, float M) {
   return ex2(__fmaf_rn(z, c, -M));
@@ -316,34 +322,44 @@ __device__ __forceinline__ float exp_of(float z, float c, float M) {
 // rejected-token zeroing: the caller applies it).  ResiSpec map: GetProxy
 // residual r = min(Z q, R) + lambda (R - min(Z q, R)), R' = r / sum r;
 // SpecInfer map: R' = (R - q)_+ / sum (Eq. recur); in the units above.
+// The ResiSpec map's two parts from R~ and q~: m = min(k q~, R~) and the
+// capacity R~ - m.
+__device__ __forceinline__ float2 min_part2(float2 k, float2 q, float2 R) {
+  const float2 kq = __fmul2_rn(k, q);
+  return make_float2(fminf(kq.x, R.x), fminf(kq.y, R.y));
+}
+
 template <bool RESI>
 __device__ __forceinline__ float apply_chain(const StreamHead& S2, int nm, float R, float q) {
   for (int i = 0; i < nm; ++i) {
+    const float2 mp = S2.map[i];
     if constexpr (RESI) {
-      const float m = fminf(__fmul_rn(S2.mk[i], q), R);
-      R = __fmaf_rn(S2.mlam[i], __fsub_rn(R, m), m);
+      const float m = fminf(__fmul_rn(mp.x, q), R);
+      R = __fmaf_rn(mp.y, __fmaf_rn(m, -1.f, R), m);
     } else {
-      R = fmaxf(__fmaf_rn(-S2.mk[i], q, R), 0.f);
+      R = fmaxf(__fmaf_rn(mp.x, q, R), 0.f);
     }
   }
   return R;
 }
 
-template <int N, bool RESI>
-__device__ __forceinline__ void apply_chain_vec(const StreamHead& S2, int nm, float (&R)[N],
-                                                const float (&q)[N]) {
+// The same on pairs: every lane rounds exactly like apply_chain.
+template <int NP, bool RESI>
+__device__ __forceinline__ void apply_chain_pairs(const StreamHead& S2, int nm, float2 (&R)[NP],
+                                                  const float2 (&q)[NP]) {
   for (int i = 0; i < nm; ++i) {
-    const float k = S2.mk[i];
+    const float2 mp = S2.map[i];
+    const float2 k = dup2(mp.x);
     if constexpr (RESI) {
-      const float lam = S2.mlam[i];
+      const float2 lam = dup2(mp.y);
 #pragma unroll
-      for (int j = 0; j < N; ++j) {
-        const float m = fminf(__fmul_rn(k, q[j]), R[j]);
-        R[j] = __fmaf_rn(lam, __fsub_rn(R[j], m), m);
+      for (int j = 0; j < NP; ++j) {
+        const float2 m = min_part2(k, q[j], R[j]);
+        R[j] = __ffma2_rn(lam, __ffma2_rn(m, dup2(-1.f), R[j]), m);
       }
     } else {
 #pragma unroll
-      for (int j = 0; j < N; ++j) R[j] = fmaxf(__fmaf_rn(-k, q[j], R[j]), 0.f);
+      for (int j = 0; j < NP; ++j) R[j] = relu2(__ffma2_rn(k, q[j], R[j]));
     }
   }
 }
@@ -370,27 +386,37 @@ __device__ __forceinline__ void final_values(const StreamHead& S2, const VisitSc
                                              const unsigned char* rt, const unsigned char* rd,
                                              int h, float (&v)[BF16 ? 8 : 4]) {
   constexpr int VEC = BF16 ? 8 : 4;
-  unpack_vec<BF16>(stage_vec(rt, h, THREADS), v);
+  constexpr int NP = VEC / 2;
+  float z[VEC];
+  unpack_vec<BF16>(stage_vec(rt, h, THREADS), z);
+  const float2 c2 = dup2(K.c);
+  float2 R[NP];
+#pragma unroll
+  for (int j = 0; j < NP; ++j)
+    R[j] = ex2x2(__ffma2_rn(make_float2(z[2 * j], z[2 * j + 1]), c2, dup2(-K.Mt)));
   if (nm == 0) {
 #pragma unroll
-    for (int j = 0; j < VEC; ++j) v[j] = prob_of(v[j], K.c, K.Mt, K.invSt);
+    for (int j = 0; j < NP; ++j) {
+      const float2 r = __fmul2_rn(R[j], dup2(K.invSt));
+      v[2 * j] = r.x;
+      v[2 * j + 1] = r.y;
+    }
     return;
   }
-  float q[VEC];
-  unpack_vec<BF16>(stage_vec(rd, h, THREADS), q);
+  unpack_vec<BF16>(stage_vec(rd, h, THREADS), z);
+  float2 q[NP];
 #pragma unroll
-  for (int j = 0; j < VEC; ++j) {
-    v[j] = exp_of(v[j], K.c, K.Mt);
-    q[j] = exp_of(q[j], K.c, K.Md);
-  }
-  if (resi) {
-    apply_chain_vec<VEC, true>(S2, nm, v, q);
-    zero_rejected_vec<VEC>(S2, nm, base, v);
-  } else {
-    apply_chain_vec<VEC, false>(S2, nm, v, q);
-  }
+  for (int j = 0; j < NP; ++j)
+    q[j] = ex2x2(__ffma2_rn(make_float2(z[2 * j], z[2 * j + 1]), c2, dup2(-K.Md)));
+  if (resi) apply_chain_pairs<NP, true>(S2, nm, R, q);
+  else apply_chain_pairs<NP, false>(S2, nm, R, q);
 #pragma unroll
-  for (int j = 0; j < VEC; ++j) v[j] = __fmul_rn(v[j], K.sig);
+  for (int j = 0; j < NP; ++j) {
+    const float2 r = __fmul2_rn(R[j], dup2(K.sig));
+    v[2 * j] = r.x;
+    v[2 * j + 1] = r.y;
+  }
+  if (resi) zero_rejected_vec<VEC>(S2, nm, base, v);
 }
 
 // ---------------------------------------------------------------- sampler
@@ -639,36 +665,43 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
   const bool resi = P.mode == 0;
   const bool bf16 = BF16;
 
-  if (tid < 4) H.pubv[tid] = 0.f;
-  if (tid == 0) {
-    mbar_init(smem_addr(&H.xbar[0]), 1);
-    mbar_init(smem_addr(&H.xbar[1]), 1);
-    fence_mbar_init();
-  }
-  for (int i = tid; i < P.npad + 16; i += THREADS) first_child[i] = -1;
-  int bad = 0;
-  for (int i = tid; i < N; i += THREADS) {
-    const int p = __ldg(P.parents + i);
-    const bool ok = p >= -1 && p < i;
-    bad |= !ok;
-    par[i] = (int16_t)(ok ? p : -2);
-    cand_s[i] = __ldg(P.cand + (size_t)b * N + i);
-  }
-  const bool tree_bad = __syncthreads_or(bad) != 0;
-  build_children(par, first_child, next_sib, N);
-  __syncthreads();
-  cluster_sync();  // every peer has started: its receive slots may now be written
-
-  int err = tree_bad ? kErrTree : 0;
+  int err = 0;
   int info = 0;
   int depth = 0, rejects = 0;
   int node = -1, row = 0;
   uint32_t xph = 0;
   int xp = 0;
 
-  while (!err) {
-    const int c1 = first_child[node + 1];
-    const bool need_draft = c1 >= 0;
+  // Kernel setup: exchange barriers, the tree's child lists and the
+  // candidates.  It runs while the first chunks of the root's rows are in
+  // flight (the root has children exactly when N > 0 in a valid tree, since
+  // node 0's parent can only be the root).
+  auto setup = [&] {
+    if (tid < 4) H.pubv[tid] = 0.f;
+    if (tid == 0) {
+      mbar_init(smem_addr(&H.xbar[0]), 1);
+      mbar_init(smem_addr(&H.xbar[1]), 1);
+      fence_mbar_init();
+    }
+    for (int i = tid; i < P.npad + 16; i += THREADS) first_child[i] = -1;
+    int bad = 0;
+    for (int i = tid; i < N; i += THREADS) {
+      const int p = __ldg(P.parents + i);
+      const bool ok = p >= -1 && p < i;
+      bad |= !ok;
+      par[i] = (int16_t)(ok ? p : -2);
+      cand_s[i] = __ldg(P.cand + (size_t)b * N + i);
+    }
+    const bool tree_bad = __syncthreads_or(bad) != 0;
+    build_children(par, first_child, next_sib, N);
+    __syncthreads();
+    cluster_sync();  // every peer has started: its receive slots may now be written
+    if (tree_bad) err = kErrTree;
+  };
+
+  for (bool first = true; !err; first = false) {
+    int c1 = first ? -1 : first_child[node + 1];
+    const bool need_draft = first ? N > 0 : c1 >= 0;
     const size_t rbase = (size_t)b * P.seq_stride + (size_t)row * V;
     Src src;
     src.t = static_cast<const char*>(P.zt) + (rbase + (size_t)lo) * es;
@@ -688,7 +721,8 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
     // raw logits and draws its accept uniform (one Philox block per logit
     // row r: word 0 is the accept draw of node r - 1, word 1 the final draw
     // at row r), and one more thread draws the visit's final uniform
-    float mt = kNoRef, st = 0.f, md = kNoRef, sd = 0.f;
+    float mt = kNoRef, md = kNoRef;
+    float2 st2 = make_float2(0.f, 0.f), sd2 = make_float2(0.f, 0.f);
     // (child t is found by walking t siblings; the loaded logits stay in
     // registers until the pass ends, so no warp waits for them; the draws
     // are computed by the last threads)
@@ -701,7 +735,11 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
     float kz_t = 0.f, kz_d = 0.f;
     stream_pass_pre<THREADS, BF16>(ring, src,
         [&] {
-          if (tid < kMaxKids && need_draft) {
+          if (first) {
+            setup();
+            c1 = first_child[0];
+          }
+          if (tid < kMaxKids && need_draft && !err) {
             const int cn = nth_child(tid);
             if (cn >= 0) {
               const int x = cand_s[cn];
@@ -712,7 +750,7 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
             }
           }
           const int j = THREADS - 1 - tid;  // kMaxKids < THREADS - kMaxKids
-          if (j < kMaxKids && need_draft) {
+          if (j < kMaxKids && need_draft && !err) {
             const int cn = nth_child(j);
             if (cn >= 0) S2.kua[j] = uniform_draw(P.seed, (uint32_t)b, (uint32_t)(cn + 1), 0);
           } else if (j == kMaxKids) {
@@ -720,19 +758,19 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
           }
         },
         [&](const unsigned char* rt, const unsigned char* rd, int) -> bool {
-#pragma unroll
-          for (int h = 0; h < G::VPT; ++h) {
-            float zt[VEC], zd[VEC];
-            unpack_vec<BF16>(stage_vec(rt, h, THREADS), zt);
-            if (need_draft) {
-              unpack_vec<BF16>(stage_vec(rd, h, THREADS), zd);
-              norm_accumulate<VEC, true>(zt, zd, P.scale_log2, mt, st, md, sd);
-            } else {
-              norm_accumulate<VEC, false>(zt, zd, P.scale_log2, mt, st, md, sd);
-            }
+          if (err) return true;  // invalid tree (uniform over the cluster)
+          float2 zt[4], zd[4];
+          load_pairs<THREADS, BF16>(rt, zt);
+          if (need_draft) {
+            load_pairs<THREADS, BF16>(rd, zd);
+            norm_accumulate<true>(zt, zd, P.scale_log2, mt, st2, md, sd2);
+          } else {
+            norm_accumulate<false>(zt, zd, P.scale_log2, mt, st2, md, sd2);
           }
           return false;
         });
+    if (err) break;
+    const float st = __fadd_rn(st2.x, st2.y), sd = __fadd_rn(sd2.x, sd2.y);
     if (have_kid) {
       S2.kzt[tid] = kz_t;
       S2.kzd[tid] = kz_d;
@@ -802,38 +840,43 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
       // unnormalised units (k: the new map's scalar).  The rejected tokens
       // get no special case here; their terms are taken out below.
       const float kq = __fdiv_rn(resi ? __fmul_rn(Z, K.invSd) : K.invSd, K.sig);
-      float s1 = 0.f, s2 = 0.f;
-      stream_pass<THREADS, BF16>(ring, src, [&](const unsigned char* rt, const unsigned char* rd,
-                                                int) -> bool {
+      // s1: sum of min(k q~, R~) (ResiSpec) or of the capacity t (SpecInfer);
+      // s2: sum of t (ResiSpec); both as pairs of lanes
+      float2 s1p = make_float2(0.f, 0.f), s2p = make_float2(0.f, 0.f);
+      {
+        const float2 c2 = dup2(K.c), nMt = dup2(-K.Mt), nMd = dup2(-K.Md), kq2 = dup2(kq),
+                     nkq = dup2(-kq);
+        stream_pass<THREADS, BF16>(ring, src, [&](const unsigned char* rt, const unsigned char* rd,
+                                                  int) -> bool {
+          float2 Rv[4], q[4];
+          load_pairs<THREADS, BF16>(rt, Rv);  // -inf past the slice: 0
+          load_pairs<THREADS, BF16>(rd, q);
 #pragma unroll
-        for (int h = 0; h < G::VPT; ++h) {
-          float Rv[VEC], q[VEC];
-          unpack_vec<BF16>(stage_vec(rt, h, THREADS), Rv);  // -inf past the slice: 0
-          unpack_vec<BF16>(stage_vec(rd, h, THREADS), q);
-#pragma unroll
-          for (int j = 0; j < VEC; ++j) {
-            Rv[j] = exp_of(Rv[j], K.c, K.Mt);
-            q[j] = exp_of(q[j], K.c, K.Md);
+          for (int j = 0; j < 4; ++j) {
+            Rv[j] = ex2x2(__ffma2_rn(Rv[j], c2, nMt));
+            q[j] = ex2x2(__ffma2_rn(q[j], c2, nMd));
           }
-          float a1[VEC], a2[VEC];
+          float2 t[4];
           if (resi) {
-            apply_chain_vec<VEC, true>(S2, nm, Rv, q);
+            apply_chain_pairs<4, true>(S2, nm, Rv, q);
+            float2 m[4];
 #pragma unroll
-            for (int j = 0; j < VEC; ++j) {
-              a1[j] = fminf(__fmul_rn(kq, q[j]), Rv[j]);
-              a2[j] = __fsub_rn(Rv[j], a1[j]);
+            for (int j = 0; j < 4; ++j) {
+              m[j] = min_part2(kq2, q[j], Rv[j]);
+              t[j] = __ffma2_rn(m[j], dup2(-1.f), Rv[j]);
             }
-            s1 = __fadd_rn(s1, tree_sum<VEC>(a1));
-            s2 = __fadd_rn(s2, tree_sum<VEC>(a2));
+            s1p = __fadd2_rn(s1p, __fadd2_rn(__fadd2_rn(m[0], m[1]), __fadd2_rn(m[2], m[3])));
+            s2p = __fadd2_rn(s2p, __fadd2_rn(__fadd2_rn(t[0], t[1]), __fadd2_rn(t[2], t[3])));
           } else {
-            apply_chain_vec<VEC, false>(S2, nm, Rv, q);
+            apply_chain_pairs<4, false>(S2, nm, Rv, q);
 #pragma unroll
-            for (int j = 0; j < VEC; ++j) a1[j] = fmaxf(__fmaf_rn(-kq, q[j], Rv[j]), 0.f);
-            s1 = __fadd_rn(s1, tree_sum<VEC>(a1));
+            for (int j = 0; j < 4; ++j) t[j] = relu2(__ffma2_rn(nkq, q[j], Rv[j]));
+            s1p = __fadd2_rn(s1p, __fadd2_rn(__fadd2_rn(t[0], t[1]), __fadd2_rn(t[2], t[3])));
           }
-        }
-        return false;
-      });
+          return false;
+        });
+      }
+      float s1 = __fadd_rn(s1p.x, s1p.y), s2 = __fadd_rn(s2p.x, s2p.y);
       if (resi) {
         // The token just rejected (r(x0) = 0) and the earlier rejected ones
         // (R = 0 there) add nothing: the thread that summed each such token
@@ -851,7 +894,7 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
           const float Ry = apply_chain<true>(S2, nm, exp_of(S2.kzt[yk], K.c, K.Mt), qy);
           const float my = fminf(__fmul_rn(kq, qy), Ry);
           s1 = __fsub_rn(s1, my);
-          s2 = __fsub_rn(s2, __fsub_rn(Ry, my));
+          s2 = __fsub_rn(s2, __fmaf_rn(my, -1.f, Ry));
         }
       }
       exchange<NW, false>(H, s1, s2, 0.f, 0.f, 0, -1, xp, xph, rank, C, o, oflags);
@@ -881,8 +924,8 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
         // per-CTA masses of the new residual: (p0 + lambda p1) sig (ResiSpec)
         // or p0 sig (SpecInfer) from this exchange's unnormalised partials
         Pm = Pending{resi ? kResi : kSpec, x, K.sig, Z, lam};
-        S2.mk[nm] = kq;  // every thread, identical values (see the visit start)
-        S2.mlam[nm] = lam;
+        // every thread, identical values (see the visit start)
+        S2.map[nm] = resi ? make_float2(kq, lam) : make_float2(-kq, 0.f);
         S2.rej[nm] = x;
         S2.rejk[nm] = i;
         S2.nmaps = nm + 1;

@@ -214,11 +214,14 @@ int plan_resident(const resispec_dims& d, int cs, int dev, int sms, Plan* p) {
 
 // Streaming kernel: cluster size.  A sequence's passes shrink as 1 / C,
 // and the batch runs in ceil(B / n) waves of n resident clusters; the
-// largest C whose waves stay within a small bound wins (per-sequence chains
-// differ in length, so the longest chain, run at C CTAs, sets the time).
-// Without a device, 2 CTAs of 512 threads per SM on 152 SMs are assumed and
-// a cluster of 16 is taken to fit 14 times (how many clusters of 16 CTAs
-// GB300 places at once), smaller ones in proportion.
+// largest C whose waves stay within a bound wins (per-sequence chains differ
+// in length, so the longest chain, run at C CTAs, sets the time).  The bound
+// (measured on GB300 over four tree shapes): 2 waves for clusters of 16; for
+// trees deeper than 2 levels (long accept/reject chains) a single wave,
+// since a second wave of long chains costs more than halving C; for shallow
+// trees up to 4 waves.  Without a device, 2 CTAs of 512 threads per SM on
+// 152 SMs are assumed and a cluster of 16 is taken to fit 14 times (how many
+// clusters of 16 CTAs GB300 places at once), smaller ones in proportion.
 int plan_stream(const resispec_dims& d, int cs, int dev, int sms, Plan* p) {
   const bool bf16 = d.dtype == RESISPEC_BF16;
   p->smem = stream_smem_for(p->threads, bf16, p->npad);
@@ -237,7 +240,8 @@ int plan_stream(const resispec_dims& d, int cs, int dev, int sms, Plan* p) {
       const int n = active_for(C);
       if (n <= 0) continue;
       const int waves = (B + n - 1) / n;
-      if (waves <= (C == 16 ? 2 : 4) || C == 1) {
+      const int bound = C == 16 ? 2 : (d.max_depth <= 2 ? 4 : 1);
+      if (waves <= bound || C == 1) {
         best = C;
         break;
       }

@@ -75,11 +75,16 @@ def test_synchronous_argument_errors(lib):
 
 def test_plan_without_device(lib):
     # the bench workload (B = 64, V = 151936 fp32) cannot sit on chip at once:
-    # the automatic choice streams it, in clusters of 8 CTAs (two waves)
+    # the automatic choice streams it, in clusters of 4 CTAs (one wave: the
+    # tree is 5 levels deep)
     p = rs.plan(64, 62, 151936, 5, "f32")
-    assert p["kernel_name"] == "stream" and p["cluster_size"] == 8
+    assert p["kernel_name"] == "stream" and p["cluster_size"] == 4
     assert p["smem_bytes"] <= 228 * 1024 // 2 - 1024   # two CTAs per SM
-    assert p["slice_elems"] % 8 == 0 and p["slice_elems"] * 8 >= 151936
+    assert p["slice_elems"] % 8 == 0 and p["slice_elems"] * 4 >= 151936
+    # shallow trees accept more waves: 128 single-position sequences in
+    # clusters of 8; deep trees of 32 sequences in clusters of 8 (one wave)
+    assert rs.plan(128, 16, 256000, 1, "bf16", kernel="stream")["cluster_size"] == 8
+    assert rs.plan(32, 488, 256000, 6, "bf16", kernel="stream")["cluster_size"] == 8
     assert p["uses_tma"] == 1
     for B in (1, 7, 64, 128, 1000):
         p = rs.plan(B, 488, 256000, 6, "bf16", kernel="stream")

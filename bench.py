@@ -158,20 +158,34 @@ class ClockSampler:
 # ------------------------------------------------------------------ helpers
 
 
+def has_children(parents_np):
+    """[N + 1] (one tree) or [B, N + 1] (a tree per sequence): whether the
+    root (index 0) / node j (index j + 1) has children."""
+    p = np.asarray(parents_np)
+    if p.ndim == 1:
+        h = np.zeros(p.size + 1, dtype=bool)
+        h[p[p >= -1] + 1] = True
+        return h
+    h = np.zeros((p.shape[0], p.shape[1] + 1), dtype=bool)
+    for b in range(p.shape[0]):
+        h[b, p[b] + 1] = True
+    return h
+
+
 def rows_visited(nodes, accept_len, haschild):
     """Logit rows each sequence read: 2 per visited node with children
     (target + draft), 1 for a visited node without children (bonus: target
     only).  Visited nodes are the root and every accepted node."""
     a = accept_len.astype(np.int64)
     D = nodes.shape[1]
-    root = 2 if haschild[0] else 1
-    rows = np.full(a.shape, root, dtype=np.int64)
+    hc = haschild if haschild.ndim == 2 else np.broadcast_to(haschild, (a.size, haschild.size))
+    rows = np.where(hc[:, 0], 2, 1).astype(np.int64)
     for d in range(D):
         mask = a > d
         if not mask.any():
             break
         nd = nodes[mask, d]
-        rows[mask] += np.where(haschild[nd + 1], 2, 1)
+        rows[mask] += np.where(hc[mask, nd + 1], 2, 1)
     return rows
 
 
@@ -329,10 +343,7 @@ def run_ours(args):
     pool = args.pool or max(2, min(8, math.ceil(4 * L2_BYTES / max(1, 2 * B * V * es))))
     sets = [W.make_inputs_torch(w, seed=replica_seed(args.seed, rank, i), device=dev, batch=B)
             for i in range(pool)]
-    parents_np = w.parents
-    haschild = np.zeros(N + 1, dtype=bool)
-    for c, p in enumerate(parents_np):
-        haschild[p + 1] = True
+    haschild = [has_children(s["parents_np"]) for s in sets]
     K, Wm = args.steps, args.warmup
     outs = [(torch.empty((B, D + 1), dtype=torch.int32, device=dev),
              torch.empty((B,), dtype=torch.int32, device=dev),
@@ -380,7 +391,7 @@ def run_ours(args):
     for i in range(K):
         alen = outs[i][1].cpu().numpy()
         nodes = outs[i][2].cpu().numpy()[:, :D]
-        rows = rows_visited(nodes, alen, haschild)
+        rows = rows_visited(nodes, alen, haschild[(Wm + i) % pool])
         alg_bytes += int(rows.sum()) * V * es
         emitted += int((alen + 1).sum())
         accepted += int(alen.sum())
@@ -485,7 +496,8 @@ def _finish_cpu(result, args, sets, w, mode, world, dev):
     dh = _host_logits(s0["draft"].index_select(0, idx))
     ch = s0["cand"].index_select(0, idx).cpu().numpy()
     omode = oracle.MODE_SPECINFER if mode == 1 else oracle.MODE_RESISPEC
-    rate, threads, sample = cpu_oracle_rate(w, th, dh, w.parents, ch,
+    pa = s0["parents_np"][:S] if w.per_sequence_tree else s0["parents_np"]
+    rate, threads, sample = cpu_oracle_rate(w, th, dh, pa, ch,
                                             np.arange(S, dtype=np.int32), omode,
                                             args.cpu_seconds, args.seed)
     result["cpu_baseline"] = {"value": rate, "unit": "nodes/s", "cores": threads,

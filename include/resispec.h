@@ -40,7 +40,7 @@
 extern "C" {
 #endif
 
-#define RESISPEC_ABI_VERSION 2
+#define RESISPEC_ABI_VERSION 3
 
 /* Synchronous return codes. */
 typedef enum {
@@ -68,8 +68,9 @@ typedef enum { RESISPEC_MODE_RESISPEC = 0, RESISPEC_MODE_SPECINFER = 1 } resispe
 #define RESISPEC_ERR_EMPTY_ROW 8   /* a visited row (or the residual) has no mass */
 #define RESISPEC_ERR_DEPTH 16      /* more accepted tokens than max_depth */
 #define RESISPEC_ERR_TIMEOUT 32    /* a bounded wait for a row copy gave up */
-#define RESISPEC_ERR_FANOUT 64     /* streaming kernel: a visited node has more than
-                                      RESISPEC_MAX_FANOUT_STREAM children */
+#define RESISPEC_ERR_FANOUT 64     /* streaming kernel: the walk reached child
+                                      RESISPEC_MAX_FANOUT_STREAM + 1 of a node (it
+                                      tests at most that many children per node) */
 #define RESISPEC_INFO_DEGENERATE 256 /* informational: a rejection left R unchanged */
 
 #define RESISPEC_MAX_VOCAB 262144
@@ -119,6 +120,11 @@ typedef struct {
                             last emitted token was drawn from (final residual
                             R, or p of the accepted leaf) */
   int32_t* out_rejects;  /* optional device [B] number of rejections */
+  int64_t parents_stride; /* int32 elements between sequences' trees in
+                             tree_parents: 0 (default) = one tree [N] shared by
+                             every sequence; N = tree_parents is [B, N], a tree
+                             per sequence (dynamic trees; a bad tree marks only
+                             its own sequence with RESISPEC_ERR_TREE) */
 } resispec_opts;
 
 /* Fills *opts with the defaults (RESISPEC mode, automatic launch shape,
@@ -130,7 +136,8 @@ void resispec_opts_default(resispec_opts* opts);
  *                  bulk-copy path (otherwise plain loads are used)
  *   draft_logits   [B, N+1, V] same layout
  *   tree_parents   [N] int32, parent of node c (-1 = root), parent < c;
- *                  siblings are tested in ascending node index
+ *                  siblings are tested in ascending node index (with
+ *                  opts->parents_stride = N: [B, N], one tree per sequence)
  *   cand_tokens    [B, N] int32, token proposed at node c (drawn i.i.d. from
  *                  the parent's tempered draft distribution by the caller)
  *   temperature    T > 0, applied to target and draft logits alike
@@ -139,7 +146,7 @@ void resispec_opts_default(resispec_opts* opts);
  *                  token, then -1 padding
  *   out_accept_len [B] int32: number of accepted candidates (-1 on a
  *                  per-sequence data error)
- * Uses RESISPEC mode and automatic launch shape. */
+ * Uses RESISPEC mode, automatic launch shape and one shared tree. */
 int resispec_verify(const void* target_logits, const void* draft_logits,
                     const int32_t* tree_parents, const int32_t* cand_tokens,
                     float temperature, uint64_t seed, int32_t* out_tokens,

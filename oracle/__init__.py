@@ -77,7 +77,7 @@ class _Args(ctypes.Structure):
         ("out_accept_margin", ctypes.c_void_p), ("out_sample_margin", ctypes.c_void_p),
         ("out_status", ctypes.c_void_p), ("out_rejects", ctypes.c_void_p),
         ("out_rows", ctypes.c_void_p), ("out_inv_err", ctypes.c_void_p),
-        ("out_cond", ctypes.c_void_p),
+        ("out_cond", ctypes.c_void_p), ("parents_stride", ctypes.c_int64),
     ]
 
 
@@ -187,7 +187,8 @@ def verify(target, draft, parents, cand, temperature, seed, *, mode=MODE_RESISPE
     ``target``/``draft``: float32 arrays, or uint16 arrays holding bf16 bit
     patterns, shaped [B, N+1, V] (or [N+1, V] with ``seq_stride=0`` to share
     one set of rows across all B sequences, in which case ``cand`` gives B).
-    ``parents``: int32 [N]; ``cand``: int32 [B, N].
+    ``parents``: int32 [N] (one tree for every sequence) or [B, N] (a tree
+    per sequence); ``cand``: int32 [B, N].
     Returns a dict of numpy arrays.
     """
     lib = load()
@@ -203,15 +204,19 @@ def verify(target, draft, parents, cand, temperature, seed, *, mode=MODE_RESISPE
     draft = np.ascontiguousarray(draft)
     parents = np.ascontiguousarray(parents, dtype=np.int32)
     cand = np.ascontiguousarray(cand, dtype=np.int32)
-    N = parents.size
+    per_seq = parents.ndim == 2
+    N = parents.shape[-1] if per_seq else parents.size
     B = cand.shape[0] if cand.ndim == 2 else (target.shape[0] if target.ndim == 3 else 1)
     if cand.ndim != 2:
         cand = cand.reshape(B, N)
     V = target.shape[-1]
     if seq_stride is None:
         seq_stride = (N + 1) * V
+    if per_seq and parents.shape[0] != B:
+        raise ValueError("per-sequence parents must be [B, N]")
     if max_depth is None:
-        max_depth = tree_depth(parents)
+        max_depth = max((tree_depth(t) for t in parents), default=0) if per_seq \
+            else tree_depth(parents)
     D = int(max_depth)
     if seq_ids is not None:
         seq_ids = np.ascontiguousarray(seq_ids, dtype=np.int32)
@@ -238,6 +243,7 @@ def verify(target, draft, parents, cand, temperature, seed, *, mode=MODE_RESISPE
     a.seq_stride = int(seq_stride)
     a.target, a.draft = target.ctypes.data, draft.ctypes.data
     a.parents, a.cand = parents.ctypes.data, cand.ctypes.data
+    a.parents_stride = N if per_seq else 0
     a.seq_ids = _ptr(seq_ids)
     a.temperature = float(np.float32(temperature))
     a.seed = int(seed) & 0xFFFFFFFFFFFFFFFF

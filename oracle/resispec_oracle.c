@@ -306,7 +306,7 @@ typedef struct {
   int64_t seq_stride; /* elements between sequences; 0 = shared rows */
   const void* target;
   const void* draft;
-  const int32_t* parents;  /* [N] */
+  const int32_t* parents;  /* [N], or [B, N] with parents_stride = N */
   const int32_t* cand;     /* [B, N] */
   const int32_t* seq_ids;  /* [B] global sequence index for the RNG, or NULL */
   double temperature;
@@ -324,6 +324,9 @@ typedef struct {
   double* out_inv_err;     /* [B] largest invariant violation */
   double* out_cond;        /* [B] 1 / prod of the SpecInfer normalisers at the
                               final node (1 without SpecInfer rejections) */
+  int64_t parents_stride;  /* elements between sequences' parent arrays:
+                              0 = one tree for all, N = parents is [B, N]
+                              (per-sequence, dynamic trees) */
 } oracle_args;
 
 typedef struct {
@@ -332,10 +335,19 @@ typedef struct {
   int tree_bad;
 } worker_ctx;
 
+/* A tree is valid when every node's parent precedes it (-1: the root). */
+static int tree_is_bad(const int32_t* parents, int N) {
+  for (int c = 0; c < N; ++c)
+    if (parents[c] < -1 || parents[c] >= c) return 1;
+  return 0;
+}
+
 static void verify_sequence(const oracle_args* a, int lb, int tree_bad,
                             double* z, double* p, double* q, double* R,
                             double* K, double* r, double* tmp, int32_t* kids) {
   const int V = a->V, N = a->N, D = a->D;
+  const int32_t* parents = a->parents + (size_t)(a->parents_stride * lb);
+  if (a->parents_stride) tree_bad = tree_is_bad(parents, N);
   const int64_t gb = a->seq_ids ? a->seq_ids[lb] : lb;
   const double T = a->temperature;
   int32_t* toks = a->out_tokens ? a->out_tokens + (size_t)lb * (D + 1) : NULL;
@@ -357,7 +369,7 @@ static void verify_sequence(const oracle_args* a, int lb, int tree_bad,
   for (;;) {
     int nk = 0;
     for (int c = 0; c < N; ++c)
-      if (a->parents[c] == node) kids[nk++] = c;
+      if (parents[c] == node) kids[nk++] = c;
 
     load_row(a->target, a->dtype, seq_off + (size_t)row * V, V, z);
     rows += 1;
@@ -470,9 +482,8 @@ static void* worker(void* arg) {
 int oracle_verify(const oracle_args* a) {
   if (a->B < 0 || a->N < 0 || a->V < 1 || a->D < 0 || !(a->temperature > 0.0))
     return -1;
-  int tree_bad = 0;
-  for (int c = 0; c < a->N; ++c)
-    if (a->parents[c] < -1 || a->parents[c] >= c) tree_bad = 1;
+  if (a->parents_stride < 0) return -1;
+  const int tree_bad = a->parents_stride ? 0 : tree_is_bad(a->parents, a->N);
   int nt = a->nthreads > 0 ? a->nthreads : 1;
   if (nt > a->B) nt = a->B > 0 ? a->B : 1;
   worker_ctx* ctx = (worker_ctx*)calloc((size_t)nt, sizeof(worker_ctx));

@@ -68,7 +68,7 @@ class Opts(ctypes.Structure):
                 ("block_threads", ctypes.c_int32), ("flags", ctypes.c_int32),
                 ("seq_stride", ctypes.c_int64), ("status", ctypes.c_void_p),
                 ("out_nodes", ctypes.c_void_p), ("out_dist", ctypes.c_void_p),
-                ("out_rejects", ctypes.c_void_p)]
+                ("out_rejects", ctypes.c_void_p), ("parents_stride", ctypes.c_int64)]
 
 
 class PlanInfo(ctypes.Structure):
@@ -207,8 +207,8 @@ def verify(target, draft, tree_parents, cand_tokens, temperature, seed, *, max_d
 
     target, draft: CUDA tensors [B, N+1, V] (float32 or bfloat16); with
     ``seq_stride=0`` they may be [N+1, V] and are shared by all B sequences.
-    tree_parents: int32 CUDA tensor [N]; cand_tokens: int32 CUDA tensor
-    [B, N].  Returns (out_tokens [B, D+1], out_accept_len [B]).  Runs on
+    tree_parents: int32 CUDA tensor [N] (one tree for every sequence) or
+    [B, N] (a tree per sequence); cand_tokens: int32 CUDA tensor [B, N].  Returns (out_tokens [B, D+1], out_accept_len [B]).  Runs on
     ``stream`` (default: torch's current stream) without synchronising.
     ``kernel``: None / "auto" (the library's choice), "resident" or "stream".
     """
@@ -224,8 +224,11 @@ def verify(target, draft, tree_parents, cand_tokens, temperature, seed, *, max_d
     dt = _dtype_code(target)
     if tree_parents.dtype != torch.int32 or cand_tokens.dtype != torch.int32:
         raise TypeError("tree_parents and cand_tokens must be int32")
-    N = int(tree_parents.numel())
+    per_seq_tree = tree_parents.dim() == 2
+    N = int(tree_parents.shape[-1]) if per_seq_tree else int(tree_parents.numel())
     B = int(cand_tokens.shape[0]) if cand_tokens.dim() == 2 else int(target.shape[0])
+    if per_seq_tree and int(tree_parents.shape[0]) != B:
+        raise ValueError("per-sequence tree_parents must be [B, N]")
     V = int(target.shape[-1])
     if max_depth is None:
         if out_tokens is None:
@@ -243,6 +246,7 @@ def verify(target, draft, tree_parents, cand_tokens, temperature, seed, *, max_d
         raise ValueError("target must be [B, N+1, V] (or pass seq_stride)")
     o = make_opts(mode, cluster_size, block_threads, no_tma, seq_stride, status, out_nodes,
                   out_dist, out_rejects, prefetch, kernel)
+    o.parents_stride = N if per_seq_tree else 0
     if stream is None:
         stream = torch.cuda.current_stream(dev)
     handle = stream.cuda_stream if hasattr(stream, "cuda_stream") else int(stream)

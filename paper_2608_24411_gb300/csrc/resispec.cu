@@ -267,6 +267,7 @@ int make_plan(const resispec_dims& d, const resispec_opts& o, int dev, int sms,
   const int cs = o.cluster_size;
   if (cs < 0 || cs > rs::kMaxCluster) return RESISPEC_E_ARG;
   if (o.seq_stride < -1) return RESISPEC_E_ARG;
+  if (o.parents_stride < 0) return RESISPEC_E_ARG;
   const bool force_res = (o.flags & RESISPEC_FLAG_RESIDENT) != 0;
   const bool force_str = (o.flags & RESISPEC_FLAG_STREAM) != 0;
   if (force_res && force_str) return RESISPEC_E_ARG;
@@ -437,6 +438,7 @@ int resispec_verify_ex(const void* target_logits, const void* draft_logits,
   prm.out_rejects = o.out_rejects;
   prm.status = o.status;
   prm.seq_stride = o.seq_stride < 0 ? (int64_t)(dims.num_nodes + 1) * dims.vocab : o.seq_stride;
+  prm.parents_stride = o.parents_stride;
   prm.seed = seed;
   prm.scale_log2 = (float)(1.4426950408889634 / (double)temperature);
   prm.B = dims.batch;

@@ -62,7 +62,7 @@ constexpr float kRebaseLog2 = 64.f;        // exponent headroom before a referen
 struct VerifyParams {
   const void* zt;
   const void* zd;
-  const int32_t* parents;
+  const int32_t* parents;  // [N], or [B, N] with parents_stride = N
   const int32_t* cand;
   int32_t* out_tokens;
   int32_t* out_len;
@@ -71,6 +71,7 @@ struct VerifyParams {
   int32_t* out_rejects;
   int32_t* status;
   int64_t seq_stride;  // elements
+  int64_t parents_stride;  // elements between sequences' trees (0: one tree)
   uint64_t seed;
   float scale_log2;    // log2(e) / T
   int32_t B, N, V, D;
@@ -818,7 +819,7 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 3)
   for (int i = tid; i < P.npad + 16; i += THREADS) first_child[i] = -1;
   int bad = 0;
   for (int i = tid; i < N; i += THREADS) {
-    const int p = __ldg(P.parents + i);
+    const int p = __ldg(P.parents + (size_t)b * P.parents_stride + i);
     const bool ok = p >= -1 && p < i;
     bad |= !ok;
     par[i] = (int16_t)(ok ? p : -2);

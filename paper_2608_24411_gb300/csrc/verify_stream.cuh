@@ -686,7 +686,7 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
     for (int i = tid; i < P.npad + 16; i += THREADS) first_child[i] = -1;
     int bad = 0;
     for (int i = tid; i < N; i += THREADS) {
-      const int p = __ldg(P.parents + i);
+      const int p = __ldg(P.parents + (size_t)b * P.parents_stride + i);
       const bool ok = p >= -1 && p < i;
       bad |= !ok;
       par[i] = (int16_t)(ok ? p : -2);

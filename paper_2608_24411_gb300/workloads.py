@@ -18,7 +18,11 @@ its datasets, Sec. 6.1):
 Tree shapes (the paper's dXbY trees and batch-sampling chains, Sec. 3):
 ``levels`` (every node of level l has b[l] children, BFS numbering),
 ``chain`` (k siblings per level, level l+1 hangs below sibling 0 of level l)
-and ``single`` (k siblings of the root).
+and ``single`` (k siblings of the root), one tree for every sequence; and
+``random`` (a tree of N nodes per sequence, as dynamic-tree drafters build
+them: node c hangs below a node drawn among the root and the earlier nodes
+less than Dmax deep, with weight 2^-depth, so the top levels are bushy and
+the deep ones thin; nodes are numbered in creation order).
 """
 from __future__ import annotations
 
@@ -65,6 +69,25 @@ def tree_depth(parents) -> int:
     return int(depth.max()) if parents.size else 0
 
 
+def tree_random(rng: np.random.Generator, B: int, N: int, dmax: int) -> np.ndarray:
+    """[B, N] int32 parents: one random tree of N nodes (depth <= dmax) per
+    sequence."""
+    out = np.zeros((int(B), int(N)), dtype=np.int32)
+    for b in range(int(B)):
+        depth = [0]          # the root, then node c at index c + 1
+        for c in range(int(N)):
+            cand = [i for i, d in enumerate(depth) if d < dmax]
+            w = np.asarray([0.5 ** depth[i] for i in cand])
+            pick = cand[int(rng.choice(len(cand), p=w / w.sum()))]
+            out[b, c] = pick - 1
+            depth.append(depth[pick] + 1)
+    return out
+
+
+def per_sequence_tree(spec) -> bool:
+    return spec[0] == "random"
+
+
 def make_tree(spec) -> np.ndarray:
     kind = spec[0]
     if kind == "levels":
@@ -96,16 +119,23 @@ class Workload:
     extra: dict = field(default_factory=dict)
 
     @property
+    def per_sequence_tree(self) -> bool:
+        return per_sequence_tree(self.tree)
+
+    @property
     def parents(self) -> np.ndarray:
+        """The shared tree ([N]); per-sequence trees come with the inputs."""
+        if self.per_sequence_tree:
+            raise ValueError(f"{self.name}: a tree per sequence, drawn with the inputs")
         return make_tree(self.tree)
 
     @property
     def num_nodes(self) -> int:
-        return int(self.parents.size)
+        return int(self.tree[1]) if self.per_sequence_tree else int(self.parents.size)
 
     @property
     def max_depth(self) -> int:
-        return tree_depth(self.parents)
+        return int(self.tree[2]) if self.per_sequence_tree else tree_depth(self.parents)
 
     @property
     def elem_bytes(self) -> int:
@@ -132,6 +162,14 @@ WORKLOADS = {
         scale=4.0, slope=1.0, rho=0.8, temperature=1.0, tree=("levels", (2, 2, 2, 2, 2)),
         steps=500, note="rho swept over {0.5, 0.8, 0.95}; 0.8 is the default"),
 }
+WORKLOADS["dyntree60-v32000"] = _w(
+    name="dyntree60-v32000", batch=64, vocab=32000, dtype="bf16", gen="zipf", scale=3.0,
+    slope=1.1, rho=0.9, temperature=1.0, tree=("random", 60, 6), steps=200,
+    note="a random 60-node tree of depth <= 6 per sequence (dynamic trees)")
+WORKLOADS["dyntree60-v128256-b64"] = _w(
+    name="dyntree60-v128256-b64", batch=64, vocab=128256, dtype="bf16", gen="zipf",
+    scale=3.0, slope=1.1, rho=0.8, temperature=1.0, tree=("random", 60, 6), steps=200,
+    note="a random 60-node tree of depth <= 6 per sequence (dynamic trees)")
 for _b in (32, 128):
     for _k in (2, 4, 8, 16):
         WORKLOADS[f"single-k{_k}-v256000-b{_b}"] = _w(
@@ -193,14 +231,18 @@ def gumbel_argmax_np(rng: np.random.Generator, z_rows: np.ndarray, T: float) -> 
 def candidates_np(rng, draft_f32: np.ndarray, parents: np.ndarray, T: float) -> np.ndarray:
     """cand[b, c] drawn from the tempered draft row of c's parent.
 
-    ``draft_f32``: [B, N+1, V] float32 (row 0 = root, row j+1 = node j).
+    ``draft_f32``: [B, N+1, V] float32 (row 0 = root, row j+1 = node j);
+    ``parents``: [N] (shared tree) or [B, N] (a tree per sequence).
     """
     B = draft_f32.shape[0]
-    N = parents.size
+    N = parents.shape[-1]
     if N == 0:
         return np.zeros((B, 0), dtype=np.int32)
     parent_rows = parents.astype(np.int64) + 1
-    z = draft_f32[:, parent_rows, :]                     # [B, N, V]
+    if parents.ndim == 2:
+        z = np.take_along_axis(draft_f32, parent_rows[:, :, None], axis=1)  # [B, N, V]
+    else:
+        z = draft_f32[:, parent_rows, :]                 # [B, N, V]
     return gumbel_argmax_np(rng, z, T).reshape(B, N)
 
 
@@ -209,8 +251,11 @@ def make_inputs_np(w: Workload, seed: int, batch: int | None = None, rho: float 
     or uint16 bf16 bits), parents, cand, temperature, max_depth."""
     rng = np.random.default_rng(seed)
     B = w.batch if batch is None else int(batch)
-    parents = w.parents
-    N = parents.size
+    if w.per_sequence_tree:
+        parents = tree_random(rng, B, w.tree[1], w.tree[2])
+    else:
+        parents = w.parents
+    N = parents.shape[-1]
     zt, zd = logits_np(rng, B * (N + 1), w.vocab, w.gen, w.scale, w.slope,
                        w.rho if rho is None else rho)
     zt = zt.reshape(B, N + 1, w.vocab)
@@ -285,8 +330,11 @@ def make_inputs_torch(w: Workload, seed: int, device, batch: int | None = None,
     g = torch.Generator(device=device)
     g.manual_seed(int(seed))
     B = w.batch if batch is None else int(batch)
-    parents = w.parents
-    N = parents.size
+    if w.per_sequence_tree:
+        parents = tree_random(np.random.default_rng([int(seed), 1]), B, w.tree[1], w.tree[2])
+    else:
+        parents = w.parents
+    N = parents.shape[-1]
     V = w.vocab
     rho = w.rho if rho is None else float(rho)
     tdtype = torch.float32 if w.dtype == "f32" else torch.bfloat16
@@ -312,14 +360,18 @@ def make_inputs_torch(w: Workload, seed: int, device, batch: int | None = None,
     if N:
         prow = torch.as_tensor(parents.astype(np.int64) + 1, device=device)
         node_chunk = max(1, (1 << 28) // max(1, B * V))
+        bidx = torch.arange(B, device=device)[:, None]
         for c0 in range(0, N, node_chunk):
             c1 = min(N, c0 + node_chunk)
-            z = draft[:, prow[c0:c1], :].to(torch.float32) / w.temperature
+            if prow.dim() == 2:
+                z = draft[bidx, prow[:, c0:c1], :].to(torch.float32) / w.temperature
+            else:
+                z = draft[:, prow[c0:c1], :].to(torch.float32) / w.temperature
             u = torch.rand(z.shape, generator=g, device=device).clamp_min_(1e-30)
             z.add_(-torch.log(-torch.log(u)))
             cand[:, c0:c1] = torch.argmax(z, dim=-1).to(torch.int32)
             del z, u
     return dict(target=target, draft=draft,
-                parents=torch.as_tensor(parents, device=device),
+                parents=torch.as_tensor(np.ascontiguousarray(parents), device=device),
                 parents_np=parents, cand=cand, temperature=w.temperature,
                 max_depth=w.max_depth, dtype=w.dtype)

@@ -39,7 +39,7 @@ def test_library_exports_every_declared_symbol(lib):
     for n in declared_functions():
         assert hasattr(lib, n), n
     assert set(rs.EXPORTED) <= set(declared_functions())
-    assert lib.resispec_abi_version() == 2
+    assert lib.resispec_abi_version() == 3
 
 
 def test_opts_default_layout(lib):

@@ -8,6 +8,7 @@ import socket
 import subprocess
 import sys
 
+import numpy as np
 import pytest
 
 ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
@@ -79,3 +80,17 @@ def test_reference_arm_under_torchrun_world2(tmp_path):
     d = json.loads(lines[0])
     assert d["impl"] == "reference" and d["n_gpus"] == 2 and d["value"] > 0
     assert d["e2e"]["h2d_bytes_per_step"] == 0 and d["cpu_baseline"]["kind"] == "oracle"
+
+
+def test_rows_visited_per_sequence_trees():
+    import bench
+    # sequence 0: root -> node 0 (leaf); sequence 1: root -> node 1 -> node 2 (leaf)
+    parents = np.array([[-1, -1, 1], [-1, -1, 1]], np.int32)
+    hc = bench.has_children(parents)
+    assert hc.shape == (2, 4) and hc[0, 0] and hc[0, 2] and not hc[0, 1] and not hc[0, 3]
+    nodes = np.array([[0, -1], [1, 2]], np.int32)
+    alen = np.array([1, 2], np.int32)
+    # root (2 rows) + leaf 0 (1 row); root (2) + node 1 (2) + leaf 2 (1)
+    np.testing.assert_array_equal(bench.rows_visited(nodes, alen, hc), [3, 5])
+    np.testing.assert_array_equal(bench.rows_visited(nodes, alen, bench.has_children(parents[0])),
+                                  [3, 5])

@@ -158,9 +158,12 @@ def test_repeat_runs_bit_identical(kernel):
 
 @pytest.mark.parametrize("mode", MODES)
 def test_wide_fanout(mode):
-    """A star of MAX_FANOUT_STREAM children (the streaming kernel's limit) with weak drafts
-    (long rejection chains) on both kernels; one child more: the streaming
-    kernel reports ERR_FANOUT, the resident kernel verifies."""
+    """A star of MAX_FANOUT_STREAM children (the streaming kernel's limit)
+    whose candidates the target all but excludes (target logit -30 at every
+    candidate: every test rejects, the walk reaches the last child, 128
+    residual maps) on both kernels; one child more: the streaming kernel
+    reports ERR_FANOUT when the walk reaches the 129th child, the resident
+    kernel verifies."""
     import torch
     V = 3000
     for kids in (rs.MAX_FANOUT_STREAM, rs.MAX_FANOUT_STREAM + 1):
@@ -169,15 +172,27 @@ def test_wide_fanout(mode):
         zt = rng.normal(0, 2, (8, kids + 1, V)).astype(np.float32)
         zd = rng.normal(0, 2, (8, kids + 1, V)).astype(np.float32)
         cand = rng.integers(0, V, (8, kids)).astype(np.int32)
+        for b in range(8):
+            zt[b, 0, cand[b]] = -30.0
         inp = {"target": zt, "draft": zd, "parents": parents, "cand": cand, "temperature": 1.0,
                "max_depth": 1}
         _check(inp, mode, seed=kids, kernel="resident")
         if kids <= rs.MAX_FANOUT_STREAM:
             _check(inp, mode, seed=kids, kernel="stream")
         else:
+            # SpecInfer rejects every candidate, so the walk reaches the
+            # 129th child; ResiSpec's shaped residual moves toward q and
+            # accepts a later candidate first (the method's over-acceptance)
             zt_, zd_, pa, ca = _np_inputs_to_gpu(inp)
             g = P.run_gpu(zt_, zd_, pa, ca, 1.0, kids, 1, mode=mode, kernel="stream")
-            assert (g["accept_len"] == -1).all() and g["status"][0] == rs.ERR_FANOUT
+            o = P.run_oracle(zt, zd, parents, cand, 1.0, kids, 1, mode)
+            far = o["rejects"] >= rs.MAX_FANOUT_STREAM
+            assert far.any() == (mode == rs.MODE_SPECINFER)
+            assert (g["accept_len"][far] == -1).all()
+            assert (g["status"][0] & rs.ERR_FANOUT) == (rs.ERR_FANOUT if far.any() else 0)
+            clean = ~far & (o["accept_margin"] > P.ACCEPT_TIE) & (o["sample_margin"] > P.SAMPLE_TIE)
+            assert (g["accept_len"][clean] == o["accept_len"][clean]).all()
+            assert (g["tokens"][clean] == o["tokens"][clean]).all()
 
 
 @pytest.mark.parametrize("kernel", KERNELS)
@@ -301,7 +316,8 @@ def _sampled_parity(w, seed, call_seed, rows, mode=rs.MODE_RESISPEC, batch=None,
     th = P.to_host_logits(inp["target"].index_select(0, ridx))
     dh = P.to_host_logits(inp["draft"].index_select(0, ridx))
     ch = inp["cand"].index_select(0, ridx).cpu().numpy()
-    o = P.run_oracle(th, dh, inp["parents_np"], ch, w.temperature, call_seed, D, mode,
+    pa = inp["parents_np"][rows] if inp["parents_np"].ndim == 2 else inp["parents_np"]
+    o = P.run_oracle(th, dh, pa, ch, w.temperature, call_seed, D, mode,
                      seq_ids=np.asarray(rows, np.int32))
     n, near = P.compare(g, o, rows=rows)
     assert near <= 1, near
@@ -402,3 +418,42 @@ def test_gpu_resispec_million_draws_vs_enumerator(kernel):
     dist, _ = en.single_position(p, q, k, en.MODE_RESISPEC)
     assert chisq_pvalue(counts, dist)[0] > 1e-4
     assert chisq_pvalue(counts, p)[0] < 1e-12
+
+
+@pytest.mark.parametrize("kernel", KERNELS)
+@pytest.mark.parametrize("mode", MODES)
+def test_parity_dynamic_trees(mode, kernel):
+    """A random 60-node tree of depth <= 6 per sequence ([B, N] parents),
+    64 sequences, V = 32000 bf16: every sequence against the oracle."""
+    w = W.WORKLOADS["dyntree60-v32000"]
+    inp = W.make_inputs_np(w, seed=61, batch=64)
+    assert inp["parents"].shape == (64, 60)
+    _check(inp, mode, seed=610 + mode, kernel=kernel)
+
+
+@pytest.mark.parametrize("kernel", KERNELS)
+def test_dynamic_tree_error_marks_only_its_sequence(kernel):
+    w = W.WORKLOADS["dyntree60-v32000"]
+    inp = W.make_inputs_np(w, seed=62, batch=16)
+    inp["parents"] = inp["parents"].copy()
+    inp["parents"][3, 10] = 11                        # a parent after its child
+    zt, zd, pa, ca = _np_inputs_to_gpu(inp)
+    g = P.run_gpu(zt, zd, pa, ca, inp["temperature"], 5, 6, kernel=kernel)
+    o = P.run_oracle(inp["target"], inp["draft"], inp["parents"], inp["cand"],
+                     inp["temperature"], 5, 6, rs.MODE_RESISPEC)
+    assert g["accept_len"][3] == -1 and (g["tokens"][3] == -1).all()
+    assert o["status"][3] == rs.ERR_TREE
+    assert g["status"][0] & rs.ERR_TREE
+    keep = np.arange(16) != 3
+    clean = keep & (o["accept_margin"] > P.ACCEPT_TIE) & (o["sample_margin"] > P.SAMPLE_TIE)
+    assert (g["accept_len"][clean] == o["accept_len"][clean]).all()
+    assert (g["tokens"][clean] == o["tokens"][clean]).all()
+
+
+@pytest.mark.parametrize("kernel", [None, "resident"])
+def test_parity_dynamic_trees_v128256_full_size(kernel):
+    """B = 64, V = 128256 bf16, a random 60-node tree per sequence, in the
+    launch shape the benchmark times (kernel None); 8 sampled sequences."""
+    w = W.WORKLOADS["dyntree60-v128256-b64"]
+    _sampled_parity(w, seed=63, call_seed=1003, rows=[0, 9, 17, 26, 35, 44, 53, 63],
+                    kernel=kernel)

@@ -337,3 +337,43 @@ def test_empty_tree_samples_root():
     for b in range(B):
         p = sp_softmax(zt[b, 0].astype(np.float64))
         assert out["tokens"][b, 0] == _searchsorted_draw(p, _np_uniform(6, b, 0, 1))
+
+
+def test_per_sequence_trees_equal_separate_shared_tree_calls():
+    """A [B, N] parents call (a tree per sequence) equals B calls that each
+    pass that sequence's tree as the shared tree (the path the other pins
+    cover), with the sequence's index for the draws; a bad tree marks only
+    its own sequence."""
+    w = W.WORKLOADS["dyntree60-v32000"]
+    inp = W.make_inputs_np(w, seed=4, batch=12)
+    parents = inp["parents"].copy()
+    parents[5, 7] = 7                                 # node 7 its own parent
+    for mode in (oracle.MODE_RESISPEC, oracle.MODE_SPECINFER):
+        batched = oracle.verify(inp["target"], inp["draft"], parents, inp["cand"], 1.0, 21,
+                                mode=mode, max_depth=6, want_dist=True)
+        for b in range(12):
+            one = oracle.verify(inp["target"][b:b + 1], inp["draft"][b:b + 1], parents[b],
+                                inp["cand"][b:b + 1], 1.0, 21, mode=mode, max_depth=6,
+                                seq_ids=np.array([b], np.int32), want_dist=True)
+            for k in ("tokens", "accept_len", "nodes", "rejects", "status", "dist"):
+                np.testing.assert_array_equal(batched[k][b], one[k][0])
+        assert batched["status"][5] == oracle.ERR_TREE
+        assert (np.delete(batched["status"], 5) & ~oracle.INFO_DEGENERATE == 0).all()
+
+
+def test_random_trees_are_valid_and_candidates_come_from_parent_rows():
+    rng = np.random.default_rng(0)
+    trees = W.tree_random(rng, 40, 60, 6)
+    for t in trees:
+        assert ((t >= -1) & (t < np.arange(60))).all()
+        assert W.tree_depth(t) <= 6
+    # candidates drawn at a tiny temperature are the argmax of the parent's
+    # draft row; every row has a distinct argmax, so each candidate names
+    # its parent's row
+    B, N, V = 40, 60, 400
+    draft = rng.normal(0, 1, (B, N + 1, V)).astype(np.float32)
+    for b in range(B):
+        for r in range(N + 1):
+            draft[b, r, r] = 50.0
+    cand = W.candidates_np(rng, draft, trees, 1e-3)
+    np.testing.assert_array_equal(cand, trees + 1)

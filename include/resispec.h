@@ -90,6 +90,12 @@ typedef struct {
 #define RESISPEC_FLAG_PREFETCH 2 /* resident kernel: warm L2 with the first child's rows */
 #define RESISPEC_FLAG_RESIDENT 4 /* force the resident kernel */
 #define RESISPEC_FLAG_STREAM 8   /* force the streaming kernel */
+#define RESISPEC_FLAG_Z_APPLIED 16 /* RESISPEC mode budget variant (Sec. 5.3 heuristic):
+                                      Z = max(Z*, |q(x0) - R(x0)|), Z* = min over
+                                      q > 0 of R/q (0 once a map of the node has
+                                      zeroed a token), clamped to Z <= 1 - R(x0);
+                                      streaming kernel only (combined with
+                                      RESISPEC_FLAG_RESIDENT: RESISPEC_E_ARG) */
 
 /* Kernels.  Both compute the same verification; they differ in where a
  * visited node's rows live between the passes of a visit.

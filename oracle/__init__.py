@@ -78,6 +78,7 @@ class _Args(ctypes.Structure):
         ("out_status", ctypes.c_void_p), ("out_rejects", ctypes.c_void_p),
         ("out_rows", ctypes.c_void_p), ("out_inv_err", ctypes.c_void_p),
         ("out_cond", ctypes.c_void_p), ("parents_stride", ctypes.c_int64),
+        ("z_rule", ctypes.c_int32), ("pad2_", ctypes.c_int32),
     ]
 
 
@@ -107,6 +108,14 @@ def load():
                                           ctypes.c_void_p, ctypes.c_void_p,
                                           ctypes.c_void_p]
             lib.oracle_reject.restype = ctypes.c_int
+            lib.oracle_reject_z.argtypes = [ctypes.c_int, ctypes.c_int, ctypes.c_void_p,
+                                            ctypes.c_void_p, ctypes.c_int, ctypes.c_int,
+                                            ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p,
+                                            ctypes.c_void_p, ctypes.c_void_p]
+            lib.oracle_reject_z.restype = ctypes.c_int
+            lib.oracle_budget.argtypes = [ctypes.c_void_p, ctypes.c_void_p, ctypes.c_int,
+                                          ctypes.c_int, ctypes.c_int]
+            lib.oracle_budget.restype = ctypes.c_double
             lib.oracle_sample.argtypes = [ctypes.c_void_p, ctypes.c_int,
                                           ctypes.c_double, ctypes.c_void_p]
             lib.oracle_sample.restype = ctypes.c_int
@@ -157,16 +166,23 @@ def get_proxy(p, q, x0: int):
     return k, r, Z
 
 
-def reject(mode: int, R, q, x0: int, check: bool = True):
+def budget(R, q, x0: int, z_rule: int = 0) -> float:
+    """The ResiSpec budget of a rejection of x0: z_rule 0 = Algorithm 1
+    (q(x0) - R(x0)), 1 = Z_applied (max(Z*, |gap|) clamped to 1 - R(x0))."""
+    R, q = _f64(R), _f64(q)
+    return load().oracle_budget(R.ctypes.data, q.ctypes.data, R.size, int(x0), int(z_rule))
+
+
+def reject(mode: int, R, q, x0: int, check: bool = True, z_rule: int = 0):
     """One rejection of x0: returns (R', changed, invariant_error)."""
     R = _f64(R).copy()
     q = _f64(q)
     V = R.size
     K, r, tmp = np.zeros(V), np.zeros(V), np.zeros(V)
     err = np.zeros(1)
-    changed = load().oracle_reject(int(mode), R.ctypes.data, q.ctypes.data, V, int(x0),
-                                   K.ctypes.data, r.ctypes.data, tmp.ctypes.data,
-                                   err.ctypes.data if check else None)
+    changed = load().oracle_reject_z(int(mode), int(z_rule), R.ctypes.data, q.ctypes.data, V,
+                                     int(x0), K.ctypes.data, r.ctypes.data, tmp.ctypes.data,
+                                     err.ctypes.data if check else None, None)
     return R, bool(changed), float(err[0])
 
 
@@ -181,7 +197,7 @@ def sample(R, u: float):
 # ---------------------------------------------------------------- full walk
 def verify(target, draft, parents, cand, temperature, seed, *, mode=MODE_RESISPEC,
            max_depth=None, seq_stride=None, seq_ids=None, nthreads=None,
-           check_invariants=False, decide_fp64=False, want_dist=False):
+           check_invariants=False, decide_fp64=False, want_dist=False, z_rule=0):
     """Run the oracle walk.
 
     ``target``/``draft``: float32 arrays, or uint16 arrays holding bf16 bit
@@ -244,6 +260,7 @@ def verify(target, draft, parents, cand, temperature, seed, *, mode=MODE_RESISPE
     a.target, a.draft = target.ctypes.data, draft.ctypes.data
     a.parents, a.cand = parents.ctypes.data, cand.ctypes.data
     a.parents_stride = N if per_seq else 0
+    a.z_rule = int(z_rule)
     a.seq_ids = _ptr(seq_ids)
     a.temperature = float(np.float32(temperature))
     a.seed = int(seed) & 0xFFFFFFFFFFFFFFFF

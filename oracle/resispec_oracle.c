@@ -45,6 +45,11 @@
  *       siblings (Algorithm 1 never updates D).
  *   R5  degenerate rejection (Z <= 0, or an all-zero residual from rounding):
  *       R is left unchanged and the event is counted.
+ *   R7  budget variant Z_applied (Sec. 5.3 heuristic, flag): Z =
+ *       max(Z*, |q(x0) - R(x0)|) with Z* = min over q > 0 of R/q, the
+ *       capacity bound of Prop. "Capacity Bound of Ideal Shaping" taken on
+ *       the current residual, clamped to Z <= 1 - R(x0) so that the
+ *       water-fill of step 3 stays feasible (r <= R off x0 sums to Z).
  *   R6  the accept decision is taken in fp32, the kernel's precision
  *       (u * q(x) < R(x) with both operands rounded to fp32); the margin
  *       |u - R/q| is reported in fp64 for near-tie accounting.
@@ -162,9 +167,29 @@ int oracle_softmax(const double* z, int V, double T, double* p) {
  *   step 4  k = p - r + s, then k(x0) = q(x0)          (s = 0 off x0, R3)
  * Writes k and r (either may be NULL) and returns Z.  The caller must only
  * use k when Z > 0 (R5). */
+double oracle_get_proxy_z(const double* p, const double* q, int V, int x0, double Z,
+                          double* k, double* r);
+
 double oracle_get_proxy(const double* p, const double* q, int V, int x0,
                         double* k, double* r) {
-  double Z = q[x0] - p[x0];
+  return oracle_get_proxy_z(p, q, V, x0, q[x0] - p[x0], k, r);
+}
+
+/* The budget of a rejection of x0: rule 0 = Algorithm 1 (R1), rule 1 =
+ * Z_applied (R7). */
+double oracle_budget(const double* R, const double* q, int V, int x0, int rule) {
+  const double gap = q[x0] - R[x0];
+  if (rule == 0) return gap;
+  double zstar = INFINITY;
+  for (int i = 0; i < V; ++i)
+    if (q[i] > 0.0 && R[i] / q[i] < zstar) zstar = R[i] / q[i];
+  double Z = fmax(zstar, fabs(gap));
+  return fmin(Z, 1.0 - R[x0]);
+}
+
+/* GetProxy with the budget Z given (steps 2-4 below). */
+double oracle_get_proxy_z(const double* p, const double* q, int V, int x0, double Z,
+                          double* k, double* r) {
   double* rr = r ? r : (double*)malloc(sizeof(double) * (size_t)V);
   double sum_r = 0.0;
   for (int i = 0; i < V; ++i) {
@@ -202,6 +227,8 @@ static double residual_from(double* R, const double* K, int V, double* tmp) {
 int oracle_reject_ex(int mode, double* R, const double* q, int V, int x0,
                      double* K, double* r, double* tmp, double* inv_err,
                      double* norm_out);
+int oracle_reject_z(int mode, int z_rule, double* R, const double* q, int V, int x0,
+                    double* K, double* r, double* tmp, double* inv_err, double* norm_out);
 
 /* One rejection of token x0 applied to the residual R (length V).
  * mode SPECINFER: R <- norm(max(R - q, 0))              (Eq. recur)
@@ -219,6 +246,12 @@ int oracle_reject(int mode, double* R, const double* q, int V, int x0,
 int oracle_reject_ex(int mode, double* R, const double* q, int V, int x0,
                      double* K, double* r, double* tmp, double* inv_err,
                      double* norm_out) {
+  return oracle_reject_z(mode, 0, R, q, V, x0, K, r, tmp, inv_err, norm_out);
+}
+
+/* As oracle_reject_ex with the ResiSpec budget chosen by z_rule (R1 / R7). */
+int oracle_reject_z(int mode, int z_rule, double* R, const double* q, int V, int x0,
+                    double* K, double* r, double* tmp, double* inv_err, double* norm_out) {
   if (norm_out) *norm_out = 1.0;
   if (mode == OR_MODE_SPECINFER) {
     double changed = residual_from(R, q, V, tmp);
@@ -234,8 +267,9 @@ int oracle_reject_ex(int mode, double* R, const double* q, int V, int x0,
     }
     return changed > 0.0;
   }
-  double Z = oracle_get_proxy(R, q, V, x0, K, r);
+  const double Z = oracle_budget(R, q, V, x0, z_rule);
   if (!(Z > 0.0)) return 0;
+  oracle_get_proxy_z(R, q, V, x0, Z, K, r);
   double e = 0.0;
   if (inv_err) {
     double sr = 0.0, sk = 0.0;
@@ -247,9 +281,14 @@ int oracle_reject_ex(int mode, double* R, const double* q, int V, int x0,
       if (-K[i] > e) e = -K[i];
     }
     if (fabs(sr - Z) > e) e = fabs(sr - Z);
-    if (fabs(sk - 1.0) > e) e = fabs(sk - 1.0);
     if (fabs(r[x0]) > e) e = fabs(r[x0]);
-    if (fabs(K[x0] - q[x0]) > e) e = fabs(K[x0] - q[x0]);
+    /* sum K = 1 with K(x0) = q(x0) holds for the budget of Algorithm 1 only;
+       under Z_applied the slack that would restore it is unspecified (it
+       never reaches R' = r / Z), so only r is checked there. */
+    if (z_rule == 0) {
+      if (fabs(sk - 1.0) > e) e = fabs(sk - 1.0);
+      if (fabs(K[x0] - q[x0]) > e) e = fabs(K[x0] - q[x0]);
+    }
   }
   double norm = residual_from(R, K, V, tmp);
   if (!(norm > 0.0)) return 0;
@@ -327,6 +366,8 @@ typedef struct {
   int64_t parents_stride;  /* elements between sequences' parent arrays:
                               0 = one tree for all, N = parents is [B, N]
                               (per-sequence, dynamic trees) */
+  int32_t z_rule;          /* ResiSpec budget: 0 Algorithm 1 (R1), 1 Z_applied (R7) */
+  int32_t pad2_;
 } oracle_args;
 
 typedef struct {
@@ -423,7 +464,7 @@ static void verify_sequence(const oracle_args* a, int lb, int tree_bad,
       }
       rejects += 1;
       double norm = 1.0;
-      if (!oracle_reject_ex(a->mode, R, q, V, x, K, r, tmp, inv_ptr, &norm))
+      if (!oracle_reject_z(a->mode, a->z_rule, R, q, V, x, K, r, tmp, inv_ptr, &norm))
         status |= OR_INFO_DEGENERATE;
       cond /= norm;
     }

@@ -80,10 +80,11 @@ struct VerifyParams {
   int32_t mode;        // 0 ResiSpec, 1 SpecInfer
   int32_t use_tma;
   int32_t prefetch;    // L2 prefetch of the first child's rows
+  int32_t z_applied;   // ResiSpec budget max(Z*, gap) clamped to 1 - R(x0) (streaming kernel)
 };
 
 struct __align__(16) Slot {
-  float v[kSlotFloats];  // [0..3] partials, [4..7] published values, [8] flags
+  float v[kSlotFloats];  // [0..3] partials, [4..7] published values, [8] flags, [9] min
 };
 
 struct __align__(16) Head {
@@ -188,13 +189,14 @@ __device__ __forceinline__ bool wait_bar(uint32_t bar, uint32_t parity) {
 //         target and draft rows; SUM: a0, a1 are sums (a2, a3 unused).
 //   H.pubv holds the values published by the owner thread of a token; every
 //   CTA reads them from the slot of the owner CTA `owner` (-1: none).
-//   flags are OR-ed.
+//   flags are OR-ed; `mn` is min-reduced over the cluster's CTAs (each CTA
+//   passes its own value; the result is left in H.bc[9]).
 // out[0..3]: reduced partials, out[4..7]: published values.
 template <int NWARPS, bool NORM>
 __device__ __forceinline__ void exchange(Head& H, float a0, float a1, float a2, float a3,
                                          int flags, int owner, int& xp, uint32_t& xph,
                                          uint32_t rank, uint32_t C, float (&out)[8],
-                                         int& oflags) {
+                                         int& oflags, float mn = INFINITY) {
   static_assert(NWARPS <= 16, "second reduction level covers 16 warps");
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   if constexpr (NORM) {
@@ -236,7 +238,7 @@ __device__ __forceinline__ void exchange(Head& H, float a0, float a1, float a2, 
                   __float_as_uint(a3), bar);
       st_async_v4(dst + 16, __float_as_uint(H.pubv[0]), __float_as_uint(H.pubv[1]),
                   __float_as_uint(H.pubv[2]), __float_as_uint(H.pubv[3]), bar);
-      st_async_v4(dst + 32, (uint32_t)f, 0u, 0u, 0u, bar);
+      st_async_v4(dst + 32, (uint32_t)f, __float_as_uint(mn), 0u, 0u, bar);
     }
     if (lane == 0) mbar_arrive_expect_tx(smem_addr(&H.xbar[p]), C * kSlotBytes);
     const bool ok = __all_sync(0xffffffffu, wait_bar(smem_addr(&H.xbar[p]), (xph >> p) & 1u));
@@ -247,6 +249,9 @@ __device__ __forceinline__ void exchange(Head& H, float a0, float a1, float a2, 
     a2 = got ? H.rx[p][lane].v[2] : id;
     a3 = got ? H.rx[p][lane].v[3] : 0.f;
     f = __reduce_or_sync(0xffffffffu, got ? __float_as_int(H.rx[p][lane].v[8]) : 0);
+    float mr = got ? H.rx[p][lane].v[9] : INFINITY;
+#pragma unroll
+    for (int o = 8; o; o >>= 1) mr = fminf(mr, __shfl_xor_sync(0xffffffffu, mr, o));
     if (got) {
       H.part[lane][0] = a0; H.part[lane][1] = a1; H.part[lane][2] = a2; H.part[lane][3] = a3;
     }
@@ -263,6 +268,7 @@ __device__ __forceinline__ void exchange(Head& H, float a0, float a1, float a2, 
 #pragma unroll
       for (int k = 0; k < 4; ++k) H.bc[4 + k] = has ? H.rx[p][owner].v[4 + k] : 0.f;
       H.bc[8] = __int_as_float(f | (ok ? 0 : kFlagTimeout));
+      H.bc[9] = mr;
     }
   }
   __syncthreads();

@@ -267,6 +267,18 @@ __device__ __forceinline__ float max8(const float2 (&z)[4]) {
                fmaxf(z[3].x, z[3].y));
 }
 
+// Smallest z_t - z_d of 8 pairs (the Z_applied bound min p / q is
+// 2^((z_t - z_d) c) scaled by row constants, so it is taken on the logit
+// difference).  A token with q = 0 (z_d = -inf) gives +inf and a padding
+// slot (both -inf) NaN; both are ignored by the minimum.
+__device__ __forceinline__ float dmin8(const float2 (&zt)[4], const float2 (&zd)[4]) {
+  float2 d[4];
+#pragma unroll
+  for (int j = 0; j < 4; ++j) d[j] = __ffma2_rn(zd[j], dup2(-1.f), zt[j]);
+  return fminf(fminf(fminf(d[0].x, d[0].y), fminf(d[1].x, d[1].y)),
+               fminf(fminf(d[2].x, d[2].y), fminf(d[3].x, d[3].y)));
+}
+
 __device__ __forceinline__ void rebase2(float vmax, float c, float& m, float2& s) {
   const float mnew = __fmul_rn(vmax, c);
   s = __fmul2_rn(s, dup2(ex2(__fsub_rn(m, mnew))));  // 0 from the sentinel
@@ -723,6 +735,8 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
     // at row r), and one more thread draws the visit's final uniform
     float mt = kNoRef, md = kNoRef;
     float2 st2 = make_float2(0.f, 0.f), sd2 = make_float2(0.f, 0.f);
+    float dmin = INFINITY;  // Z_applied: smallest z_t - z_d of the slice
+    const bool zapp = P.z_applied != 0 && resi;
     // (child t is found by walking t siblings; the loaded logits stay in
     // registers until the pass ends, so no warp waits for them; the draws
     // are computed by the last threads)
@@ -764,6 +778,7 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
           if (need_draft) {
             load_pairs<THREADS, BF16>(rd, zd);
             norm_accumulate<true>(zt, zd, P.scale_log2, mt, st2, md, sd2);
+            if (zapp) dmin = fminf(dmin, dmin8(zt, zd));
           } else {
             norm_accumulate<false>(zt, zd, P.scale_log2, mt, st2, md, sd2);
           }
@@ -781,7 +796,21 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
     const int flags = (bad_t ? kFlagTargetBad : 0) | (bad_d ? kFlagDraftBad : 0);
     float o[8];
     int oflags;
-    exchange<NW, true>(H, mt, st, md, sd, flags, -1, xp, xph, rank, C, o, oflags);
+    if (zapp) {
+#pragma unroll
+      for (int off = 16; off; off >>= 1) dmin = fminf(dmin, __shfl_xor_sync(0xffffffffu, dmin, off));
+      if ((tid & 31) == 0) H.wpart[tid >> 5][0] = dmin;
+      __syncthreads();
+      if (tid < 32) {
+        float v = tid < NW ? H.wpart[tid][0] : INFINITY;
+#pragma unroll
+        for (int off = 16; off; off >>= 1) v = fminf(v, __shfl_xor_sync(0xffffffffu, v, off));
+        dmin = v;
+      }
+      __syncthreads();  // the exchange below reuses H.wpart
+    }
+    exchange<NW, true>(H, mt, st, md, sd, flags, -1, xp, xph, rank, C, o, oflags, dmin);
+    const float dmin_all = H.bc[9];
     if (oflags & kFlagTimeout) { err |= kErrTimeout; break; }
     if (oflags & kFlagTargetBad) { err |= kErrNonfinite; break; }
     if (o[0] == -INFINITY) { err |= kErrEmpty; break; }
@@ -794,6 +823,12 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
     K.Md = o[2];
     K.invSd = need_draft ? __frcp_rn(o[3]) : 0.f;
     K.sig = K.invSt;
+    // Z_applied: Z* = min_{q>0} p / q = 2^(c min(z_t - z_d) - M_t + M_d) S_d / S_t,
+    // valid while no map has zeroed a token (after one, Z* = 0)
+    const float zstar = zapp ? __fdiv_rn(__fmul_rn(ex2(__fmaf_rn(dmin_all, K.c, __fsub_rn(K.Md, K.Mt))),
+                                                   K.invSt),
+                                         K.invSd)
+                             : 0.f;
     Pending Pm{kScale, -1, 0.f, 0.f, 0.f};  // parameters of the latest map (sampler masses)
     int mass_kind = 1;
 
@@ -830,6 +865,8 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
       float Z = 0.f;
       if (resi) {
         Z = __fsub_rn(qx, Rx);
+        if (zapp)  // max(Z*, |gap|), at most 1 - R(x0)
+          Z = fminf(fmaxf(nm == 0 ? zstar : 0.f, fabsf(Z)), __fsub_rn(1.f, Rx));
         if (!(Z > 0.f)) {  // degenerate rejection: R is kept unchanged
           info |= kInfoDegenerate;
           continue;

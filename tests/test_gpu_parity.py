@@ -34,7 +34,7 @@ def _check(inp, mode, seed, **kw):
     D = int(inp["max_depth"])
     g = P.run_gpu(zt, zd, pa, ca, inp["temperature"], seed, D, mode=mode, **kw)
     o = P.run_oracle(inp["target"], inp["draft"], inp["parents"], inp["cand"],
-                     inp["temperature"], seed, D, mode)
+                     inp["temperature"], seed, D, mode, z_rule=kw.get("z_rule", 0))
     n, near = P.compare(g, o)
     # near-tie differences are allowed but must stay rare
     assert near <= max(2, 0.002 * n), (near, n)
@@ -457,3 +457,29 @@ def test_parity_dynamic_trees_v128256_full_size(kernel):
     w = W.WORKLOADS["dyntree60-v128256-b64"]
     _sampled_parity(w, seed=63, call_seed=1003, rows=[0, 9, 17, 26, 35, 44, 53, 63],
                     kernel=kernel)
+
+
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+@pytest.mark.parametrize("V", [8, 64, 1000, 20001])
+def test_parity_z_applied_budget(V, dtype):
+    """The Z_applied budget variant (max(Z*, gap) clamped to 1 - R(x0)) on
+    close drafts (rho = 0.9, so min p / q can exceed the gap at a node's
+    first rejection) with single-child levels (a rejected only child leads
+    to a draw from the shaped residual, where the budget shows), every
+    sequence against the oracle with the same rule; at small V the variant
+    must change some walks."""
+    base = W.Workload(name="zapp", batch=2000, vocab=V, dtype=dtype, gen="gauss", scale=1.0,
+                      slope=0.0, rho=0.9, temperature=1.0, tree=("levels", (2, 1, 1)), steps=1)
+    B = 2000 if V <= 1000 else 200
+    inp = W.make_inputs_np(base, seed=V + 5, batch=B)
+    g, o = _check(inp, rs.MODE_RESISPEC, seed=77, z_rule=rs.Z_RULE_APPLIED)
+    o0 = P.run_oracle(inp["target"], inp["draft"], inp["parents"], inp["cand"],
+                      inp["temperature"], 77, int(inp["max_depth"]), rs.MODE_RESISPEC, z_rule=0)
+    if V <= 1000:
+        assert (o0["tokens"] != o["tokens"]).any(axis=1).sum() > 0
+
+
+def test_parity_z_applied_tree60():
+    w = W.WORKLOADS["tree60-v32000"]
+    inp = W.make_inputs_np(w, seed=8, batch=256)
+    _check(inp, rs.MODE_RESISPEC, seed=88, z_rule=rs.Z_RULE_APPLIED)

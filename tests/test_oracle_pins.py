@@ -230,3 +230,48 @@ def test_sample_endpoints():
     R = np.array([0.0, 0.3, 0.0, 0.7, 0.0])
     assert oracle.sample(R, 0.0)[0] == 1
     assert oracle.sample(R, 1 - 2 ** -24)[0] == 3
+
+
+def test_z_applied_budget_worked_examples():
+    """Z_applied = max(Z*, |q(x0) - R(x0)|), Z* = min_{q>0} R/q, clamped to
+    1 - R(x0) (Sec. 5.3 heuristic; the clamp keeps the water-fill feasible).
+    Hand-worked cases:
+      V = 2, R = (.5, .5), q = (.6, .4), reject x0 = 0: Z* = 5/6 > gap = .1,
+      clamped to 1 - R(x0) = .5; r(1) = min(.5 * .4, .5) = .2, the deficit .3
+      fills x1's capacity .3, so r = (0, .5) and R' = r / Z = (0, 1).
+      V = 3, R = (.1, .6, .3), q = (.12, .5, .38), reject x0 = 0: Z* = .3/.38
+      = 15/19 (unclamped: 1 - R(x0) = .9); r_pre = (0, 7.5/19, .3), the
+      deficit 7.5/19 - .3 fills x1 (x2 has no capacity left), so r(1) =
+      15/19 - .3 and R' = (0, 1 - .3 * 19/15, .3 * 19/15) = (0, .62, .38)."""
+    R, q = np.array([.5, .5]), np.array([.6, .4])
+    assert abs(oracle.budget(R, q, 0, 0) - 0.1) < 1e-15
+    assert abs(oracle.budget(R, q, 0, 1) - 0.5) < 1e-15
+    Rn, changed, err = oracle.reject(oracle.MODE_RESISPEC, R, q, 0, z_rule=1)
+    assert changed and err < 1e-12
+    np.testing.assert_allclose(Rn, [0.0, 1.0], atol=1e-15)
+    R, q = np.array([.1, .6, .3]), np.array([.12, .5, .38])
+    assert abs(oracle.budget(R, q, 0, 1) - 15 / 19) < 1e-15
+    Rn, changed, err = oracle.reject(oracle.MODE_RESISPEC, R, q, 0, z_rule=1)
+    assert changed and err < 1e-12
+    np.testing.assert_allclose(Rn, [0.0, 0.62, 0.38], atol=1e-14)
+
+
+def test_z_applied_equals_algorithm1_when_capacity_bound_is_below_gap():
+    """When min_{q>0} R/q <= q(x0) - R(x0) the heuristic's max picks the gap
+    and the rejection is Algorithm 1's; the bound itself is computed here
+    with numpy from R and q."""
+    rng = np.random.default_rng(11)
+    seen = 0
+    for _ in range(400):
+        V = int(rng.integers(3, 40))
+        R = rng.dirichlet(np.full(V, 0.7))
+        q = rng.dirichlet(np.full(V, 0.7))
+        x0 = int(np.argmax(q - R))
+        gap = q[x0] - R[x0]
+        if not (gap > 0) or np.min(R[q > 0] / q[q > 0]) > gap:
+            continue
+        seen += 1
+        a = oracle.reject(oracle.MODE_RESISPEC, R, q, x0, z_rule=0)[0]
+        b = oracle.reject(oracle.MODE_RESISPEC, R, q, x0, z_rule=1)[0]
+        np.testing.assert_array_equal(a, b)
+    assert seen > 100

@@ -50,6 +50,8 @@ def parse_args(argv=None):
     ap.add_argument("--rho", type=float, default=None)
     ap.add_argument("--batch", type=int, default=None, help="override the workload's batch")
     ap.add_argument("--mode", choices=["resispec", "specinfer"], default="resispec")
+    ap.add_argument("--z-rule", choices=["alg1", "applied"], default="alg1",
+                    help="ResiSpec budget: Algorithm 1's gap, or the Z_applied heuristic")
     ap.add_argument("--pool", type=int, default=0, help="input sets rotated between steps (0 = auto)")
     ap.add_argument("--cluster-size", type=int, default=0)
     ap.add_argument("--block-threads", type=int, default=0)
@@ -350,11 +352,12 @@ def run_ours(args):
              torch.empty((B, max(D, 1)), dtype=torch.int32, device=dev)) for _ in range(K)]
     status = torch.zeros((1,), dtype=torch.int32, device=dev)
     kernel = None if args.kernel == "auto" else args.kernel
+    z_rule = rs.Z_RULE_APPLIED if args.z_rule == "applied" else rs.Z_RULE_ALG1
     kw = dict(max_depth=D, mode=mode, cluster_size=args.cluster_size,
-              block_threads=args.block_threads, status=status, kernel=kernel)
+              block_threads=args.block_threads, status=status, kernel=kernel, z_rule=z_rule)
     stream = torch.cuda.current_stream(dev)
     plan = rs.plan(B, N, V, D, w.dtype, cluster_size=args.cluster_size,
-                   block_threads=args.block_threads, kernel=kernel)
+                   block_threads=args.block_threads, kernel=kernel, z_rule=z_rule)
 
     def launch(i, out):
         s = sets[i % pool]
@@ -407,7 +410,7 @@ def run_ours(args):
             "workload": w.name if B == w.batch else f"{w.name}@batch{B}", "batch": B, "vocab": V, "nodes_per_seq": N, "max_depth": D,
             "tree": list(w.tree[1]) if w.tree[0] == "levels" else list(w.tree[1:]),
             "logits": f"{w.gen} slope {w.slope} scale {w.scale} rho {w.rho}",
-            "temperature": w.temperature, "mode": args.mode,
+            "temperature": w.temperature, "mode": args.mode, "z_rule": args.z_rule,
             "parallelism": f"replicas{world}" if world > 1 else "single",
             "launch": {k: plan[k] for k in ("kernel_name", "cluster_size", "block_threads",
                                             "smem_bytes", "slice_elems", "uses_tma",
@@ -448,7 +451,7 @@ def run_ours(args):
                 dbuf[k].copy_(host[k], non_blocking=True)
             rs.verify(dbuf["target"], dbuf["draft"], dbuf["parents"], dbuf["cand"],
                       w.temperature, args.seed + i, out_tokens=d_tok, out_accept_len=d_len,
-                      max_depth=D, mode=mode, stream=stream, kernel=kernel)
+                      max_depth=D, mode=mode, stream=stream, kernel=kernel, z_rule=z_rule)
             h_tok.copy_(d_tok, non_blocking=True)
             h_len.copy_(d_len, non_blocking=True)
 

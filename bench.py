@@ -52,6 +52,8 @@ def parse_args(argv=None):
     ap.add_argument("--mode", choices=["resispec", "specinfer"], default="resispec")
     ap.add_argument("--z-rule", choices=["alg1", "applied"], default="alg1",
                     help="ResiSpec budget: Algorithm 1's gap, or the Z_applied heuristic")
+    ap.add_argument("--proxy-denominator", action="store_true",
+                    help="ResiSpec variant: each rejection's proxy becomes the test denominator")
     ap.add_argument("--pool", type=int, default=0, help="input sets rotated between steps (0 = auto)")
     ap.add_argument("--cluster-size", type=int, default=0)
     ap.add_argument("--block-threads", type=int, default=0)
@@ -354,10 +356,12 @@ def run_ours(args):
     kernel = None if args.kernel == "auto" else args.kernel
     z_rule = rs.Z_RULE_APPLIED if args.z_rule == "applied" else rs.Z_RULE_ALG1
     kw = dict(max_depth=D, mode=mode, cluster_size=args.cluster_size,
-              block_threads=args.block_threads, status=status, kernel=kernel, z_rule=z_rule)
+              block_threads=args.block_threads, status=status, kernel=kernel, z_rule=z_rule,
+              proxy_denominator=args.proxy_denominator)
     stream = torch.cuda.current_stream(dev)
     plan = rs.plan(B, N, V, D, w.dtype, cluster_size=args.cluster_size,
-                   block_threads=args.block_threads, kernel=kernel, z_rule=z_rule)
+                   block_threads=args.block_threads, kernel=kernel, z_rule=z_rule,
+                   proxy_denominator=args.proxy_denominator)
 
     def launch(i, out):
         s = sets[i % pool]
@@ -411,6 +415,7 @@ def run_ours(args):
             "tree": list(w.tree[1]) if w.tree[0] == "levels" else list(w.tree[1:]),
             "logits": f"{w.gen} slope {w.slope} scale {w.scale} rho {w.rho}",
             "temperature": w.temperature, "mode": args.mode, "z_rule": args.z_rule,
+            "proxy_denominator": args.proxy_denominator,
             "parallelism": f"replicas{world}" if world > 1 else "single",
             "launch": {k: plan[k] for k in ("kernel_name", "cluster_size", "block_threads",
                                             "smem_bytes", "slice_elems", "uses_tma",
@@ -451,7 +456,8 @@ def run_ours(args):
                 dbuf[k].copy_(host[k], non_blocking=True)
             rs.verify(dbuf["target"], dbuf["draft"], dbuf["parents"], dbuf["cand"],
                       w.temperature, args.seed + i, out_tokens=d_tok, out_accept_len=d_len,
-                      max_depth=D, mode=mode, stream=stream, kernel=kernel, z_rule=z_rule)
+                      max_depth=D, mode=mode, stream=stream, kernel=kernel, z_rule=z_rule,
+                      proxy_denominator=args.proxy_denominator)
             h_tok.copy_(d_tok, non_blocking=True)
             h_len.copy_(d_len, non_blocking=True)
 

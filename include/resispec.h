@@ -96,6 +96,14 @@ typedef struct {
                                       zeroed a token), clamped to Z <= 1 - R(x0);
                                       streaming kernel only (combined with
                                       RESISPEC_FLAG_RESIDENT: RESISPEC_E_ARG) */
+#define RESISPEC_FLAG_PROXY_DENOM 32 /* RESISPEC mode variant (the paper's EAGLE
+                                      integration, App. C): after each rejection
+                                      the test denominator becomes that rejection's
+                                      proxy K (K = R - r off x0, K(x0) = D(x0)),
+                                      and the next GetProxy takes it in place of
+                                      q; candidates stay draws from q.  Streaming
+                                      kernel only (with RESISPEC_FLAG_RESIDENT:
+                                      RESISPEC_E_ARG); no effect in SPECINFER mode */
 
 /* Kernels.  Both compute the same verification; they differ in where a
  * visited node's rows live between the passes of a visit.

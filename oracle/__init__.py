@@ -78,7 +78,7 @@ class _Args(ctypes.Structure):
         ("out_status", ctypes.c_void_p), ("out_rejects", ctypes.c_void_p),
         ("out_rows", ctypes.c_void_p), ("out_inv_err", ctypes.c_void_p),
         ("out_cond", ctypes.c_void_p), ("parents_stride", ctypes.c_int64),
-        ("z_rule", ctypes.c_int32), ("pad2_", ctypes.c_int32),
+        ("z_rule", ctypes.c_int32), ("denom_update", ctypes.c_int32),
     ]
 
 
@@ -197,7 +197,8 @@ def sample(R, u: float):
 # ---------------------------------------------------------------- full walk
 def verify(target, draft, parents, cand, temperature, seed, *, mode=MODE_RESISPEC,
            max_depth=None, seq_stride=None, seq_ids=None, nthreads=None,
-           check_invariants=False, decide_fp64=False, want_dist=False, z_rule=0):
+           check_invariants=False, decide_fp64=False, want_dist=False, z_rule=0,
+           denom_update=False):
     """Run the oracle walk.
 
     ``target``/``draft``: float32 arrays, or uint16 arrays holding bf16 bit
@@ -261,6 +262,7 @@ def verify(target, draft, parents, cand, temperature, seed, *, mode=MODE_RESISPE
     a.parents, a.cand = parents.ctypes.data, cand.ctypes.data
     a.parents_stride = N if per_seq else 0
     a.z_rule = int(z_rule)
+    a.denom_update = int(bool(denom_update))
     a.seq_ids = _ptr(seq_ids)
     a.temperature = float(np.float32(temperature))
     a.seed = int(seed) & 0xFFFFFFFFFFFFFFFF

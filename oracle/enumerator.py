@@ -16,6 +16,10 @@ oracle and vectorised over the vocabulary:
   projection r = min(Z q, R) with r(x0) = 0, the deficit filled in
   proportion to the remaining capacity R - r off x0, then
   R' = norm(max(R - K, 0)) with K = R - r and K(x0) = q(x0).
+* RESISPEC with the proxy as the next test denominator (the paper's EAGLE
+  integration, App. C): after each rejection the denominator D used by the
+  accept tests and by the next GetProxy becomes that rejection's K; the
+  candidates are still drawn from the draft q.
 """
 from __future__ import annotations
 
@@ -61,10 +65,32 @@ def shape(mode, R, q, x0):
     return shape_specinfer(R, q) if mode == MODE_SPECINFER else shape_resispec(R, q, x0)
 
 
-def single_position(p, q, k, mode):
+def accept_prob(R, D, x):
+    """P(u D(x) < R(x)) for u ~ U[0, 1)."""
+    if D[x] > 0:
+        return min(1.0, R[x] / D[x])
+    return 1.0 if R[x] > 0 else 0.0
+
+
+def reject_step(mode, R, D, x, denom_update):
+    """(R', D') after candidate x is rejected."""
+    if mode == MODE_SPECINFER or not denom_update:
+        return shape(mode, R, D, x), D
+    K, r, Z = proxy_resispec(R, D, x)
+    if not Z > 0:
+        return R.copy(), D
+    d = np.maximum(R - K, 0.0)
+    s = d.sum()
+    if not s > 0:
+        return R.copy(), D
+    return d / s, K
+
+
+def single_position(p, q, k, mode, denom_update=False):
     """Exact distribution of the emitted token when k i.i.d. candidates from q
     are tested in order against the residual chain starting at p, with the
-    residual sample after k rejections.
+    residual sample after k rejections (``denom_update``: the test
+    denominator becomes each rejection's proxy, ResiSpec mode).
 
     Returns (dist, accept_prob_by_position) where accept_prob_by_position[i]
     is P(candidate i+1 is the accepted one).
@@ -74,22 +100,23 @@ def single_position(p, q, k, mode):
     V = p.size
     acc = np.zeros(k)
 
-    def rec(R, m, weight, depth):
+    def rec(R, D, m, weight, depth):
         out = np.zeros(V)
         if m == 0:
             return R.copy()
         for x in range(V):
             if q[x] <= 0:
                 continue
-            a = min(1.0, R[x] / q[x])
+            a = accept_prob(R, D, x)
             out[x] += q[x] * a
             acc[depth] += weight * q[x] * a
             if a < 1.0:
-                R2 = shape(mode, R, q, x)
-                out += q[x] * (1.0 - a) * rec(R2, m - 1, weight * q[x] * (1.0 - a), depth + 1)
+                R2, D2 = reject_step(mode, R, D, x, denom_update)
+                out += q[x] * (1.0 - a) * rec(R2, D2, m - 1, weight * q[x] * (1.0 - a),
+                                              depth + 1)
         return out
 
-    dist = rec(p.copy(), k, 1.0, 0)
+    dist = rec(p.copy(), q.copy(), k, 1.0, 0)
     return dist, acc
 
 

@@ -50,6 +50,13 @@
  *       capacity bound of Prop. "Capacity Bound of Ideal Shaping" taken on
  *       the current residual, clamped to Z <= 1 - R(x0) so that the
  *       water-fill of step 3 stays feasible (r <= R off x0 sums to Z).
+ *   R8  proxy-as-denominator variant (flag; App. C, the EAGLE integration
+ *       "updates the current target distribution p and draft/proxy
+ *       distribution q ... before verifying the next sibling"): after a
+ *       ResiSpec rejection the test denominator D becomes the proxy K of
+ *       that rejection (K = R - r off x0, K(x0) = D(x0): a distribution),
+ *       and the next GetProxy takes D in place of q.  D starts as q at each
+ *       node.
  *   R6  the accept decision is taken in fp32, the kernel's precision
  *       (u * q(x) < R(x) with both operands rounded to fp32); the margin
  *       |u - R/q| is reported in fp64 for near-tie accounting.
@@ -367,7 +374,8 @@ typedef struct {
                               0 = one tree for all, N = parents is [B, N]
                               (per-sequence, dynamic trees) */
   int32_t z_rule;          /* ResiSpec budget: 0 Algorithm 1 (R1), 1 Z_applied (R7) */
-  int32_t pad2_;
+  int32_t denom_update;    /* 1: the test denominator becomes the proxy after
+                              each ResiSpec rejection (R8) */
 } oracle_args;
 
 typedef struct {
@@ -385,7 +393,8 @@ static int tree_is_bad(const int32_t* parents, int N) {
 
 static void verify_sequence(const oracle_args* a, int lb, int tree_bad,
                             double* z, double* p, double* q, double* R,
-                            double* K, double* r, double* tmp, int32_t* kids) {
+                            double* K, double* r, double* tmp, double* Dbuf,
+                            int32_t* kids) {
   const int V = a->V, N = a->N, D = a->D;
   const int32_t* parents = a->parents + (size_t)(a->parents_stride * lb);
   if (a->parents_stride) tree_bad = tree_is_bad(parents, N);
@@ -436,6 +445,11 @@ static void verify_sequence(const oracle_args* a, int lb, int tree_bad,
       goto done;
     }
     memcpy(R, p, sizeof(double) * V); /* R <- P, D <- Q (Algorithm 1) */
+    double* Dn = q;                   /* the test denominator */
+    if (a->denom_update && a->mode == OR_MODE_RESISPEC) {
+      memcpy(Dbuf, q, sizeof(double) * V);
+      Dn = Dbuf;                      /* becomes each rejection's proxy (R8) */
+    }
     cond = 1.0;
     int accepted = -1;
     for (int j = 0; j < nk; ++j) {
@@ -446,15 +460,15 @@ static void verify_sequence(const oracle_args* a, int lb, int tree_bad,
         goto done;
       }
       double u = oracle_uniform(a->seed, gb, c + 1, 0);
-      if (q[x] > 0.0) {
-        double m = fabs(u - R[x] / q[x]);
+      if (Dn[x] > 0.0) {
+        double m = fabs(u - R[x] / Dn[x]);
         if (m < amargin) amargin = m;
       }
       int accept;
       if (a->decide_fp64) {
-        accept = (q[x] > 0.0) ? (u < R[x] / q[x]) : (R[x] > 0.0);
+        accept = (Dn[x] > 0.0) ? (u < R[x] / Dn[x]) : (R[x] > 0.0);
       } else {
-        float uf = (float)u, qf = (float)q[x], Rf = (float)R[x];
+        float uf = (float)u, qf = (float)Dn[x], Rf = (float)R[x];
         float lhs = uf * qf;
         accept = lhs < Rf;
       }
@@ -464,8 +478,10 @@ static void verify_sequence(const oracle_args* a, int lb, int tree_bad,
       }
       rejects += 1;
       double norm = 1.0;
-      if (!oracle_reject_z(a->mode, a->z_rule, R, q, V, x, K, r, tmp, inv_ptr, &norm))
+      if (!oracle_reject_z(a->mode, a->z_rule, R, Dn, V, x, K, r, tmp, inv_ptr, &norm))
         status |= OR_INFO_DEGENERATE;
+      else if (Dn == Dbuf)
+        memcpy(Dbuf, K, sizeof(double) * V);
       cond /= norm;
     }
     if (accepted < 0) {
@@ -507,11 +523,11 @@ static void* worker(void* arg) {
   worker_ctx* w = (worker_ctx*)arg;
   const oracle_args* a = w->a;
   size_t V = (size_t)(a->V > 0 ? a->V : 1);
-  double* buf = (double*)malloc(sizeof(double) * V * 7);
+  double* buf = (double*)malloc(sizeof(double) * V * 8);
   int32_t* kids = (int32_t*)malloc(sizeof(int32_t) * (size_t)(a->N > 0 ? a->N : 1));
   for (int lb = w->tid; lb < a->B; lb += w->nthreads)
     verify_sequence(a, lb, w->tree_bad, buf, buf + V, buf + 2 * V, buf + 3 * V,
-                    buf + 4 * V, buf + 5 * V, buf + 6 * V, kids);
+                    buf + 4 * V, buf + 5 * V, buf + 6 * V, buf + 7 * V, kids);
   free(kids);
   free(buf);
   return NULL;

@@ -38,6 +38,7 @@ FLAG_PREFETCH = 2
 FLAG_RESIDENT = 4
 FLAG_STREAM = 8
 FLAG_Z_APPLIED = 16
+FLAG_PROXY_DENOM = 32
 Z_RULE_ALG1 = 0       # ResiSpec budget Z = q(x0) - R(x0) (Algorithm 1)
 Z_RULE_APPLIED = 1    # Z = max(Z*, |gap|) clamped to 1 - R(x0) (Sec. 5.3 heuristic)
 KERNEL_RESIDENT = 0
@@ -170,7 +171,8 @@ def _kernel_flags(kernel) -> int:
 
 def make_opts(mode=MODE_RESISPEC, cluster_size=0, block_threads=0, no_tma=False,
               seq_stride=None, status=None, out_nodes=None, out_dist=None,
-              out_rejects=None, prefetch=False, kernel=None, z_rule=Z_RULE_ALG1) -> Opts:
+              out_rejects=None, prefetch=False, kernel=None, z_rule=Z_RULE_ALG1,
+              proxy_denominator=False) -> Opts:
     lib = load_library()
     o = Opts()
     lib.resispec_opts_default(ctypes.byref(o))
@@ -178,7 +180,8 @@ def make_opts(mode=MODE_RESISPEC, cluster_size=0, block_threads=0, no_tma=False,
     o.cluster_size = int(cluster_size)
     o.block_threads = int(block_threads)
     o.flags = ((FLAG_NO_TMA if no_tma else 0) | (FLAG_PREFETCH if prefetch else 0)
-               | _kernel_flags(kernel) | (FLAG_Z_APPLIED if z_rule == Z_RULE_APPLIED else 0))
+               | _kernel_flags(kernel) | (FLAG_Z_APPLIED if z_rule == Z_RULE_APPLIED else 0)
+               | (FLAG_PROXY_DENOM if proxy_denominator else 0))
     o.seq_stride = -1 if seq_stride is None else int(seq_stride)
     o.status = None if status is None else status.data_ptr()
     o.out_nodes = None if out_nodes is None else out_nodes.data_ptr()
@@ -206,7 +209,7 @@ def verify(target, draft, tree_parents, cand_tokens, temperature, seed, *, max_d
            mode=MODE_RESISPEC, out_tokens=None, out_accept_len=None, out_nodes=None,
            out_dist=None, out_rejects=None, status=None, cluster_size=0, block_threads=0,
            no_tma=False, seq_stride=None, stream=None, prefetch=False, kernel=None,
-           z_rule=Z_RULE_ALG1):
+           z_rule=Z_RULE_ALG1, proxy_denominator=False):
     """Verify a batch of draft trees on the GPU.
 
     target, draft: CUDA tensors [B, N+1, V] (float32 or bfloat16); with
@@ -217,6 +220,9 @@ def verify(target, draft, tree_parents, cand_tokens, temperature, seed, *, max_d
     ``kernel``: None / "auto" (the library's choice), "resident" or "stream".
     ``z_rule``: the ResiSpec budget, Z_RULE_ALG1 (Algorithm 1) or
     Z_RULE_APPLIED (Sec. 5.3 heuristic; streaming kernel).
+    ``proxy_denominator``: after each ResiSpec rejection the accept tests
+    and the next GetProxy use that rejection's proxy in place of q (the
+    paper's EAGLE integration; streaming kernel).
     """
     torch = _torch()
     lib = load_library()
@@ -251,7 +257,7 @@ def verify(target, draft, tree_parents, cand_tokens, temperature, seed, *, max_d
     if seq_stride is None and target.numel() != B * (N + 1) * V:
         raise ValueError("target must be [B, N+1, V] (or pass seq_stride)")
     o = make_opts(mode, cluster_size, block_threads, no_tma, seq_stride, status, out_nodes,
-                  out_dist, out_rejects, prefetch, kernel, z_rule)
+                  out_dist, out_rejects, prefetch, kernel, z_rule, proxy_denominator)
     o.parents_stride = N if per_seq_tree else 0
     if stream is None:
         stream = torch.cuda.current_stream(dev)

@@ -81,6 +81,7 @@ struct VerifyParams {
   int32_t use_tma;
   int32_t prefetch;    // L2 prefetch of the first child's rows
   int32_t z_applied;   // ResiSpec budget max(Z*, gap) clamped to 1 - R(x0) (streaming kernel)
+  int32_t denom_update;  // ResiSpec: each rejection's proxy becomes the test denominator (streaming)
 };
 
 struct __align__(16) Slot {

@@ -32,6 +32,8 @@
 // cluster-wide scalars only, so any thread may compute any element and every
 // CTA evaluates the accept tests itself from the candidates' raw logits.
 #pragma once
+#include <type_traits>
+
 #include "verify_kernel.cuh"
 
 namespace rs {
@@ -56,8 +58,9 @@ constexpr int kErrFanout = 64;
 // is much smaller than R~.  Maps are applied two lanes per instruction.
 struct __align__(16) StreamHead {
   float2 map[kMaxMaps];  // {k_i, lambda_i} of map i (SpecInfer: {-k_i, 0})
+  float mdsc[kMaxMaps];  // scale of the test denominator's D~ after map i
   int rej[kMaxMaps];     // tokens whose residual is 0 (ResiSpec maps)
-  int rejk[kMaxMaps];    // their child index in this visit
+  int16_t rejk[kMaxMaps];  // their child index in this visit
   float kzt[kMaxKids];   // raw target / draft logits of the children's tokens
   float kzd[kMaxKids];
   float kua[kMaxKids];   // their accept draws U(seed, b, child + 1, 0)
@@ -341,39 +344,63 @@ __device__ __forceinline__ float2 min_part2(float2 k, float2 q, float2 R) {
   return make_float2(fminf(kq.x, R.x), fminf(kq.y, R.y));
 }
 
-template <bool RESI>
-__device__ __forceinline__ float apply_chain(const StreamHead& S2, int nm, float R, float q) {
+// Kinds of residual chain: SpecInfer maps; ResiSpec maps with the draft q
+// as the test denominator D throughout (Algorithm 1); ResiSpec maps with the
+// proxy as the next denominator (the paper's EAGLE integration, App. C).
+// With the proxy update the map is written with the current denominator:
+// m = min(k D~, R~), t = R~ - m, R~' = m + lambda t, and the proxy off the
+// rejected token is K = R - r = (1 - lambda) t, so D~' = t in units of
+// sigma_before (1 - lambda): one more value per element, no more work.
+enum : int { kChainSpec = 0, kChainResi = 1, kChainResiDenom = 2 };
+
+// The chain on one element: R~ and the denominator D~ (a draft value q~ on
+// entry; changed only by kChainResiDenom).  No rejected-token rule is
+// applied here (the callers do).
+template <int KIND>
+__device__ __forceinline__ float apply_chain(const StreamHead& S2, int nm, float R, float& D) {
   for (int i = 0; i < nm; ++i) {
     const float2 mp = S2.map[i];
-    if constexpr (RESI) {
-      const float m = fminf(__fmul_rn(mp.x, q), R);
-      R = __fmaf_rn(mp.y, __fmaf_rn(m, -1.f, R), m);
+    if constexpr (KIND == kChainSpec) {
+      R = fmaxf(__fmaf_rn(mp.x, D, R), 0.f);
     } else {
-      R = fmaxf(__fmaf_rn(mp.x, q, R), 0.f);
+      const float m = fminf(__fmul_rn(mp.x, D), R);
+      const float t = __fmaf_rn(m, -1.f, R);
+      R = __fmaf_rn(mp.y, t, m);
+      if constexpr (KIND == kChainResiDenom) D = t;
     }
   }
   return R;
 }
 
 // The same on pairs: every lane rounds exactly like apply_chain.
-template <int NP, bool RESI>
+template <int NP, int KIND>
 __device__ __forceinline__ void apply_chain_pairs(const StreamHead& S2, int nm, float2 (&R)[NP],
-                                                  const float2 (&q)[NP]) {
+                                                  float2 (&D)[NP]) {
   for (int i = 0; i < nm; ++i) {
     const float2 mp = S2.map[i];
     const float2 k = dup2(mp.x);
-    if constexpr (RESI) {
+    if constexpr (KIND == kChainSpec) {
+#pragma unroll
+      for (int j = 0; j < NP; ++j) R[j] = relu2(__ffma2_rn(k, D[j], R[j]));
+    } else {
       const float2 lam = dup2(mp.y);
 #pragma unroll
       for (int j = 0; j < NP; ++j) {
-        const float2 m = min_part2(k, q[j], R[j]);
-        R[j] = __ffma2_rn(lam, __ffma2_rn(m, dup2(-1.f), R[j]), m);
+        const float2 m = min_part2(k, D[j], R[j]);
+        const float2 t = __ffma2_rn(m, dup2(-1.f), R[j]);
+        R[j] = __ffma2_rn(lam, t, m);
+        if constexpr (KIND == kChainResiDenom) D[j] = t;
       }
-    } else {
-#pragma unroll
-      for (int j = 0; j < NP; ++j) R[j] = relu2(__ffma2_rn(k, q[j], R[j]));
     }
   }
+}
+
+template <int NP>
+__device__ __forceinline__ void apply_chain_any(const StreamHead& S2, int chain, int nm,
+                                                float2 (&R)[NP], float2 (&D)[NP]) {
+  if (chain == kChainResiDenom) apply_chain_pairs<NP, kChainResiDenom>(S2, nm, R, D);
+  else if (chain == kChainResi) apply_chain_pairs<NP, kChainResi>(S2, nm, R, D);
+  else apply_chain_pairs<NP, kChainSpec>(S2, nm, R, D);
 }
 
 // Zero the residual at rejected tokens (ResiSpec: r(x0) = 0 and the later
@@ -394,7 +421,7 @@ __device__ __forceinline__ void zero_rejected_vec(const StreamHead& S2, int nm, 
 // the rejected tokens).  base: its first token.
 template <int THREADS, bool BF16>
 __device__ __forceinline__ void final_values(const StreamHead& S2, const VisitScalars& K,
-                                             bool resi, int nm, int base,
+                                             int chain, int nm, int base,
                                              const unsigned char* rt, const unsigned char* rd,
                                              int h, float (&v)[BF16 ? 8 : 4]) {
   constexpr int VEC = BF16 ? 8 : 4;
@@ -420,15 +447,14 @@ __device__ __forceinline__ void final_values(const StreamHead& S2, const VisitSc
 #pragma unroll
   for (int j = 0; j < NP; ++j)
     q[j] = ex2x2(__ffma2_rn(make_float2(z[2 * j], z[2 * j + 1]), c2, dup2(-K.Md)));
-  if (resi) apply_chain_pairs<NP, true>(S2, nm, R, q);
-  else apply_chain_pairs<NP, false>(S2, nm, R, q);
+  apply_chain_any<NP>(S2, chain, nm, R, q);
 #pragma unroll
   for (int j = 0; j < NP; ++j) {
     const float2 r = __fmul2_rn(R[j], dup2(K.sig));
     v[2 * j] = r.x;
     v[2 * j + 1] = r.y;
   }
-  if (resi) zero_rejected_vec<VEC>(S2, nm, base, v);
+  if (chain != kChainSpec) zero_rejected_vec<VEC>(S2, nm, base, v);
 }
 
 // ---------------------------------------------------------------- sampler
@@ -441,7 +467,7 @@ __device__ __forceinline__ void final_values(const StreamHead& S2, const VisitSc
 // the token's offset in the slice (-1 if the slice has no mass).
 template <int THREADS, bool BF16>
 __device__ int stream_search(Head& H, const StreamHead& S2, float* F, unsigned char* ring,
-                             const Src& s, const VisitScalars& K, bool resi, int lo,
+                             const Src& s, const VisitScalars& K, int chain, int lo,
                              unsigned long long tau) {
   using G = StreamGeom<THREADS, BF16>;
   constexpr int VEC = G::VEC;
@@ -461,7 +487,7 @@ __device__ int stream_search(Head& H, const StreamHead& S2, float* F, unsigned c
 #pragma unroll
     for (int h = 0; h < G::VPT; ++h) {
       float v[VEC];
-      final_values<THREADS, BF16>(S2, K, resi, nm, lo + k * G::CE + (h * THREADS + (int)threadIdx.x) * VEC,
+      final_values<THREADS, BF16>(S2, K, chain, nm, lo + k * G::CE + (h * THREADS + (int)threadIdx.x) * VEC,
                                   rt, rd, h, v);
 #pragma unroll
       for (int j = 0; j < VEC; ++j) acc += to_fix(v[j]);
@@ -495,7 +521,7 @@ __device__ int stream_search(Head& H, const StreamHead& S2, float* F, unsigned c
   for (int h = 0; h < G::VPT; ++h) {
     float v[VEC];
     const int g = h * THREADS + (int)threadIdx.x;
-    final_values<THREADS, BF16>(S2, K, resi, nm, lo + ks * G::CE + g * VEC, ring, ring + G::RB, h,
+    final_values<THREADS, BF16>(S2, K, chain, nm, lo + ks * G::CE + g * VEC, ring, ring + G::RB, h,
                                 v);
 #pragma unroll
     for (int j = 0; j < VEC; ++j) F[g * VEC + j] = v[j];
@@ -577,7 +603,7 @@ __device__ int stream_search(Head& H, const StreamHead& S2, float* F, unsigned c
 // u * total (as the resident kernel's sampler); that CTA searches its slice.
 template <int THREADS, bool BF16>
 __device__ bool stream_sample(Head& H, const StreamHead& S2, float* F, unsigned char* ring,
-                              const VerifyParams& P, const Src& s_in, const VisitScalars& K, bool resi, int mass_kind,
+                              const VerifyParams& P, const Src& s_in, const VisitScalars& K, int chain, int mass_kind,
                               const Pending& Pm, float u, int b, int depth, int lo,
                               uint32_t rank, uint32_t C, int& xp, uint32_t& xph, bool& timeout) {
   using G = StreamGeom<THREADS, BF16>;
@@ -596,7 +622,7 @@ __device__ bool stream_sample(Head& H, const StreamHead& S2, float* F, unsigned 
       for (int h = 0; h < G::VPT; ++h) {
         float v[VEC];
         const int e0 = k * G::CE + (h * THREADS + (int)threadIdx.x) * VEC;  // offset in the slice
-        final_values<THREADS, BF16>(S2, K, resi, nm, lo + e0, rt, rd, h, v);
+        final_values<THREADS, BF16>(S2, K, chain, nm, lo + e0, rt, rd, h, v);
 #pragma unroll
         for (int j = 0; j < VEC; ++j) {
           sum += v[j];
@@ -640,7 +666,7 @@ __device__ bool stream_sample(Head& H, const StreamHead& S2, float* F, unsigned 
   if ((int)rank != cstar) return true;
   // A slice whose exchange mass is positive but whose every element rounds
   // to zero mass yields its first token.
-  const int pick = stream_search<THREADS, BF16>(H, S2, F, ring, s, K, resi, lo, tau);
+  const int pick = stream_search<THREADS, BF16>(H, S2, F, ring, s, K, chain, lo, tau);
   if (threadIdx.x == 0) P.out_tokens[(size_t)b * (P.D + 1) + depth] = lo + max(pick, 0);
   return true;
 }
@@ -675,6 +701,7 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
   const int lo = (int)rank * L;
   const int nloc = max(0, min(V, lo + L) - lo);
   const bool resi = P.mode == 0;
+  const int chain = !resi ? kChainSpec : (P.denom_update ? kChainResiDenom : kChainResi);
   const bool bf16 = BF16;
 
   int err = 0;
@@ -835,7 +862,7 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
     if (!need_draft) {
       // accepted leaf (or a root without children): bonus token from p
       bool to = false;
-      if (!stream_sample<THREADS, BF16>(H, S2, F, ring, P, src, K, resi, mass_kind, Pm, S2.ufin,
+      if (!stream_sample<THREADS, BF16>(H, S2, F, ring, P, src, K, chain, mass_kind, Pm, S2.ufin,
                                         b, depth, lo, rank, C, xp, xph, to))
         err |= kErrEmpty;
       if (to) err |= kErrTimeout;
@@ -843,20 +870,47 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
     }
     // ---- sequential accept tests over the children (S3), shaping on reject
     int accepted = -1, acc_tok = -1;
+    // scale of the test denominator's unnormalised values D~ (q~ until a
+    // proxy replaces it)
+    float dsc = K.invSd;
     for (int i = 0, cn = c1; cn >= 0; ++i, cn = next_sib[cn]) {
       if (i == kMaxKids) { err |= kErrFanout; break; }
       const int x = cand_s[cn];
       if (x < 0 || x >= V) { err |= kErrToken; break; }
       const int nm = S2.nmaps;
       const float qt = exp_of(S2.kzd[i], K.c, K.Md);
-      const float qx = __fmul_rn(qt, K.invSd);
+      float qx = __fmul_rn(qt, K.invSd);
       float Rt = exp_of(S2.kzt[i], K.c, K.Mt);
-      if (resi) {
-        Rt = apply_chain<true>(S2, nm, Rt, qt);
+      if (chain == kChainResiDenom) {
+        // The exact chain at x: a map that rejected x leaves R(x) = 0 and
+        // the denominator's value there unchanged (K(x0) = D(x0)); a later
+        // map then gives it R - r = 0.  D~ changes units at every map
+        // (mdsc), so keeping its value means rescaling it.
+        float D = qt, Rc = Rt, dprev = K.invSd;
+        for (int j = 0; j < nm; ++j) {
+          const float dj = S2.mdsc[j];
+          if (S2.rej[j] == x) {
+            Rc = 0.f;
+            D = __fdiv_rn(__fmul_rn(D, dprev), dj);
+          } else {
+            const float2 mp = S2.map[j];
+            const float m = fminf(__fmul_rn(mp.x, D), Rc);
+            const float t = __fmaf_rn(m, -1.f, Rc);
+            Rc = __fmaf_rn(mp.y, t, m);
+            D = t;
+          }
+          dprev = dj;
+        }
+        Rt = Rc;
+        qx = __fmul_rn(D, dprev);
+      } else if (resi) {
+        float D = qt;
+        Rt = apply_chain<kChainResi>(S2, nm, Rt, D);
         for (int j = 0; j < nm; ++j)
           if (S2.rej[j] == x) Rt = 0.f;
       } else {
-        Rt = apply_chain<false>(S2, nm, Rt, qt);
+        float D = qt;
+        Rt = apply_chain<kChainSpec>(S2, nm, Rt, D);
       }
       const float Rx = __fmul_rn(Rt, K.sig);
       const float u = S2.kua[i];
@@ -876,11 +930,13 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
       // one pass: the residual so far and the sums of the new map, in
       // unnormalised units (k: the new map's scalar).  The rejected tokens
       // get no special case here; their terms are taken out below.
-      const float kq = __fdiv_rn(resi ? __fmul_rn(Z, K.invSd) : K.invSd, K.sig);
-      // s1: sum of min(k q~, R~) (ResiSpec) or of the capacity t (SpecInfer);
-      // s2: sum of t (ResiSpec); both as pairs of lanes
+      const float kq = __fdiv_rn(resi ? __fmul_rn(Z, dsc) : K.invSd, K.sig);
+      // s1: sum of min(k D~, R~) (ResiSpec) or of the capacity t (SpecInfer);
+      // s2: sum of t (ResiSpec); both as pairs of lanes.  D~ is q~ unless the
+      // proxies replace the denominator (then the chain leaves it in q[]).
       float2 s1p = make_float2(0.f, 0.f), s2p = make_float2(0.f, 0.f);
-      {
+      auto rej_pass = [&](auto kind_c) {
+        constexpr int KIND = decltype(kind_c)::value;
         const float2 c2 = dup2(K.c), nMt = dup2(-K.Mt), nMd = dup2(-K.Md), kq2 = dup2(kq),
                      nkq = dup2(-kq);
         stream_pass<THREADS, BF16>(ring, src, [&](const unsigned char* rt, const unsigned char* rd,
@@ -894,8 +950,8 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
             q[j] = ex2x2(__ffma2_rn(q[j], c2, nMd));
           }
           float2 t[4];
-          if (resi) {
-            apply_chain_pairs<4, true>(S2, nm, Rv, q);
+          if constexpr (KIND != kChainSpec) {
+            apply_chain_pairs<4, KIND>(S2, nm, Rv, q);
             float2 m[4];
 #pragma unroll
             for (int j = 0; j < 4; ++j) {
@@ -905,14 +961,17 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
             s1p = __fadd2_rn(s1p, __fadd2_rn(__fadd2_rn(m[0], m[1]), __fadd2_rn(m[2], m[3])));
             s2p = __fadd2_rn(s2p, __fadd2_rn(__fadd2_rn(t[0], t[1]), __fadd2_rn(t[2], t[3])));
           } else {
-            apply_chain_pairs<4, false>(S2, nm, Rv, q);
+            apply_chain_pairs<4, kChainSpec>(S2, nm, Rv, q);
 #pragma unroll
             for (int j = 0; j < 4; ++j) t[j] = relu2(__ffma2_rn(nkq, q[j], Rv[j]));
             s1p = __fadd2_rn(s1p, __fadd2_rn(__fadd2_rn(t[0], t[1]), __fadd2_rn(t[2], t[3])));
           }
           return false;
         });
-      }
+      };
+      if (chain == kChainResiDenom) rej_pass(std::integral_constant<int, kChainResiDenom>{});
+      else if (chain == kChainResi) rej_pass(std::integral_constant<int, kChainResi>{});
+      else rej_pass(std::integral_constant<int, kChainSpec>{});
       float s1 = __fadd_rn(s1p.x, s1p.y), s2 = __fadd_rn(s2p.x, s2p.y);
       if (resi) {
         // The token just rejected (r(x0) = 0) and the earlier rejected ones
@@ -927,9 +986,11 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
           bool seen = t >= 0 && y == x;
           for (int t2 = 0; t2 < t && !seen; ++t2) seen = S2.rej[t2] == y;
           if (seen) continue;
-          const float qy = exp_of(S2.kzd[yk], K.c, K.Md);
-          const float Ry = apply_chain<true>(S2, nm, exp_of(S2.kzt[yk], K.c, K.Mt), qy);
-          const float my = fminf(__fmul_rn(kq, qy), Ry);
+          float Dy = exp_of(S2.kzd[yk], K.c, K.Md);
+          const float py = exp_of(S2.kzt[yk], K.c, K.Mt);
+          const float Ry = chain == kChainResiDenom ? apply_chain<kChainResiDenom>(S2, nm, py, Dy)
+                                                    : apply_chain<kChainResi>(S2, nm, py, Dy);
+          const float my = fminf(__fmul_rn(kq, Dy), Ry);
           s1 = __fsub_rn(s1, my);
           s2 = __fsub_rn(s2, __fmaf_rn(my, -1.f, Ry));
         }
@@ -957,14 +1018,17 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
         }
       }
       if (has_map) {
+        if (chain == kChainResiDenom)  // the proxy (1 - lambda) t~ becomes the denominator
+          dsc = __fmul_rn(K.sig, __fsub_rn(1.f, lam));
         K.sig = __fmul_rn(K.sig, a);
         // per-CTA masses of the new residual: (p0 + lambda p1) sig (ResiSpec)
         // or p0 sig (SpecInfer) from this exchange's unnormalised partials
         Pm = Pending{resi ? kResi : kSpec, x, K.sig, Z, lam};
         // every thread, identical values (see the visit start)
         S2.map[nm] = resi ? make_float2(kq, lam) : make_float2(-kq, 0.f);
+        S2.mdsc[nm] = dsc;
         S2.rej[nm] = x;
-        S2.rejk[nm] = i;
+        S2.rejk[nm] = (int16_t)i;
         S2.nmaps = nm + 1;
       } else {
         info |= kInfoDegenerate;
@@ -976,7 +1040,7 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
     if (accepted < 0) {
       // every child rejected: residual draw (Algorithm 1, last step)
       bool to = false;
-      if (!stream_sample<THREADS, BF16>(H, S2, F, ring, P, src, K, resi, mass_kind, Pm, S2.ufin,
+      if (!stream_sample<THREADS, BF16>(H, S2, F, ring, P, src, K, chain, mass_kind, Pm, S2.ufin,
                                         b, depth, lo, rank, C, xp, xph, to))
         err |= kErrEmpty;
       if (to) err |= kErrTimeout;

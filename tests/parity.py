@@ -72,10 +72,10 @@ def run_gpu(target, draft, parents, cand, T, seed, max_depth, mode=rs.MODE_RESIS
 
 
 def run_oracle(target_h, draft_h, parents_h, cand_h, T, seed, max_depth, mode, seq_ids=None,
-               want_dist=True, seq_stride=None, z_rule=0):
+               want_dist=True, seq_stride=None, z_rule=0, denom_update=False):
     return oracle.verify(target_h, draft_h, parents_h, cand_h, T, seed, mode=mode,
                          max_depth=max_depth, seq_ids=seq_ids, want_dist=want_dist,
-                         seq_stride=seq_stride, z_rule=z_rule)
+                         seq_stride=seq_stride, z_rule=z_rule, denom_update=denom_update)
 
 
 def compare(g, o, rows=None, check_dist=True):

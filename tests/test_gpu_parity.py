@@ -34,7 +34,8 @@ def _check(inp, mode, seed, **kw):
     D = int(inp["max_depth"])
     g = P.run_gpu(zt, zd, pa, ca, inp["temperature"], seed, D, mode=mode, **kw)
     o = P.run_oracle(inp["target"], inp["draft"], inp["parents"], inp["cand"],
-                     inp["temperature"], seed, D, mode, z_rule=kw.get("z_rule", 0))
+                     inp["temperature"], seed, D, mode, z_rule=kw.get("z_rule", 0),
+                     denom_update=kw.get("proxy_denominator", False))
     n, near = P.compare(g, o)
     # near-tie differences are allowed but must stay rare
     assert near <= max(2, 0.002 * n), (near, n)
@@ -304,21 +305,22 @@ def test_nondefault_stream():
 
 
 def _sampled_parity(w, seed, call_seed, rows, mode=rs.MODE_RESISPEC, batch=None, rho=None,
-                    kernel=None):
+                    kernel=None, **kw):
     """Full-size inputs drawn on the GPU; the oracle recomputes the sampled
     sequences `rows` one by one from the same tensors."""
     import torch
     inp = W.make_inputs_torch(w, seed, "cuda", batch=batch, rho=rho)
     D = inp["max_depth"]
     g = P.run_gpu(inp["target"], inp["draft"], inp["parents"], inp["cand"], w.temperature,
-                  call_seed, D, mode=mode, kernel=kernel)
+                  call_seed, D, mode=mode, kernel=kernel, **kw)
     ridx = torch.as_tensor(rows, device="cuda")
     th = P.to_host_logits(inp["target"].index_select(0, ridx))
     dh = P.to_host_logits(inp["draft"].index_select(0, ridx))
     ch = inp["cand"].index_select(0, ridx).cpu().numpy()
     pa = inp["parents_np"][rows] if inp["parents_np"].ndim == 2 else inp["parents_np"]
     o = P.run_oracle(th, dh, pa, ch, w.temperature, call_seed, D, mode,
-                     seq_ids=np.asarray(rows, np.int32))
+                     seq_ids=np.asarray(rows, np.int32), z_rule=kw.get("z_rule", 0),
+                     denom_update=kw.get("proxy_denominator", False))
     n, near = P.compare(g, o, rows=rows)
     assert near <= 1, near
     assert g["status"][0] & ~rs.INFO_DEGENERATE == 0
@@ -483,3 +485,62 @@ def test_parity_z_applied_tree60():
     w = W.WORKLOADS["tree60-v32000"]
     inp = W.make_inputs_np(w, seed=8, batch=256)
     _check(inp, rs.MODE_RESISPEC, seed=88, z_rule=rs.Z_RULE_APPLIED)
+
+
+@pytest.mark.parametrize("wl", ["tree60-v32000", "chain8x4-v128256-b16", "dyntree60-v32000"])
+def test_parity_proxy_denominator(wl):
+    """The proxy-as-denominator variant (the paper's EAGLE integration): the
+    accept tests and the next GetProxy use each rejection's proxy; every
+    sequence against the oracle with the same rule, which must change some
+    walks."""
+    w = W.WORKLOADS[wl]
+    inp = W.make_inputs_np(w, seed=13, batch=256 if wl != "chain8x4-v128256-b16" else 16)
+    g, o = _check(inp, rs.MODE_RESISPEC, seed=131, proxy_denominator=True)
+    o0 = P.run_oracle(inp["target"], inp["draft"], inp["parents"], inp["cand"],
+                      inp["temperature"], 131, int(inp["max_depth"]), rs.MODE_RESISPEC)
+    if wl != "chain8x4-v128256-b16":
+        assert ((o0["tokens"] != o["tokens"]).any(axis=1) | (o0["rejects"] != o["rejects"])).any()
+
+
+@pytest.mark.parametrize("mode", MODES)
+def test_proxy_denominator_wide_fanout(mode):
+    """128 children whose candidates the target all but excludes: up to 128
+    proxy updates at one node, against the oracle (SpecInfer: the flag has
+    no effect)."""
+    V, kids = 3000, rs.MAX_FANOUT_STREAM
+    rng = np.random.default_rng(kids)
+    zt = rng.normal(0, 2, (8, kids + 1, V)).astype(np.float32)
+    zd = rng.normal(0, 2, (8, kids + 1, V)).astype(np.float32)
+    cand = rng.integers(0, V, (8, kids)).astype(np.int32)
+    for b in range(8):
+        zt[b, 0, cand[b]] = -30.0
+    inp = {"target": zt, "draft": zd, "parents": np.full(kids, -1, np.int32), "cand": cand,
+           "temperature": 1.0, "max_depth": 1}
+    _check(inp, mode, seed=kids, proxy_denominator=True)
+
+
+def test_parity_proxy_denominator_binary5_full_size():
+    w = W.WORKLOADS["binary5-v151936-b64"]
+    _sampled_parity(w, seed=33, call_seed=1004, rows=[2, 19, 37, 58], proxy_denominator=True)
+
+
+def test_gpu_proxy_denominator_million_draws_vs_enumerator():
+    """The proxy-as-denominator variant on the GPU follows its own
+    enumerated law."""
+    import torch
+    V, k, n = 16, 3, 1_000_000
+    rng = np.random.default_rng(6)
+    zt = (2.0 * rng.standard_normal(V)).astype(np.float32)
+    zd = (0.8 * zt + 1.2 * rng.standard_normal(V)).astype(np.float32)
+    p, q = sp_softmax(zt.astype(np.float64)), sp_softmax(zd.astype(np.float64))
+    cand = rng.choice(V, size=(n, k), p=q).astype(np.int32)
+    toks, _ = rs.verify(P.to_device(np.broadcast_to(zt, (k + 1, V)).copy()),
+                        P.to_device(np.broadcast_to(zd, (k + 1, V)).copy()),
+                        torch.full((k,), -1, dtype=torch.int32, device="cuda"),
+                        torch.as_tensor(cand, device="cuda"), 1.0, 98, max_depth=1,
+                        seq_stride=0, proxy_denominator=True)
+    counts = np.bincount(toks[:, 0].cpu().numpy(), minlength=V)
+    dist, _ = en.single_position(p, q, k, en.MODE_RESISPEC, denom_update=True)
+    dist0, _ = en.single_position(p, q, k, en.MODE_RESISPEC)
+    assert chisq_pvalue(counts, dist)[0] > 1e-4
+    assert np.abs(dist - dist0).max() > 1e-3

@@ -377,3 +377,45 @@ def test_random_trees_are_valid_and_candidates_come_from_parent_rows():
             draft[b, r, r] = 50.0
     cand = W.candidates_np(rng, draft, trees, 1e-3)
     np.testing.assert_array_equal(cand, trees + 1)
+
+
+def test_oracle_denominator_update_matches_enumerator():
+    """Proxy-as-denominator variant (the test denominator becomes each
+    rejection's proxy K): oracle draws against the independently enumerated
+    law of the same rule, GetProxy invariants at every rejection, and the law
+    differs from Algorithm 1's."""
+    V, k, n = 8, 3, 400_000
+    zt, zd = _pq(43, V, scale=1.5, rho=0.3)
+    target, draft, cand = _single_position_draws(6, V, k, n, zt, zd)
+    out = oracle.verify(target, draft, W.tree_single(k), cand, 1.0, seed=4321,
+                        mode=oracle.MODE_RESISPEC, seq_stride=0, check_invariants=True,
+                        denom_update=True)
+    assert (out["status"] & ~oracle.INFO_DEGENERATE == 0).all()
+    assert out["inv_err"].max() < 1e-12
+    p = sp_softmax(zt.astype(np.float64))
+    q = sp_softmax(zd.astype(np.float64))
+    dist, acc = en.single_position(p, q, k, oracle.MODE_RESISPEC, denom_update=True)
+    pv, nb = chisq_pvalue(np.bincount(out["tokens"][:, 0], minlength=V), dist)
+    assert pv > 1e-4, (pv, nb)
+    which = np.where(out["accept_len"] > 0, out["nodes"][:, 0], k)
+    pv2, _ = chisq_pvalue(np.bincount(which, minlength=k + 1), np.append(acc, 1 - acc.sum()))
+    assert pv2 > 1e-4
+    dist0, _ = en.single_position(p, q, k, oracle.MODE_RESISPEC)
+    assert np.abs(dist - dist0).max() > 1e-3
+
+
+def test_denominator_update_is_algorithm1_at_two_tokens():
+    """V = 2: after a rejection the residual is the point mass on the other
+    token under either denominator, so every later test of it accepts and
+    every test of the rejected token rejects: the variant's outputs equal
+    Algorithm 1's."""
+    rng = np.random.default_rng(9)
+    for _ in range(20):
+        zt = rng.normal(0, 1.5, (1, 5, 2)).astype(np.float32)
+        zd = rng.normal(0, 1.5, (1, 5, 2)).astype(np.float32)
+        cand = rng.integers(0, 2, (300, 4)).astype(np.int32)
+        kw = dict(mode=oracle.MODE_RESISPEC, seq_stride=0, want_dist=True)
+        a = oracle.verify(zt[0], zd[0], W.tree_single(4), cand, 1.0, 3, **kw)
+        b = oracle.verify(zt[0], zd[0], W.tree_single(4), cand, 1.0, 3, denom_update=True, **kw)
+        for key in ("tokens", "accept_len", "nodes", "rejects", "dist"):
+            np.testing.assert_array_equal(a[key], b[key])

@@ -73,6 +73,18 @@ typedef enum { RESISPEC_MODE_RESISPEC = 0, RESISPEC_MODE_SPECINFER = 1 } resispe
                                       tests at most that many children per node) */
 #define RESISPEC_INFO_DEGENERATE 256 /* informational: a rejection left R unchanged */
 
+/* Phases of out_phase_cycles.  The paper splits ResiSpec's cost into
+ * budgeting, redistribution and proxy formulation: budgeting is part of
+ * RESISPEC_PHASE_TEST, redistribution is RESISPEC_PHASE_REJECT, and the
+ * proxy is never materialised (R' = r / Z directly). */
+#define RESISPEC_PHASE_SETUP 0     /* before the first pass (setup overlaps it) */
+#define RESISPEC_PHASE_NORM 1      /* normaliser passes */
+#define RESISPEC_PHASE_NORM_X 2    /* their cluster exchanges */
+#define RESISPEC_PHASE_TEST 3      /* accept tests and budgets */
+#define RESISPEC_PHASE_REJECT 4    /* rejection passes and their exchanges */
+#define RESISPEC_PHASE_DRAW 5      /* residual / bonus draw */
+#define RESISPEC_PHASES 6
+
 #define RESISPEC_MAX_VOCAB 262144
 #define RESISPEC_MAX_NODES 4096
 #define RESISPEC_MAX_FANOUT_STREAM 128
@@ -134,6 +146,10 @@ typedef struct {
                             last emitted token was drawn from (final residual
                             R, or p of the accepted leaf) */
   int32_t* out_rejects;  /* optional device [B] number of rejections */
+  int64_t* out_phase_cycles; /* optional device [B, RESISPEC_PHASES] int64: SM
+                                cycles (clock64 on the sequence's first CTA)
+                                spent per phase, RESISPEC_PHASE_*; asking for
+                                it selects the streaming kernel */
   int64_t parents_stride; /* int32 elements between sequences' trees in
                              tree_parents: 0 (default) = one tree [N] shared by
                              every sequence; N = tree_parents is [B, N], a tree

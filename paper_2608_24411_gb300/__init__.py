@@ -41,6 +41,7 @@ FLAG_Z_APPLIED = 16
 FLAG_PROXY_DENOM = 32
 Z_RULE_ALG1 = 0       # ResiSpec budget Z = q(x0) - R(x0) (Algorithm 1)
 Z_RULE_APPLIED = 1    # Z = max(Z*, |gap|) clamped to 1 - R(x0) (Sec. 5.3 heuristic)
+PHASES = ("setup", "norm", "norm_exchange", "test", "reject", "draw")
 KERNEL_RESIDENT = 0
 KERNEL_STREAM = 1
 KERNELS = {"auto": None, "resident": KERNEL_RESIDENT, "stream": KERNEL_STREAM}
@@ -72,7 +73,8 @@ class Opts(ctypes.Structure):
                 ("block_threads", ctypes.c_int32), ("flags", ctypes.c_int32),
                 ("seq_stride", ctypes.c_int64), ("status", ctypes.c_void_p),
                 ("out_nodes", ctypes.c_void_p), ("out_dist", ctypes.c_void_p),
-                ("out_rejects", ctypes.c_void_p), ("parents_stride", ctypes.c_int64)]
+                ("out_rejects", ctypes.c_void_p), ("out_phase_cycles", ctypes.c_void_p),
+                ("parents_stride", ctypes.c_int64)]
 
 
 class PlanInfo(ctypes.Structure):
@@ -209,7 +211,7 @@ def verify(target, draft, tree_parents, cand_tokens, temperature, seed, *, max_d
            mode=MODE_RESISPEC, out_tokens=None, out_accept_len=None, out_nodes=None,
            out_dist=None, out_rejects=None, status=None, cluster_size=0, block_threads=0,
            no_tma=False, seq_stride=None, stream=None, prefetch=False, kernel=None,
-           z_rule=Z_RULE_ALG1, proxy_denominator=False):
+           z_rule=Z_RULE_ALG1, proxy_denominator=False, out_phase=None):
     """Verify a batch of draft trees on the GPU.
 
     target, draft: CUDA tensors [B, N+1, V] (float32 or bfloat16); with
@@ -223,6 +225,8 @@ def verify(target, draft, tree_parents, cand_tokens, temperature, seed, *, max_d
     ``proxy_denominator``: after each ResiSpec rejection the accept tests
     and the next GetProxy use that rejection's proxy in place of q (the
     paper's EAGLE integration; streaming kernel).
+    ``out_phase``: optional int64 CUDA tensor [B, len(PHASES)] receiving the
+    SM cycles each sequence spent per phase (selects the streaming kernel).
     """
     torch = _torch()
     lib = load_library()
@@ -259,6 +263,11 @@ def verify(target, draft, tree_parents, cand_tokens, temperature, seed, *, max_d
     o = make_opts(mode, cluster_size, block_threads, no_tma, seq_stride, status, out_nodes,
                   out_dist, out_rejects, prefetch, kernel, z_rule, proxy_denominator)
     o.parents_stride = N if per_seq_tree else 0
+    if out_phase is not None:
+        _need_cuda("out_phase", out_phase)
+        if out_phase.dtype != torch.int64 or tuple(out_phase.shape) != (B, len(PHASES)):
+            raise ValueError("out_phase must be int64 [B, 6]")
+        o.out_phase_cycles = out_phase.data_ptr()
     if stream is None:
         stream = torch.cuda.current_stream(dev)
     handle = stream.cuda_stream if hasattr(stream, "cuda_stream") else int(stream)

@@ -269,7 +269,8 @@ int make_plan(const resispec_dims& d, const resispec_opts& o, int dev, int sms,
   if (o.seq_stride < -1) return RESISPEC_E_ARG;
   if (o.parents_stride < 0) return RESISPEC_E_ARG;
   const bool force_res = (o.flags & RESISPEC_FLAG_RESIDENT) != 0;
-  const bool variant = (o.flags & (RESISPEC_FLAG_Z_APPLIED | RESISPEC_FLAG_PROXY_DENOM)) != 0;
+  const bool variant = (o.flags & (RESISPEC_FLAG_Z_APPLIED | RESISPEC_FLAG_PROXY_DENOM)) != 0 ||
+                       o.out_phase_cycles != nullptr;
   const bool force_str = (o.flags & RESISPEC_FLAG_STREAM) != 0 || variant;
   if (force_res && force_str) return RESISPEC_E_ARG;
   p->threads = o.block_threads ? o.block_threads : 512;
@@ -437,6 +438,7 @@ int resispec_verify_ex(const void* target_logits, const void* draft_logits,
   prm.out_nodes = o.out_nodes;
   prm.out_dist = o.out_dist;
   prm.out_rejects = o.out_rejects;
+  prm.out_phase = o.out_phase_cycles;
   prm.status = o.status;
   prm.seq_stride = o.seq_stride < 0 ? (int64_t)(dims.num_nodes + 1) * dims.vocab : o.seq_stride;
   prm.parents_stride = o.parents_stride;

@@ -69,6 +69,7 @@ struct VerifyParams {
   int32_t* out_nodes;
   float* out_dist;
   int32_t* out_rejects;
+  int64_t* out_phase;    // optional [B, 6] cycles per phase (streaming kernel)
   int32_t* status;
   int64_t seq_stride;  // elements
   int64_t parents_stride;  // elements between sequences' trees (0: one tree)

@@ -39,6 +39,11 @@
 namespace rs {
 
 constexpr int kMaxMaps = 128;          // residual maps per node (rejections with a map)
+// Phases of the optional per-sequence cycle counters: setup, normaliser
+// passes, normaliser exchanges, accept tests and budgets (the paper's
+// "budgeting"), rejection passes with their exchanges ("redistribution"; the
+// proxy is never materialised), the final draw.
+enum : int { kPhaseSetup = 0, kPhaseNorm, kPhaseNormX, kPhaseTest, kPhaseRej, kPhaseDraw, kPhases };
 constexpr int kMaxKids = kMaxMaps;      // children per node the streaming kernel walks
 static_assert(2 * kMaxKids <= 256, "per-visit loads and draws use distinct threads of a CTA");
 constexpr int kErrFanout = 64;
@@ -66,6 +71,10 @@ struct __align__(16) StreamHead {
   float kua[kMaxKids];   // their accept draws U(seed, b, child + 1, 0)
   float ufin;            // the visit's final draw U(seed, b, row, 1)
   int nmaps;
+  // optional phase counters (clock64 cycles, thread 0): see kPhase*
+  unsigned long long phc[kPhases];
+  unsigned long long ph_last;
+  int ph_cur;
 };
 constexpr int kStreamHeadBytes = 4096;
 static_assert(sizeof(StreamHead) <= kStreamHeadBytes, "stream head too large");
@@ -738,6 +747,22 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
     if (tree_bad) err = kErrTree;
   };
 
+  // optional phase counters (thread 0 of every CTA; rank 0 writes them)
+  const bool prof = P.out_phase != nullptr;
+  auto mark = [&](int ph) {
+    if (prof && tid == 0) {
+      const unsigned long long now = clock64();
+      S2.phc[S2.ph_cur] += now - S2.ph_last;
+      S2.ph_last = now;
+      S2.ph_cur = ph;
+    }
+  };
+  if (prof && tid == 0) {
+    for (int k = 0; k < kPhases; ++k) S2.phc[k] = 0ull;
+    S2.ph_last = clock64();
+    S2.ph_cur = kPhaseSetup;
+  }
+
   for (bool first = true; !err; first = false) {
     int c1 = first ? -1 : first_child[node + 1];
     const bool need_draft = first ? N > 0 : c1 >= 0;
@@ -755,6 +780,7 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
     // orders these writes after every read of the old values.
     S2.nmaps = 0;
 
+    mark(kPhaseNorm);
     // ---- tempered normaliser (S2): online (reference, sum) per row; while
     // the first chunks are in flight, one thread per child reads its token's
     // raw logits and draws its accept uniform (one Philox block per logit
@@ -836,7 +862,9 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
       }
       __syncthreads();  // the exchange below reuses H.wpart
     }
+    mark(kPhaseNormX);
     exchange<NW, true>(H, mt, st, md, sd, flags, -1, xp, xph, rank, C, o, oflags, dmin);
+    mark(kPhaseTest);
     const float dmin_all = H.bc[9];
     if (oflags & kFlagTimeout) { err |= kErrTimeout; break; }
     if (oflags & kFlagTargetBad) { err |= kErrNonfinite; break; }
@@ -862,6 +890,7 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
     if (!need_draft) {
       // accepted leaf (or a root without children): bonus token from p
       bool to = false;
+      mark(kPhaseDraw);
       if (!stream_sample<THREADS, BF16>(H, S2, F, ring, P, src, K, chain, mass_kind, Pm, S2.ufin,
                                         b, depth, lo, rank, C, xp, xph, to))
         err |= kErrEmpty;
@@ -927,6 +956,7 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
         }
       }
       if (nm >= kMaxMaps) { err |= kErrFanout; break; }
+      mark(kPhaseRej);
       // one pass: the residual so far and the sums of the new map, in
       // unnormalised units (k: the new map's scalar).  The rejected tokens
       // get no special case here; their terms are taken out below.
@@ -996,6 +1026,7 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
         }
       }
       exchange<NW, false>(H, s1, s2, 0.f, 0.f, 0, -1, xp, xph, rank, C, o, oflags);
+      mark(kPhaseTest);
       if (oflags & kFlagTimeout) { err |= kErrTimeout; break; }
       bool has_map = false;
       float a = 0.f, lam = 0.f;
@@ -1040,6 +1071,7 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
     if (accepted < 0) {
       // every child rejected: residual draw (Algorithm 1, last step)
       bool to = false;
+      mark(kPhaseDraw);
       if (!stream_sample<THREADS, BF16>(H, S2, F, ring, P, src, K, chain, mass_kind, Pm, S2.ufin,
                                         b, depth, lo, rank, C, xp, xph, to))
         err |= kErrEmpty;
@@ -1057,6 +1089,9 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
     __syncthreads();  // every read of this visit's S2 state precedes the next visit's writes
   }
 
+  mark(kPhaseSetup);
+  if (prof && rank == 0 && tid == 0)
+    for (int k = 0; k < kPhases; ++k) P.out_phase[(size_t)b * kPhases + k] = (int64_t)S2.phc[k];
   if (rank == 0 && tid == 0) {
     int32_t* toks = P.out_tokens + (size_t)b * (D + 1);
     if (err) {

@@ -544,3 +544,51 @@ def test_gpu_proxy_denominator_million_draws_vs_enumerator():
     dist0, _ = en.single_position(p, q, k, en.MODE_RESISPEC)
     assert chisq_pvalue(counts, dist)[0] > 1e-4
     assert np.abs(dist - dist0).max() > 1e-3
+
+
+@pytest.mark.parametrize("mode", MODES)
+def test_diagnostics_match_oracle(mode):
+    """Acceptance by candidate position (one position, 8 candidates) and the
+    accepted length of a depth-4 chain with 4 candidates per position, from
+    the kernel's outputs and from the oracle's on the same inputs, over the
+    sequences without a near tie."""
+    from paper_2608_24411_gb300 import diagnostics as dg
+    for tree, B in ((("single", 8), 512), (("chain", 4, 4), 256)):
+        w = W.Workload(name="diag", batch=B, vocab=32000, dtype="bf16", gen="zipf", scale=3.0,
+                       slope=1.1, rho=0.8, temperature=1.0, tree=tree, steps=1)
+        inp = W.make_inputs_np(w, seed=91, batch=B)
+        g, o = _check(inp, mode, seed=92)
+        clean = (o["accept_margin"] > P.ACCEPT_TIE) & (o["sample_margin"] > P.SAMPLE_TIE)
+        if tree[0] == "single":
+            pg = dg.accepted_position(g["accept_len"], g["nodes"], 8)[clean]
+            po = dg.accepted_position(o["accept_len"], o["nodes"], 8)[clean]
+            for a, b in zip(dg.position_rates(pg, 8), dg.position_rates(po, 8)):
+                np.testing.assert_array_equal(a, b)
+        else:
+            assert (g["accept_len"][clean] + 1).mean() == (o["accept_len"][clean] + 1).mean()
+
+
+def test_phase_counters():
+    """Per-sequence cycle counters: filled for every sequence, no rejection
+    phase when every first candidate is accepted (identical rows), a
+    rejection phase when the target excludes every candidate."""
+    import torch
+    V, k, B = 4000, 4, 32
+    rng = np.random.default_rng(3)
+    z = rng.normal(0, 2, (B, k + 1, V)).astype(np.float32)
+    cand = rng.integers(0, V, (B, k)).astype(np.int32)
+    parents = np.full(k, -1, np.int32)
+    for same in (True, False):
+        zt = z.copy()
+        if not same:
+            for b in range(B):
+                zt[b, 0, cand[b]] = -30.0
+        cyc = torch.full((B, len(rs.PHASES)), -1, dtype=torch.int64, device="cuda")
+        toks, alen = rs.verify(P.to_device(zt), P.to_device(z), torch.as_tensor(parents, device="cuda"),
+                               torch.as_tensor(cand, device="cuda"), 1.0, 4, max_depth=1,
+                               mode=rs.MODE_SPECINFER, out_phase=cyc)
+        c = cyc.cpu().numpy()
+        assert (c >= 0).all() and (c.sum(axis=1) > 0).all()
+        rej = c[:, rs.PHASES.index("reject")]
+        assert (rej == 0).all() if same else (rej > 0).all()
+        assert (c[:, rs.PHASES.index("norm")] > 0).all() and (c[:, rs.PHASES.index("draw")] > 0).all()

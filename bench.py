@@ -54,6 +54,8 @@ def parse_args(argv=None):
                     help="ResiSpec budget: Algorithm 1's gap, or the Z_applied heuristic")
     ap.add_argument("--proxy-denominator", action="store_true",
                     help="ResiSpec variant: each rejection's proxy becomes the test denominator")
+    ap.add_argument("--draft", action="store_true",
+                    help="drafting mode: the kernel draws the visited nodes' children from q")
     ap.add_argument("--pool", type=int, default=0, help="input sets rotated between steps (0 = auto)")
     ap.add_argument("--cluster-size", type=int, default=0)
     ap.add_argument("--block-threads", type=int, default=0)
@@ -360,14 +362,17 @@ def run_ours(args):
               proxy_denominator=args.proxy_denominator)
     stream = torch.cuda.current_stream(dev)
     plan = rs.plan(B, N, V, D, w.dtype, cluster_size=args.cluster_size,
-                   block_threads=args.block_threads, kernel=kernel, z_rule=z_rule,
-                   proxy_denominator=args.proxy_denominator)
+                   block_threads=args.block_threads,
+                   kernel="stream" if (args.draft and kernel is None) else kernel,
+                   z_rule=z_rule, proxy_denominator=args.proxy_denominator)
+
+    drafted = torch.empty((B, N), dtype=torch.int32, device=dev) if args.draft else None
 
     def launch(i, out):
         s = sets[i % pool]
-        rs.verify(s["target"], s["draft"], s["parents"], s["cand"], w.temperature,
-                  args.seed + i, out_tokens=out[0], out_accept_len=out[1], out_nodes=out[2],
-                  stream=stream, **kw)
+        rs.verify(s["target"], s["draft"], s["parents"], None if args.draft else s["cand"],
+                  w.temperature, args.seed + i, out_tokens=out[0], out_accept_len=out[1],
+                  out_nodes=out[2], stream=stream, out_candidates=drafted, **kw)
 
     for i in range(Wm):
         launch(i, outs[i % K])
@@ -415,7 +420,7 @@ def run_ours(args):
             "tree": list(w.tree[1]) if w.tree[0] == "levels" else list(w.tree[1:]),
             "logits": f"{w.gen} slope {w.slope} scale {w.scale} rho {w.rho}",
             "temperature": w.temperature, "mode": args.mode, "z_rule": args.z_rule,
-            "proxy_denominator": args.proxy_denominator,
+            "proxy_denominator": args.proxy_denominator, "draft": args.draft,
             "parallelism": f"replicas{world}" if world > 1 else "single",
             "launch": {k: plan[k] for k in ("kernel_name", "cluster_size", "block_threads",
                                             "smem_bytes", "slice_elems", "uses_tma",

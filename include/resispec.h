@@ -150,6 +150,15 @@ typedef struct {
                                 cycles (clock64 on the sequence's first CTA)
                                 spent per phase, RESISPEC_PHASE_*; asking for
                                 it selects the streaming kernel */
+  int32_t* out_candidates; /* optional device [B, N] int32: drafting mode.  The
+                              children of every visited node are drawn from that
+                              node's tempered draft distribution (Algorithm 1,
+                              "x_1..x_k ~ Q i.i.d.": inverse CDF over ascending
+                              token ids, child c with u = word 2 of the Philox
+                              block of row c + 1) and written here (-1 for the
+                              nodes whose parent is not visited); cand_tokens is
+                              then not read (may be NULL).  Selects the
+                              streaming kernel */
   int64_t parents_stride; /* int32 elements between sequences' trees in
                              tree_parents: 0 (default) = one tree [N] shared by
                              every sequence; N = tree_parents is [B, N], a tree

@@ -79,6 +79,7 @@ class _Args(ctypes.Structure):
         ("out_rows", ctypes.c_void_p), ("out_inv_err", ctypes.c_void_p),
         ("out_cond", ctypes.c_void_p), ("parents_stride", ctypes.c_int64),
         ("z_rule", ctypes.c_int32), ("denom_update", ctypes.c_int32),
+        ("draft_out", ctypes.c_void_p), ("out_draft_margin", ctypes.c_void_p),
     ]
 
 
@@ -198,7 +199,7 @@ def sample(R, u: float):
 def verify(target, draft, parents, cand, temperature, seed, *, mode=MODE_RESISPEC,
            max_depth=None, seq_stride=None, seq_ids=None, nthreads=None,
            check_invariants=False, decide_fp64=False, want_dist=False, z_rule=0,
-           denom_update=False):
+           denom_update=False, draft_children=False):
     """Run the oracle walk.
 
     ``target``/``draft``: float32 arrays, or uint16 arrays holding bf16 bit
@@ -263,6 +264,11 @@ def verify(target, draft, parents, cand, temperature, seed, *, mode=MODE_RESISPE
     a.parents_stride = N if per_seq else 0
     a.z_rule = int(z_rule)
     a.denom_update = int(bool(denom_update))
+    if draft_children:  # candidates drawn from each visited node's q (cand is ignored)
+        out["drafted"] = np.full((B, N), -1, np.int32)
+        out["draft_margin"] = np.zeros(B)
+        a.draft_out = out["drafted"].ctypes.data
+        a.out_draft_margin = out["draft_margin"].ctypes.data
     a.seq_ids = _ptr(seq_ids)
     a.temperature = float(np.float32(temperature))
     a.seed = int(seed) & 0xFFFFFFFFFFFFFFFF

@@ -57,6 +57,11 @@
  *       that rejection (K = R - r off x0, K(x0) = D(x0): a distribution),
  *       and the next GetProxy takes D in place of q.  D starts as q at each
  *       node.
+ *   R9  drafting (flag; Algorithm 1's "x_1..x_k ~ Q i.i.d."): the children of
+ *       each visited node are drawn from that node's tempered draft
+ *       distribution q by inverse CDF over ascending token ids, child c
+ *       with u = word 2 of the Philox block of row c + 1, in child order
+ *       before the node's accept tests; the drawn tokens replace cand.
  *   R6  the accept decision is taken in fp32, the kernel's precision
  *       (u * q(x) < R(x) with both operands rounded to fp32); the margin
  *       |u - R/q| is reported in fp64 for near-tie accounting.
@@ -376,6 +381,10 @@ typedef struct {
   int32_t z_rule;          /* ResiSpec budget: 0 Algorithm 1 (R1), 1 Z_applied (R7) */
   int32_t denom_update;    /* 1: the test denominator becomes the proxy after
                               each ResiSpec rejection (R8) */
+  int32_t* draft_out;      /* non-NULL: draft the children of visited nodes
+                              (R9) into [B, N] (-1 elsewhere) instead of
+                              reading cand */
+  double* out_draft_margin; /* [B] smallest relative CDF margin of those draws */
 } oracle_args;
 
 typedef struct {
@@ -401,6 +410,10 @@ static void verify_sequence(const oracle_args* a, int lb, int tree_bad,
   const int64_t gb = a->seq_ids ? a->seq_ids[lb] : lb;
   const double T = a->temperature;
   int32_t* toks = a->out_tokens ? a->out_tokens + (size_t)lb * (D + 1) : NULL;
+  int32_t* drafted = a->draft_out ? a->draft_out + (size_t)lb * N : NULL;
+  double dmargin = INFINITY;
+  if (drafted)
+    for (int c = 0; c < N; ++c) drafted[c] = -1;
   int32_t* nodes = a->out_nodes ? a->out_nodes + (size_t)lb * D : NULL;
   if (toks)
     for (int i = 0; i <= D; ++i) toks[i] = -1;
@@ -444,6 +457,12 @@ static void verify_sequence(const oracle_args* a, int lb, int tree_bad,
       status |= st;
       goto done;
     }
+    if (drafted) /* x_1..x_k ~ Q i.i.d. (R9) */
+      for (int j = 0; j < nk; ++j) {
+        double m = INFINITY;
+        drafted[kids[j]] = oracle_sample(q, V, oracle_uniform(a->seed, gb, kids[j] + 1, 2), &m);
+        if (m < dmargin) dmargin = m;
+      }
     memcpy(R, p, sizeof(double) * V); /* R <- P, D <- Q (Algorithm 1) */
     double* Dn = q;                   /* the test denominator */
     if (a->denom_update && a->mode == OR_MODE_RESISPEC) {
@@ -454,7 +473,7 @@ static void verify_sequence(const oracle_args* a, int lb, int tree_bad,
     int accepted = -1;
     for (int j = 0; j < nk; ++j) {
       int c = kids[j];
-      int x = a->cand[(size_t)lb * N + c];
+      int x = drafted ? drafted[c] : a->cand[(size_t)lb * N + c];
       if (x < 0 || x >= V) {
         status |= OR_ERR_TOKEN;
         goto done;
@@ -495,7 +514,7 @@ static void verify_sequence(const oracle_args* a, int lb, int tree_bad,
       status |= OR_ERR_DEPTH;
       goto done;
     }
-    if (toks) toks[depth] = a->cand[(size_t)lb * N + accepted];
+    if (toks) toks[depth] = drafted ? drafted[accepted] : a->cand[(size_t)lb * N + accepted];
     if (nodes) nodes[depth] = accepted;
     depth += 1;
     node = accepted;
@@ -513,6 +532,7 @@ done:
   if (a->out_status) a->out_status[lb] = status;
   if (a->out_accept_margin) a->out_accept_margin[lb] = amargin;
   if (a->out_sample_margin) a->out_sample_margin[lb] = smargin;
+  if (a->out_draft_margin) a->out_draft_margin[lb] = dmargin;
   if (a->out_rejects) a->out_rejects[lb] = rejects;
   if (a->out_rows) a->out_rows[lb] = rows;
   if (a->out_inv_err) a->out_inv_err[lb] = inv;

@@ -74,6 +74,7 @@ class Opts(ctypes.Structure):
                 ("seq_stride", ctypes.c_int64), ("status", ctypes.c_void_p),
                 ("out_nodes", ctypes.c_void_p), ("out_dist", ctypes.c_void_p),
                 ("out_rejects", ctypes.c_void_p), ("out_phase_cycles", ctypes.c_void_p),
+                ("out_candidates", ctypes.c_void_p),
                 ("parents_stride", ctypes.c_int64)]
 
 
@@ -211,7 +212,8 @@ def verify(target, draft, tree_parents, cand_tokens, temperature, seed, *, max_d
            mode=MODE_RESISPEC, out_tokens=None, out_accept_len=None, out_nodes=None,
            out_dist=None, out_rejects=None, status=None, cluster_size=0, block_threads=0,
            no_tma=False, seq_stride=None, stream=None, prefetch=False, kernel=None,
-           z_rule=Z_RULE_ALG1, proxy_denominator=False, out_phase=None):
+           z_rule=Z_RULE_ALG1, proxy_denominator=False, out_phase=None,
+           out_candidates=None):
     """Verify a batch of draft trees on the GPU.
 
     target, draft: CUDA tensors [B, N+1, V] (float32 or bfloat16); with
@@ -227,17 +229,25 @@ def verify(target, draft, tree_parents, cand_tokens, temperature, seed, *, max_d
     paper's EAGLE integration; streaming kernel).
     ``out_phase``: optional int64 CUDA tensor [B, len(PHASES)] receiving the
     SM cycles each sequence spent per phase (selects the streaming kernel).
+    ``out_candidates``: drafting mode, an int32 CUDA tensor [B, N] that
+    receives the children of every visited node drawn from that node's draft
+    distribution (then verified); ``cand_tokens`` may be None.
     """
     torch = _torch()
     lib = load_library()
     for name, t in (("target", target), ("draft", draft), ("tree_parents", tree_parents),
-                    ("cand_tokens", cand_tokens), ("out_tokens", out_tokens),
+                    ("cand_tokens", cand_tokens), ("out_candidates", out_candidates),
+                    ("out_tokens", out_tokens),
                     ("out_accept_len", out_accept_len), ("out_nodes", out_nodes),
                     ("out_dist", out_dist), ("out_rejects", out_rejects), ("status", status)):
         _need_cuda(name, t)
     if draft.dtype != target.dtype:
         raise TypeError("target and draft must have the same dtype")
     dt = _dtype_code(target)
+    if cand_tokens is None:
+        if out_candidates is None:
+            raise ValueError("pass cand_tokens, or out_candidates to draft them")
+        cand_tokens = out_candidates   # not read in drafting mode; gives B
     if tree_parents.dtype != torch.int32 or cand_tokens.dtype != torch.int32:
         raise TypeError("tree_parents and cand_tokens must be int32")
     per_seq_tree = tree_parents.dim() == 2
@@ -268,6 +278,10 @@ def verify(target, draft, tree_parents, cand_tokens, temperature, seed, *, max_d
         if out_phase.dtype != torch.int64 or tuple(out_phase.shape) != (B, len(PHASES)):
             raise ValueError("out_phase must be int64 [B, 6]")
         o.out_phase_cycles = out_phase.data_ptr()
+    if out_candidates is not None:
+        if out_candidates.dtype != torch.int32 or tuple(out_candidates.shape) != (B, N):
+            raise ValueError("out_candidates must be int32 [B, N]")
+        o.out_candidates = out_candidates.data_ptr()
     if stream is None:
         stream = torch.cuda.current_stream(dev)
     handle = stream.cuda_stream if hasattr(stream, "cuda_stream") else int(stream)

@@ -270,7 +270,7 @@ int make_plan(const resispec_dims& d, const resispec_opts& o, int dev, int sms,
   if (o.parents_stride < 0) return RESISPEC_E_ARG;
   const bool force_res = (o.flags & RESISPEC_FLAG_RESIDENT) != 0;
   const bool variant = (o.flags & (RESISPEC_FLAG_Z_APPLIED | RESISPEC_FLAG_PROXY_DENOM)) != 0 ||
-                       o.out_phase_cycles != nullptr;
+                       o.out_phase_cycles != nullptr || o.out_candidates != nullptr;
   const bool force_str = (o.flags & RESISPEC_FLAG_STREAM) != 0 || variant;
   if (force_res && force_str) return RESISPEC_E_ARG;
   p->threads = o.block_threads ? o.block_threads : 512;
@@ -412,7 +412,8 @@ int resispec_verify_ex(const void* target_logits, const void* draft_logits,
   if (!(temperature > 0.f) || !isfinite(temperature)) return RESISPEC_E_ARG;
   if (dims.batch == 0) return RESISPEC_OK;
   if (!target_logits || !draft_logits || !out_tokens || !out_accept_len) return RESISPEC_E_ARG;
-  if (dims.num_nodes > 0 && (!tree_parents || !cand_tokens)) return RESISPEC_E_ARG;
+  if (dims.num_nodes > 0 && (!tree_parents || (!cand_tokens && !o.out_candidates)))
+    return RESISPEC_E_ARG;
   int dev = 0;
   DeviceInfo info;
   st = query_device(&dev, &info);
@@ -439,6 +440,7 @@ int resispec_verify_ex(const void* target_logits, const void* draft_logits,
   prm.out_dist = o.out_dist;
   prm.out_rejects = o.out_rejects;
   prm.out_phase = o.out_phase_cycles;
+  prm.draft_out = o.out_candidates;
   prm.status = o.status;
   prm.seq_stride = o.seq_stride < 0 ? (int64_t)(dims.num_nodes + 1) * dims.vocab : o.seq_stride;
   prm.parents_stride = o.parents_stride;

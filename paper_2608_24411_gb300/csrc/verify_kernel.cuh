@@ -70,6 +70,7 @@ struct VerifyParams {
   float* out_dist;
   int32_t* out_rejects;
   int64_t* out_phase;    // optional [B, 6] cycles per phase (streaming kernel)
+  int32_t* draft_out;    // drafting: [B, N] children drawn from q (streaming kernel)
   int32_t* status;
   int64_t seq_stride;  // elements
   int64_t parents_stride;  // elements between sequences' trees (0: one tree)

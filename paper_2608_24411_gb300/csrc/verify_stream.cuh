@@ -711,6 +711,7 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
   const int nloc = max(0, min(V, lo + L) - lo);
   const bool resi = P.mode == 0;
   const int chain = !resi ? kChainSpec : (P.denom_update ? kChainResiDenom : kChainResi);
+  const bool drafting = P.draft_out != nullptr;
   const bool bf16 = BF16;
 
   int err = 0;
@@ -738,13 +739,83 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
       const bool ok = p >= -1 && p < i;
       bad |= !ok;
       par[i] = (int16_t)(ok ? p : -2);
-      cand_s[i] = __ldg(P.cand + (size_t)b * N + i);
+      cand_s[i] = drafting ? -1 : __ldg(P.cand + (size_t)b * N + i);
+      if (drafting && rank == 0) P.draft_out[(size_t)b * N + i] = -1;
     }
     const bool tree_bad = __syncthreads_or(bad) != 0;
     build_children(par, first_child, next_sib, N);
     __syncthreads();
     cluster_sync();  // every peer has started: its receive slots may now be written
     if (tree_bad) err = kErrTree;
+  };
+
+  // Drafting (Algorithm 1's "x_1..x_k ~ Q i.i.d."): the children of each
+  // visited node are drawn here from the node's tempered draft row, after
+  // its normaliser, instead of being read from cand.
+  auto draft_children = [&](int c1d, const VisitScalars& K, size_t rbase) {
+    // per-CTA draft masses from the normaliser exchange, the CTA and the
+    // threshold inside it of each child's draw; kept in the children's logit
+    // slots (refilled below) and the rejected-token list (empty until the
+    // node's first map), which the searches do not touch
+    static_assert(offsetof(StreamHead, kzd) == offsetof(StreamHead, kzt) + sizeof(StreamHead::kzt) &&
+                      offsetof(StreamHead, kzt) % 8 == 0 &&
+                      sizeof(StreamHead::kzt) + sizeof(StreamHead::kzd) >=
+                          kMaxKids * sizeof(unsigned long long),
+                  "draft thresholds fit the logit slots");
+    unsigned long long* tau = reinterpret_cast<unsigned long long*>(S2.kzt);
+    int* owner = S2.rej;
+    if (tid == 0) {
+      unsigned long long total = 0;
+      for (uint32_t r = 0; r < C; ++r)
+        total += to_fix(__fmul_rn(H.part[r][3], ref_scale(H.part[r][2], K.Md, K.invSd)));
+      int i = 0;
+      for (int cn = c1d; cn >= 0 && i < kMaxKids; cn = next_sib[cn], ++i) {
+        const float u = uniform_draw(P.seed, (uint32_t)b, (uint32_t)(cn + 1), 2);
+        const unsigned long long kk = (unsigned long long)(u * 16777216.f);
+        const unsigned long long t = (__umul64hi(kk, total) << 40) | ((kk * total) >> 24);
+        unsigned long long a = 0;
+        int r_own = total > 0 ? (int)C - 1 : -1;
+        for (uint32_t r = 0; r < C && total > 0; ++r) {
+          const unsigned long long m =
+              to_fix(__fmul_rn(H.part[r][3], ref_scale(H.part[r][2], K.Md, K.invSd)));
+          if (a + m > t) { r_own = (int)r; break; }
+          a += m;
+        }
+        tau[i] = t > a ? t - a : 0ull;
+        owner[i] = r_own;
+      }
+      H.misc[6] = i;
+    }
+    __syncthreads();
+    const int nk = H.misc[6];
+    // q values come out of the sampler's search with the draft row in
+    // place of the target row and the draft's scalars
+    Src sq;
+    sq.t = static_cast<const char*>(P.zd) + (rbase + (size_t)lo) * es;
+    sq.d = sq.t;
+    sq.rows = 1;
+    sq.nloc = nloc;
+    sq.vec = P.use_tma != 0;
+    VisitScalars Kq = K;
+    Kq.Mt = K.Md;
+    Kq.invSt = K.invSd;
+    for (int i = 0, cn = c1d; i < nk; ++i, cn = next_sib[cn]) {
+      if (owner[i] != (int)rank) continue;
+      const int pick = stream_search<THREADS, BF16>(H, S2, F, ring, sq, Kq, chain, lo, tau[i]);
+      if (tid == 0) P.draft_out[(size_t)b * N + cn] = lo + max(pick, 0);
+    }
+    cluster_sync();  // every drawn token written (release / acquire at cluster scope)
+    // the children's tokens and their raw logits
+    if (tid < nk) {
+      int cn = c1d;
+      for (int k = 0; k < tid; ++k) cn = next_sib[cn];
+      const int x = __ldcg(P.draft_out + (size_t)b * N + cn);
+      cand_s[cn] = x;
+      const bool okx = x >= 0 && x < V;
+      S2.kzt[tid] = okx ? raw_logit(P.zt, rbase + (size_t)x, bf16) : 0.f;
+      S2.kzd[tid] = okx ? raw_logit(P.zd, rbase + (size_t)x, bf16) : 0.f;
+    }
+    __syncthreads();
   };
 
   // optional phase counters (thread 0 of every CTA; rank 0 writes them)
@@ -806,7 +877,7 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
             setup();
             c1 = first_child[0];
           }
-          if (tid < kMaxKids && need_draft && !err) {
+          if (tid < kMaxKids && need_draft && !err && !drafting) {
             const int cn = nth_child(tid);
             if (cn >= 0) {
               const int x = cand_s[cn];
@@ -878,6 +949,7 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
     K.Md = o[2];
     K.invSd = need_draft ? __frcp_rn(o[3]) : 0.f;
     K.sig = K.invSt;
+    if (drafting && need_draft) draft_children(c1, K, rbase);
     // Z_applied: Z* = min_{q>0} p / q = 2^(c min(z_t - z_d) - M_t + M_d) S_d / S_t,
     // valid while no map has zeroed a token (after one, Z* = 0)
     const float zstar = zapp ? __fdiv_rn(__fmul_rn(ex2(__fmaf_rn(dmin_all, K.c, __fsub_rn(K.Md, K.Mt))),

@@ -50,7 +50,7 @@ def run_gpu(target, draft, parents, cand, T, seed, max_depth, mode=rs.MODE_RESIS
             want_dist=True, **kw):
     """target/draft/parents/cand: torch CUDA tensors."""
     import torch
-    B = cand.shape[0]
+    B = (cand if cand is not None else kw["out_candidates"]).shape[0]
     V = target.shape[-1]
     dev = target.device
     out = {

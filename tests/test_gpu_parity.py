@@ -592,3 +592,52 @@ def test_phase_counters():
         rej = c[:, rs.PHASES.index("reject")]
         assert (rej == 0).all() if same else (rej > 0).all()
         assert (c[:, rs.PHASES.index("norm")] > 0).all() and (c[:, rs.PHASES.index("draw")] > 0).all()
+
+
+def _check_drafting(inp, mode, seed, **kw):
+    import torch
+    zt, zd, pa, _ = _np_inputs_to_gpu(inp)
+    D = int(inp["max_depth"])
+    B, N = inp["cand"].shape
+    drafted = torch.full((B, N), -7, dtype=torch.int32, device="cuda")
+    g = P.run_gpu(zt, zd, pa, None, inp["temperature"], seed, D, mode=mode,
+                  out_candidates=drafted, **kw)
+    o = oracle.verify(inp["target"], inp["draft"], inp["parents"], inp["cand"],
+                      inp["temperature"], seed, mode=mode, max_depth=D, want_dist=True,
+                      draft_children=True)
+    o["sample_margin"] = np.minimum(o["sample_margin"], o["draft_margin"])
+    n, near = P.compare(g, o)
+    assert near <= max(2, 0.01 * n), (near, n)
+    gd = drafted.cpu().numpy()
+    clean = (o["accept_margin"] > P.ACCEPT_TIE) & (o["sample_margin"] > P.SAMPLE_TIE)
+    np.testing.assert_array_equal(gd[clean], o["drafted"][clean])
+    return gd, o
+
+
+@pytest.mark.parametrize("mode", MODES)
+@pytest.mark.parametrize("wl", ["tree60-v32000", "chain8x4-v128256-b16", "dyntree60-v32000"])
+def test_parity_drafting(wl, mode):
+    """Drafting mode: the kernel draws the children of every visited node
+    from the node's draft distribution, then verifies them; tokens, accept
+    lengths and drafted candidates against the oracle's drafting walk."""
+    w = W.WORKLOADS[wl]
+    inp = W.make_inputs_np(w, seed=17, batch=256 if wl != "chain8x4-v128256-b16" else 16)
+    gd, _ = _check_drafting(inp, mode, seed=170 + mode)
+    assert (gd[:, :1] >= 0).all()   # the root's first child is always drawn
+
+
+def test_gpu_drafted_candidates_follow_q():
+    import torch
+    V, k, n = 16, 3, 1_000_000
+    rng = np.random.default_rng(8)
+    zt = (2.0 * rng.standard_normal(V)).astype(np.float32)
+    zd = (0.8 * zt + 1.2 * rng.standard_normal(V)).astype(np.float32)
+    q = sp_softmax(zd.astype(np.float64))
+    drafted = torch.full((n, k), -7, dtype=torch.int32, device="cuda")
+    rs.verify(P.to_device(np.broadcast_to(zt, (k + 1, V)).copy()),
+              P.to_device(np.broadcast_to(zd, (k + 1, V)).copy()),
+              torch.full((k,), -1, dtype=torch.int32, device="cuda"), None, 1.0, 97,
+              max_depth=1, seq_stride=0, out_candidates=drafted)
+    d = drafted.cpu().numpy()
+    assert (d[:, 0] >= 0).all()
+    assert chisq_pvalue(np.bincount(d[:, 0], minlength=V), q)[0] > 1e-4

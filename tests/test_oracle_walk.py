@@ -419,3 +419,26 @@ def test_denominator_update_is_algorithm1_at_two_tokens():
         b = oracle.verify(zt[0], zd[0], W.tree_single(4), cand, 1.0, 3, denom_update=True, **kw)
         for key in ("tokens", "accept_len", "nodes", "rejects", "dist"):
             np.testing.assert_array_equal(a[key], b[key])
+
+
+def test_oracle_drafted_candidates_follow_q():
+    """Drafting (Algorithm 1's x_1..x_k ~ Q i.i.d.): every drafted child of
+    the root is a draw from the root's tempered draft softmax; the first two
+    children are drawn independently of each other."""
+    V, k, n = 16, 3, 200_000
+    zt, zd = _pq(44, V, scale=1.5, rho=0.5)
+    target = np.ascontiguousarray(np.broadcast_to(zt, (k + 1, V)), dtype=np.float32)
+    draft = np.ascontiguousarray(np.broadcast_to(zd, (k + 1, V)), dtype=np.float32)
+    cand = np.zeros((n, k), np.int32)
+    out = oracle.verify(target, draft, W.tree_single(k), cand, 1.0, seed=77, seq_stride=0,
+                        draft_children=True)
+    q = sp_softmax(zd.astype(np.float64))
+    d = out["drafted"]
+    for j in range(k):
+        assert (d[:, j] >= 0).all()
+        assert chisq_pvalue(np.bincount(d[:, j], minlength=V), q)[0] > 1e-4
+    joint = np.bincount(d[:, 0] * V + d[:, 1], minlength=V * V)
+    assert chisq_pvalue(joint, np.outer(q, q).ravel())[0] > 1e-4
+    # an accepted candidate is emitted as drafted
+    acc = out["accept_len"] >= 1
+    np.testing.assert_array_equal(out["tokens"][acc, 0], d[acc, out["nodes"][acc, 0]])

@@ -35,6 +35,8 @@ MODE_RESISPEC = 0
 MODE_SPECINFER = 1
 F32 = 0
 BF16 = 1
+FILL_CAPACITY = 0  # the deficit in proportion to the remaining capacity (R2)
+FILL_LEVEL = 1     # r = min(lam q, p) at a common level lam (R10)
 
 ERR_TREE = 1
 ERR_TOKEN = 2
@@ -80,6 +82,7 @@ class _Args(ctypes.Structure):
         ("out_cond", ctypes.c_void_p), ("parents_stride", ctypes.c_int64),
         ("z_rule", ctypes.c_int32), ("denom_update", ctypes.c_int32),
         ("draft_out", ctypes.c_void_p), ("out_draft_margin", ctypes.c_void_p),
+        ("fill", ctypes.c_int32), ("pad2_", ctypes.c_int32),
     ]
 
 
@@ -104,12 +107,17 @@ def load():
                                              ctypes.c_int, ctypes.c_int,
                                              ctypes.c_void_p, ctypes.c_void_p]
             lib.oracle_get_proxy.restype = ctypes.c_double
+            lib.oracle_get_proxy_z.argtypes = [ctypes.c_void_p, ctypes.c_void_p,
+                                               ctypes.c_int, ctypes.c_int, ctypes.c_double,
+                                               ctypes.c_int, ctypes.c_void_p, ctypes.c_void_p]
+            lib.oracle_get_proxy_z.restype = ctypes.c_double
             lib.oracle_reject.argtypes = [ctypes.c_int, ctypes.c_void_p, ctypes.c_void_p,
                                           ctypes.c_int, ctypes.c_int, ctypes.c_void_p,
                                           ctypes.c_void_p, ctypes.c_void_p,
                                           ctypes.c_void_p]
             lib.oracle_reject.restype = ctypes.c_int
-            lib.oracle_reject_z.argtypes = [ctypes.c_int, ctypes.c_int, ctypes.c_void_p,
+            lib.oracle_reject_z.argtypes = [ctypes.c_int, ctypes.c_int, ctypes.c_int,
+                                            ctypes.c_void_p,
                                             ctypes.c_void_p, ctypes.c_int, ctypes.c_int,
                                             ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p,
                                             ctypes.c_void_p, ctypes.c_void_p]
@@ -158,12 +166,17 @@ def softmax(z, temperature: float):
     return p, st
 
 
-def get_proxy(p, q, x0: int):
-    """GetProxy(p, q, x0) -> (k, r, Z)."""
+def get_proxy(p, q, x0: int, fill: int = FILL_CAPACITY, Z=None):
+    """GetProxy(p, q, x0) -> (k, r, Z).  ``fill``: FILL_CAPACITY (the deficit
+    in proportion to the capacity p - r) or FILL_LEVEL (r = min(lam q, p) at
+    the level lam that meets the budget); ``Z``: the budget (default
+    q(x0) - p(x0), Algorithm 1)."""
     p, q = _f64(p), _f64(q)
     k, r = np.zeros_like(p), np.zeros_like(p)
-    Z = load().oracle_get_proxy(p.ctypes.data, q.ctypes.data, p.size, int(x0),
-                                k.ctypes.data, r.ctypes.data)
+    if Z is None:
+        Z = q[int(x0)] - p[int(x0)]
+    Z = load().oracle_get_proxy_z(p.ctypes.data, q.ctypes.data, p.size, int(x0), float(Z),
+                                  int(fill), k.ctypes.data, r.ctypes.data)
     return k, r, Z
 
 
@@ -174,14 +187,16 @@ def budget(R, q, x0: int, z_rule: int = 0) -> float:
     return load().oracle_budget(R.ctypes.data, q.ctypes.data, R.size, int(x0), int(z_rule))
 
 
-def reject(mode: int, R, q, x0: int, check: bool = True, z_rule: int = 0):
+def reject(mode: int, R, q, x0: int, check: bool = True, z_rule: int = 0,
+           fill: int = FILL_CAPACITY):
     """One rejection of x0: returns (R', changed, invariant_error)."""
     R = _f64(R).copy()
     q = _f64(q)
     V = R.size
     K, r, tmp = np.zeros(V), np.zeros(V), np.zeros(V)
     err = np.zeros(1)
-    changed = load().oracle_reject_z(int(mode), int(z_rule), R.ctypes.data, q.ctypes.data, V,
+    changed = load().oracle_reject_z(int(mode), int(z_rule), int(fill), R.ctypes.data,
+                                     q.ctypes.data, V,
                                      int(x0), K.ctypes.data, r.ctypes.data, tmp.ctypes.data,
                                      err.ctypes.data if check else None, None)
     return R, bool(changed), float(err[0])
@@ -199,7 +214,7 @@ def sample(R, u: float):
 def verify(target, draft, parents, cand, temperature, seed, *, mode=MODE_RESISPEC,
            max_depth=None, seq_stride=None, seq_ids=None, nthreads=None,
            check_invariants=False, decide_fp64=False, want_dist=False, z_rule=0,
-           denom_update=False, draft_children=False):
+           denom_update=False, draft_children=False, fill=0):
     """Run the oracle walk.
 
     ``target``/``draft``: float32 arrays, or uint16 arrays holding bf16 bit
@@ -264,6 +279,7 @@ def verify(target, draft, parents, cand, temperature, seed, *, mode=MODE_RESISPE
     a.parents_stride = N if per_seq else 0
     a.z_rule = int(z_rule)
     a.denom_update = int(bool(denom_update))
+    a.fill = int(fill)
     if draft_children:  # candidates drawn from each visited node's q (cand is ignored)
         out["drafted"] = np.full((B, N), -1, np.int32)
         out["draft_margin"] = np.zeros(B)

@@ -20,6 +20,12 @@ oracle and vectorised over the vocabulary:
   integration, App. C): after each rejection the denominator D used by the
   accept tests and by the next GetProxy becomes that rejection's K; the
   candidates are still drawn from the draft q.
+* RESISPEC with the level fill (``fill=1``): r = min(lam q, R) off x0 with
+  the level lam >= Z that makes sum r = Z, found here by bisection on the
+  nondecreasing function lam -> sum min(lam q, R) (the C oracle solves it
+  exactly on the sorted ratios instead); when no finite level reaches Z,
+  r = R on the support of q and the tokens with q = 0 take the rest in
+  proportion to R.
 """
 from __future__ import annotations
 
@@ -37,23 +43,46 @@ def shape_specinfer(R, q, x0=None):
     return R.copy() if not s > 0 else d / s
 
 
-def proxy_resispec(R, q, x0):
+def level_by_bisection(R, q, x0, Z, iters=200):
+    """The level lam with sum_{x != x0} min(lam q, R) = Z, or inf when the
+    support of q cannot hold Z."""
+    w = np.ones(R.size, dtype=bool)
+    w[x0] = False
+    f = lambda lam: float(np.minimum(lam * q[w], R[w]).sum())
+    if R[w & (q > 0)].sum() < Z:
+        return np.inf
+    lo, hi = 0.0, 1.0
+    while f(hi) < Z:
+        hi *= 2.0
+    for _ in range(iters):
+        mid = 0.5 * (lo + hi)
+        if f(mid) < Z:
+            lo = mid
+        else:
+            hi = mid
+        if hi - lo <= 4e-16 * hi:
+            break
+    return hi
+
+
+def proxy_resispec(R, q, x0, fill=0):
     """Returns (K, r, Z) of GetProxy(R, q, x0)."""
     Z = q[x0] - R[x0]
-    r = np.minimum(Z * q, R)
+    lam = Z if fill == 0 else level_by_bisection(R, q, x0, Z)
+    r = np.minimum(lam * q, R) if np.isfinite(lam) else np.where(q > 0, R, 0.0)
     r[x0] = 0.0
     cap = R - r
     cap[x0] = 0.0
     deficit = Z - r.sum()
-    if cap.sum() > 0:
+    if cap.sum() > 0 and (fill == 0 or not np.isfinite(lam)):
         r = r + deficit * cap / cap.sum()
     K = R - r
     K[x0] = q[x0]
     return K, r, Z
 
 
-def shape_resispec(R, q, x0):
-    K, r, Z = proxy_resispec(R, q, x0)
+def shape_resispec(R, q, x0, fill=0):
+    K, r, Z = proxy_resispec(R, q, x0, fill)
     if not Z > 0:
         return R.copy()
     d = np.maximum(R - K, 0.0)
@@ -61,8 +90,8 @@ def shape_resispec(R, q, x0):
     return R.copy() if not s > 0 else d / s
 
 
-def shape(mode, R, q, x0):
-    return shape_specinfer(R, q) if mode == MODE_SPECINFER else shape_resispec(R, q, x0)
+def shape(mode, R, q, x0, fill=0):
+    return shape_specinfer(R, q) if mode == MODE_SPECINFER else shape_resispec(R, q, x0, fill)
 
 
 def accept_prob(R, D, x):
@@ -72,11 +101,11 @@ def accept_prob(R, D, x):
     return 1.0 if R[x] > 0 else 0.0
 
 
-def reject_step(mode, R, D, x, denom_update):
+def reject_step(mode, R, D, x, denom_update, fill=0):
     """(R', D') after candidate x is rejected."""
     if mode == MODE_SPECINFER or not denom_update:
-        return shape(mode, R, D, x), D
-    K, r, Z = proxy_resispec(R, D, x)
+        return shape(mode, R, D, x, fill), D
+    K, r, Z = proxy_resispec(R, D, x, fill)
     if not Z > 0:
         return R.copy(), D
     d = np.maximum(R - K, 0.0)
@@ -86,7 +115,7 @@ def reject_step(mode, R, D, x, denom_update):
     return d / s, K
 
 
-def single_position(p, q, k, mode, denom_update=False):
+def single_position(p, q, k, mode, denom_update=False, fill=0):
     """Exact distribution of the emitted token when k i.i.d. candidates from q
     are tested in order against the residual chain starting at p, with the
     residual sample after k rejections (``denom_update``: the test
@@ -111,7 +140,7 @@ def single_position(p, q, k, mode, denom_update=False):
             out[x] += q[x] * a
             acc[depth] += weight * q[x] * a
             if a < 1.0:
-                R2, D2 = reject_step(mode, R, D, x, denom_update)
+                R2, D2 = reject_step(mode, R, D, x, denom_update, fill)
                 out += q[x] * (1.0 - a) * rec(R2, D2, m - 1, weight * q[x] * (1.0 - a),
                                               depth + 1)
         return out
@@ -120,7 +149,7 @@ def single_position(p, q, k, mode, denom_update=False):
     return dist, acc
 
 
-def tree_walk(parents, rows, mode):
+def tree_walk(parents, rows, mode, fill=0):
     """Exact distribution over emitted token tuples for a draft tree.
 
     ``parents``: int [N] (parent < child, -1 = root).  ``rows(path)`` returns
@@ -160,7 +189,7 @@ def tree_walk(parents, rows, mode):
                         key = (x,) + seq
                         out[key] = out.get(key, 0.0) + q[x] * a * pr
                 if a < 1.0:
-                    R2 = shape(mode, R, q, x)
+                    R2 = shape(mode, R, q, x, fill)
                     for seq, pr in rec(R2, j + 1).items():
                         out[seq] = out.get(seq, 0.0) + q[x] * (1.0 - a) * pr
             return out

@@ -62,6 +62,14 @@
  *       distribution q by inverse CDF over ascending token ids, child c
  *       with u = word 2 of the Philox block of row c + 1, in child order
  *       before the node's accept tests; the drawn tokens replace cand.
+ *   R10 lambda-level fill (flag; another reading of step 3, which only asks
+ *       that the deficit go to tokens still below their capacity p): the
+ *       filled mass is the draft raised to a common level, r = min(lam q, p)
+ *       off x0 with lam chosen so that sum r = Z.  sum_{i != x0} min(lam q_i,
+ *       p_i) is continuous, nondecreasing and linear between the ratios
+ *       p_i / q_i, so lam is found exactly on the sorted ratios.  If even
+ *       r = p on the support of q leaves a deficit, the tokens with q = 0
+ *       (other than x0) take it in proportion to p, the rule of R2.
  *   R6  the accept decision is taken in fp32, the kernel's precision
  *       (u * q(x) < R(x) with both operands rounded to fp32); the margin
  *       |u - R/q| is reported in fp64 for near-tie accounting.
@@ -175,16 +183,17 @@ int oracle_softmax(const double* z, int V, double T, double* p) {
 /* GetProxy(p, q, x0) of Algorithm 1, with p the current residual R.
  *   step 1  Z = q(x0) - p(x0)                         (budget, Sec. 5.3)
  *   step 2  r_i = min(Z q_i, p_i) for i != x0, r_x0 = 0 (projection)
- *   step 3  Delta = Z - sum r; fill Delta into the capacity p - r (R2)
+ *   step 3  Delta = Z - sum r; fill Delta into the capacity p - r (R2), or
+ *           raise the draft to a common level (fill 1, R10)
  *   step 4  k = p - r + s, then k(x0) = q(x0)          (s = 0 off x0, R3)
  * Writes k and r (either may be NULL) and returns Z.  The caller must only
  * use k when Z > 0 (R5). */
-double oracle_get_proxy_z(const double* p, const double* q, int V, int x0, double Z,
+double oracle_get_proxy_z(const double* p, const double* q, int V, int x0, double Z, int fill,
                           double* k, double* r);
 
 double oracle_get_proxy(const double* p, const double* q, int V, int x0,
                         double* k, double* r) {
-  return oracle_get_proxy_z(p, q, V, x0, q[x0] - p[x0], k, r);
+  return oracle_get_proxy_z(p, q, V, x0, q[x0] - p[x0], 0, k, r);
 }
 
 /* The budget of a rejection of x0: rule 0 = Algorithm 1 (R1), rule 1 =
@@ -199,20 +208,68 @@ double oracle_budget(const double* R, const double* q, int V, int x0, int rule) 
   return fmin(Z, 1.0 - R[x0]);
 }
 
-/* GetProxy with the budget Z given (steps 2-4 below). */
-double oracle_get_proxy_z(const double* p, const double* q, int V, int x0, double Z,
+typedef struct {
+  double ratio;
+  int i;
+} ratio_item;
+
+static int by_ratio(const void* a, const void* b) {
+  const double x = ((const ratio_item*)a)->ratio, y = ((const ratio_item*)b)->ratio;
+  return x < y ? -1 : (x > y ? 1 : 0);
+}
+
+/* The level of R10: the lam >= 0 with sum_{i != x0, q_i > 0} min(lam q_i,
+ * p_i) = Z, or INFINITY when even lam = inf leaves the sum below Z.  The
+ * ratios p_i / q_i are visited in ascending order; before ratio j the tokens
+ * below it are saturated (they give p_i) and the rest give lam q_i, so the
+ * crossing piece is solved in closed form. */
+static double lambda_level(const double* p, const double* q, int V, int x0, double Z) {
+  int n = 0;
+  ratio_item* it = (ratio_item*)malloc(sizeof(ratio_item) * (size_t)(V > 0 ? V : 1));
+  double* suf_q = (double*)malloc(sizeof(double) * (size_t)(V + 1));
+  for (int i = 0; i < V; ++i)
+    if (i != x0 && q[i] > 0.0) {
+      it[n].ratio = p[i] / q[i];
+      it[n].i = i;
+      ++n;
+    }
+  qsort(it, (size_t)n, sizeof(ratio_item), by_ratio);
+  suf_q[n] = 0.0;
+  for (int j = n - 1; j >= 0; --j) suf_q[j] = suf_q[j + 1] + q[it[j].i];
+  double lam = INFINITY, pre_p = 0.0;
+  for (int j = 0; j < n; ++j) {
+    const double at = pre_p + it[j].ratio * suf_q[j]; /* S(ratio_j) */
+    if (at >= Z) {
+      lam = (Z - pre_p) / suf_q[j];
+      break;
+    }
+    pre_p += p[it[j].i];
+  }
+  free(it);
+  free(suf_q);
+  return lam;
+}
+
+/* GetProxy with the budget Z and the fill rule given (steps 2-4 below). */
+double oracle_get_proxy_z(const double* p, const double* q, int V, int x0, double Z, int fill,
                           double* k, double* r) {
   double* rr = r ? r : (double*)malloc(sizeof(double) * (size_t)V);
+  const double level = fill == 1 ? lambda_level(p, q, V, x0, Z) : Z;
   double sum_r = 0.0;
   for (int i = 0; i < V; ++i) {
-    rr[i] = (i == x0) ? 0.0 : fmin(Z * q[i], p[i]);
+    /* step 2 at the level Z (R2), or at the level that meets Z (R10); with
+       lam = inf the support of q is saturated */
+    const double lq = (level == INFINITY) ? (q[i] > 0.0 ? INFINITY : 0.0) : level * q[i];
+    rr[i] = (i == x0) ? 0.0 : fmin(lq, p[i]);
     sum_r += rr[i];
   }
   double delta = Z - sum_r;
   double sum_cap = 0.0;
   for (int i = 0; i < V; ++i)
     if (i != x0) sum_cap += p[i] - rr[i];
-  if (sum_cap > 0.0) {
+  /* the capacity fill (R2; for R10 only the deficit that the level cannot
+     meet, which leaves capacity on q = 0 tokens alone) */
+  if (sum_cap > 0.0 && (fill != 1 || level == INFINITY)) {
     for (int i = 0; i < V; ++i)
       if (i != x0) rr[i] += delta * (p[i] - rr[i]) / sum_cap;
   }
@@ -239,7 +296,7 @@ static double residual_from(double* R, const double* K, int V, double* tmp) {
 int oracle_reject_ex(int mode, double* R, const double* q, int V, int x0,
                      double* K, double* r, double* tmp, double* inv_err,
                      double* norm_out);
-int oracle_reject_z(int mode, int z_rule, double* R, const double* q, int V, int x0,
+int oracle_reject_z(int mode, int z_rule, int fill, double* R, const double* q, int V, int x0,
                     double* K, double* r, double* tmp, double* inv_err, double* norm_out);
 
 /* One rejection of token x0 applied to the residual R (length V).
@@ -258,11 +315,12 @@ int oracle_reject(int mode, double* R, const double* q, int V, int x0,
 int oracle_reject_ex(int mode, double* R, const double* q, int V, int x0,
                      double* K, double* r, double* tmp, double* inv_err,
                      double* norm_out) {
-  return oracle_reject_z(mode, 0, R, q, V, x0, K, r, tmp, inv_err, norm_out);
+  return oracle_reject_z(mode, 0, 0, R, q, V, x0, K, r, tmp, inv_err, norm_out);
 }
 
-/* As oracle_reject_ex with the ResiSpec budget chosen by z_rule (R1 / R7). */
-int oracle_reject_z(int mode, int z_rule, double* R, const double* q, int V, int x0,
+/* As oracle_reject_ex with the ResiSpec budget chosen by z_rule (R1 / R7)
+ * and the fill of step 3 by fill (0: R2, 1: R10). */
+int oracle_reject_z(int mode, int z_rule, int fill, double* R, const double* q, int V, int x0,
                     double* K, double* r, double* tmp, double* inv_err, double* norm_out) {
   if (norm_out) *norm_out = 1.0;
   if (mode == OR_MODE_SPECINFER) {
@@ -281,7 +339,7 @@ int oracle_reject_z(int mode, int z_rule, double* R, const double* q, int V, int
   }
   const double Z = oracle_budget(R, q, V, x0, z_rule);
   if (!(Z > 0.0)) return 0;
-  oracle_get_proxy_z(R, q, V, x0, Z, K, r);
+  oracle_get_proxy_z(R, q, V, x0, Z, fill, K, r);
   double e = 0.0;
   if (inv_err) {
     double sr = 0.0, sk = 0.0;
@@ -385,6 +443,8 @@ typedef struct {
                               (R9) into [B, N] (-1 elsewhere) instead of
                               reading cand */
   double* out_draft_margin; /* [B] smallest relative CDF margin of those draws */
+  int32_t fill;            /* ResiSpec fill of step 3: 0 capacity (R2), 1 level (R10) */
+  int32_t pad2_;
 } oracle_args;
 
 typedef struct {
@@ -497,7 +557,7 @@ static void verify_sequence(const oracle_args* a, int lb, int tree_bad,
       }
       rejects += 1;
       double norm = 1.0;
-      if (!oracle_reject_z(a->mode, a->z_rule, R, Dn, V, x, K, r, tmp, inv_ptr, &norm))
+      if (!oracle_reject_z(a->mode, a->z_rule, a->fill, R, Dn, V, x, K, r, tmp, inv_ptr, &norm))
         status |= OR_INFO_DEGENERATE;
       else if (Dn == Dbuf)
         memcpy(Dbuf, K, sizeof(double) * V);

@@ -120,17 +120,19 @@ def test_get_proxy_invariants():
             assert abs((k - p + r).sum() - Z) < 1e-13
 
 
-def test_theorem2_l1_closed_form():
+@pytest.mark.parametrize("fill", [0, 1])
+def test_theorem2_l1_closed_form(fill):
     """Theorem 2's proof: with capacity p (here p with p(x0) = 0, because
     GetProxy reserves nothing at x0) and budget Z, the smallest reachable
     L1(r/Z, q) is (2/Z) * sum max(0, Z q - p).  The residual of GetProxy must
-    reach it, i.e. mass is added only to tokens that are not bottlenecks."""
+    reach it, i.e. mass is added only to tokens that are not bottlenecks;
+    both fills (capacity, level lam >= Z) do."""
     rng = np.random.default_rng(2)
     for V in (3, 8, 50, 500):
         for _ in range(40):
             p, q = _random_case(rng, V)
             x0 = _rejectable(rng, p, q)
-            k, r, Z = oracle.get_proxy(p, q, x0)
+            k, r, Z = oracle.get_proxy(p, q, x0, fill=fill)
             Rp = r / Z
             pt = p.copy()
             pt[x0] = 0.0
@@ -186,15 +188,111 @@ def test_golden_v4_clipped():
     np.testing.assert_allclose(r2, g["r"], atol=1e-15)
 
 
-def test_binary_vocab_resispec_equals_specinfer():
+def test_golden_v4_level_fill():
+    """The level reading of GetProxy's step 3 on a hand-worked case where one
+    token saturates at its capacity before the level meets the budget."""
+    g = json.load(open(os.path.join(GOLDEN, "resispec_proxy_v4_level_fill.json")))
+    p, q = np.array(g["p"]), np.array(g["q"])
+    k, r, Z = oracle.get_proxy(p, q, g["x0"], fill=oracle.FILL_LEVEL)
+    assert Z == pytest.approx(g["Z"], abs=1e-15)
+    np.testing.assert_allclose(r, g["r"], atol=1e-15)
+    np.testing.assert_allclose(k, g["K"], atol=1e-15)
+    R2, changed, err = oracle.reject(oracle.MODE_RESISPEC, p, q, g["x0"], fill=oracle.FILL_LEVEL)
+    assert changed and err < 1e-14
+    np.testing.assert_allclose(R2, g["residual"], atol=1e-15)
+    assert abs(np.abs(R2 - q).sum() - g["l1_to_q"]) < 1e-14
+    assert en.level_by_bisection(p, q, g["x0"], g["Z"]) == pytest.approx(g["level"], rel=1e-14)
+    K2, r2, _ = en.proxy_resispec(p, q, g["x0"], fill=1)
+    np.testing.assert_allclose(r2, g["r"], atol=1e-14)
+    # the capacity fill differs on this input
+    assert np.abs(oracle.get_proxy(p, q, g["x0"])[1] - r).max() > 1e-2
+
+
+def test_level_fill_without_room_on_the_draft_support():
+    """When r = p on the support of q cannot hold Z, the rest goes to the
+    q = 0 tokens in proportion to p.  Hand-worked: p = (.1, .1, .1, .7),
+    q = (.6, .4, 0, 0), x0 = 0: Z = 0.5, token 1 saturates at 0.1, the
+    deficit 0.4 splits 1 : 7 over tokens 2 and 3."""
+    p = np.array([0.1, 0.1, 0.1, 0.7])
+    q = np.array([0.6, 0.4, 0.0, 0.0])
+    k, r, Z = oracle.get_proxy(p, q, 0, fill=oracle.FILL_LEVEL)
+    assert Z == pytest.approx(0.5, abs=1e-15)
+    np.testing.assert_allclose(r, [0.0, 0.1, 0.05, 0.35], atol=1e-15)
+    np.testing.assert_allclose(en.proxy_resispec(p, q, 0, fill=1)[1], r, atol=1e-15)
+
+
+def _level_case(rng, V):
+    """A rejectable case; a third of them with draft zeros."""
+    p, q = _random_case(rng, V)
+    if V > 3 and rng.random() < 0.33:
+        z = rng.choice(V, size=max(1, V // 4), replace=False)
+        q[z] = 0.0
+        q /= q.sum()
+    return p, q
+
+
+def test_level_fill_structure():
+    """fill = level: r = min(lam q, p) off x0 for one lam >= Z, sum r = Z,
+    with the invariants of Sec. 5.1 (0 <= r <= p, r(x0) = 0, sum K = 1,
+    K >= 0, K(x0) = q(x0)) and R' = r / Z."""
+    rng = np.random.default_rng(21)
+    seen = 0
+    for V in (2, 3, 5, 17, 64, 1000):
+        for _ in range(30):
+            p, q = _level_case(rng, V)
+            if not (q - p).max() > 0:
+                continue
+            x0 = _rejectable(rng, p, q)
+            k, r, Z = oracle.get_proxy(p, q, x0, fill=oracle.FILL_LEVEL)
+            assert abs(r.sum() - Z) < 1e-13
+            assert (r >= -1e-15).all() and (r <= p + 1e-15).all() and r[x0] == 0
+            assert abs(k.sum() - 1) < 1e-13 and (k >= -1e-15).all() and k[x0] == q[x0]
+            off = np.arange(V) != x0
+            if p[off & (q > 0)].sum() < Z:  # no finite level: q-support saturated
+                np.testing.assert_allclose(r[off & (q > 0)], p[off & (q > 0)], atol=1e-15)
+                continue
+            below = off & (q > 0) & (r < p - 1e-12)
+            assert (r[off & (q == 0)] == 0).all()
+            if below.any():
+                lam = r[below] / q[below]
+                assert lam.max() - lam.min() <= 1e-11 * lam.max()
+                lam = lam.mean()
+                assert lam >= Z * (1 - 1e-12)
+                sat = off & (q > 0) & ~below
+                assert (p[sat] <= lam * q[sat] * (1 + 1e-9) + 1e-15).all()
+                seen += 1
+            R2, changed, err = oracle.reject(oracle.MODE_RESISPEC, p, q, x0,
+                                             fill=oracle.FILL_LEVEL)
+            assert changed and err < 1e-12
+            np.testing.assert_allclose(R2 * Z, r, atol=1e-15)
+    assert seen > 100
+
+
+def test_level_fill_matches_bisection():
+    """The oracle's exact level (sorted ratios) against the enumerator's
+    bisection of lam -> sum min(lam q, p), an independent method."""
+    rng = np.random.default_rng(22)
+    for V in (3, 9, 50, 700):
+        for _ in range(25):
+            p, q = _level_case(rng, V)
+            if not (q - p).max() > 0:
+                continue
+            x0 = _rejectable(rng, p, q)
+            _, r, _ = oracle.get_proxy(p, q, x0, fill=oracle.FILL_LEVEL)
+            _, r2, _ = en.proxy_resispec(p, q, x0, fill=1)
+            np.testing.assert_allclose(r, r2, atol=1e-13)
+
+
+@pytest.mark.parametrize("fill", [0, 1])
+def test_binary_vocab_resispec_equals_specinfer(fill):
     """V = 2: the only token with capacity receives the whole budget, so the
     ResiSpec residual equals the SpecInfer residual (delta at the other
-    token)."""
+    token), whatever the fill."""
     rng = np.random.default_rng(5)
     for _ in range(50):
         p, q = _random_case(rng, 2)
         x0 = int(np.argmax(q - p))
-        Rr, _, _ = oracle.reject(oracle.MODE_RESISPEC, p, q, x0)
+        Rr, _, _ = oracle.reject(oracle.MODE_RESISPEC, p, q, x0, fill=fill)
         Rs, _, _ = oracle.reject(oracle.MODE_SPECINFER, p, q, x0)
         np.testing.assert_allclose(Rr, Rs, atol=1e-15)
         np.testing.assert_allclose(Rr, np.eye(2)[1 - x0], atol=1e-15)

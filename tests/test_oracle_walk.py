@@ -133,21 +133,24 @@ def _single_position_draws(seed, V, k, n, zt, zd, T=1.0):
     return target, draft, cand
 
 
-@pytest.mark.parametrize("mode", [oracle.MODE_SPECINFER, oracle.MODE_RESISPEC])
-def test_oracle_matches_enumerator_single_position(mode):
+@pytest.mark.parametrize("mode,fill", [(oracle.MODE_SPECINFER, 0), (oracle.MODE_RESISPEC, 0),
+                                       (oracle.MODE_RESISPEC, oracle.FILL_LEVEL)])
+def test_oracle_matches_enumerator_single_position(mode, fill):
     V, k, n = 8, 3, 400_000
     zt, zd = _pq(42, V, scale=1.5, rho=0.4)
     target, draft, cand = _single_position_draws(5, V, k, n, zt, zd)
     out = oracle.verify(target, draft, W.tree_single(k), cand, 1.0, seed=1234, mode=mode,
-                        seq_stride=0, check_invariants=True)
+                        seq_stride=0, check_invariants=True, fill=fill)
     assert (out["status"] & ~oracle.INFO_DEGENERATE == 0).all()
     assert out["inv_err"].max() < 1e-12
     y = out["tokens"][:, 0]          # first emitted token (accepted or residual)
     p = sp_softmax(zt.astype(np.float64))
     q = sp_softmax(zd.astype(np.float64))
-    dist, acc = en.single_position(p, q, k, mode)
+    dist, acc = en.single_position(p, q, k, mode, fill=fill)
     pv, nb = chisq_pvalue(np.bincount(y, minlength=V), dist)
     assert pv > 1e-4, (pv, nb)
+    if fill:  # a different law from the capacity fill's (close to it on this input)
+        assert 0.5 * np.abs(dist - en.single_position(p, q, k, mode)[0]).sum() > 1e-5
     # which candidate got accepted: enumerated per-position probabilities
     which = np.bincount(out["accept_len"] * 0 + np.where(out["accept_len"] > 0,
                                                          out["nodes"][:, 0], k), minlength=k + 1)
@@ -191,22 +194,23 @@ def test_oracle_resispec_million_draws_rejects_target():
     assert 0.5 * np.abs(dist - p).sum() > 1e-2
 
 
-@pytest.mark.parametrize("mode", [oracle.MODE_SPECINFER, oracle.MODE_RESISPEC])
-def test_oracle_tree_walk_matches_enumerator(mode):
+@pytest.mark.parametrize("mode,fill", [(oracle.MODE_SPECINFER, 0), (oracle.MODE_RESISPEC, 0),
+                                       (oracle.MODE_RESISPEC, oracle.FILL_LEVEL)])
+def test_oracle_tree_walk_matches_enumerator(mode, fill):
     """Two-level tree with path-consistent rows: the oracle's emitted
     (first, second) token pairs follow the enumerated joint law."""
     parents = W.tree_levels([2, 2])
     V, B, T = 4, 60_000, 1.0
     target, draft, cand, rows_z = W.make_path_inputs_np(21, parents, B, V, T,
                                                         scale=1.0, rho=0.5)
-    out = oracle.verify(target, draft, parents, cand, T, seed=5, mode=mode)
+    out = oracle.verify(target, draft, parents, cand, T, seed=5, mode=mode, fill=fill)
     assert (out["status"] & ~oracle.INFO_DEGENERATE == 0).all()
 
     def rows(path):
         zt, zd = rows_z(path)
         return sp_softmax(zt.astype(np.float64) / T), sp_softmax(zd.astype(np.float64) / T)
 
-    dist = en.tree_walk(parents, rows, mode)
+    dist = en.tree_walk(parents, rows, mode, fill=fill)
     keys = sorted(dist)
     index = {kk: i for i, kk in enumerate(keys)}
     counts = np.zeros(len(keys))
@@ -379,28 +383,29 @@ def test_random_trees_are_valid_and_candidates_come_from_parent_rows():
     np.testing.assert_array_equal(cand, trees + 1)
 
 
-def test_oracle_denominator_update_matches_enumerator():
+@pytest.mark.parametrize("fill", [0, 1])
+def test_oracle_denominator_update_matches_enumerator(fill):
     """Proxy-as-denominator variant (the test denominator becomes each
     rejection's proxy K): oracle draws against the independently enumerated
     law of the same rule, GetProxy invariants at every rejection, and the law
-    differs from Algorithm 1's."""
+    differs from Algorithm 1's.  Also with the level fill."""
     V, k, n = 8, 3, 400_000
     zt, zd = _pq(43, V, scale=1.5, rho=0.3)
     target, draft, cand = _single_position_draws(6, V, k, n, zt, zd)
     out = oracle.verify(target, draft, W.tree_single(k), cand, 1.0, seed=4321,
                         mode=oracle.MODE_RESISPEC, seq_stride=0, check_invariants=True,
-                        denom_update=True)
+                        denom_update=True, fill=fill)
     assert (out["status"] & ~oracle.INFO_DEGENERATE == 0).all()
     assert out["inv_err"].max() < 1e-12
     p = sp_softmax(zt.astype(np.float64))
     q = sp_softmax(zd.astype(np.float64))
-    dist, acc = en.single_position(p, q, k, oracle.MODE_RESISPEC, denom_update=True)
+    dist, acc = en.single_position(p, q, k, oracle.MODE_RESISPEC, denom_update=True, fill=fill)
     pv, nb = chisq_pvalue(np.bincount(out["tokens"][:, 0], minlength=V), dist)
     assert pv > 1e-4, (pv, nb)
     which = np.where(out["accept_len"] > 0, out["nodes"][:, 0], k)
     pv2, _ = chisq_pvalue(np.bincount(which, minlength=k + 1), np.append(acc, 1 - acc.sum()))
     assert pv2 > 1e-4
-    dist0, _ = en.single_position(p, q, k, oracle.MODE_RESISPEC)
+    dist0, _ = en.single_position(p, q, k, oracle.MODE_RESISPEC, fill=fill)
     assert np.abs(dist - dist0).max() > 1e-3
 
 

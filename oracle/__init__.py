@@ -83,6 +83,7 @@ class _Args(ctypes.Structure):
         ("z_rule", ctypes.c_int32), ("denom_update", ctypes.c_int32),
         ("draft_out", ctypes.c_void_p), ("out_draft_margin", ctypes.c_void_p),
         ("fill", ctypes.c_int32), ("pad2_", ctypes.c_int32),
+        ("out_dist_err", ctypes.c_void_p),
     ]
 
 
@@ -214,7 +215,7 @@ def sample(R, u: float):
 def verify(target, draft, parents, cand, temperature, seed, *, mode=MODE_RESISPEC,
            max_depth=None, seq_stride=None, seq_ids=None, nthreads=None,
            check_invariants=False, decide_fp64=False, want_dist=False, z_rule=0,
-           denom_update=False, draft_children=False, fill=0):
+           denom_update=False, draft_children=False, fill=0, want_dist_err=False):
     """Run the oracle walk.
 
     ``target``/``draft``: float32 arrays, or uint16 arrays holding bf16 bit
@@ -222,6 +223,9 @@ def verify(target, draft, parents, cand, temperature, seed, *, mode=MODE_RESISPE
     one set of rows across all B sequences, in which case ``cand`` gives B).
     ``parents``: int32 [N] (one tree for every sequence) or [B, N] (a tree
     per sequence); ``cand``: int32 [B, N].
+    ``want_dist_err``: also return "dist_err" [B, V], a first-order bound of
+    the error of an fp32 evaluation of "dist" for rows whose test
+    denominator is the proxy (``denom_update``; reading R11), 0 elsewhere.
     Returns a dict of numpy arrays.
     """
     lib = load()
@@ -267,6 +271,8 @@ def verify(target, draft, parents, cand, temperature, seed, *, mode=MODE_RESISPE
     }
     if want_dist:
         out["dist"] = np.zeros((B, V))
+    if want_dist_err:
+        out["dist_err"] = np.zeros((B, V))
     a = _Args()
     a.B, a.N, a.V, a.D = B, N, V, D
     a.dtype, a.mode = dtype, int(mode)
@@ -292,6 +298,7 @@ def verify(target, draft, parents, cand, temperature, seed, *, mode=MODE_RESISPE
     a.out_len = out["accept_len"].ctypes.data
     a.out_nodes = out["nodes"].ctypes.data
     a.out_dist = out["dist"].ctypes.data if want_dist else None
+    a.out_dist_err = out["dist_err"].ctypes.data if want_dist_err else None
     a.out_accept_margin = out["accept_margin"].ctypes.data
     a.out_sample_margin = out["sample_margin"].ctypes.data
     a.out_status = out["status"].ctypes.data

@@ -70,6 +70,17 @@
  *       p_i / q_i, so lam is found exactly on the sorted ratios.  If even
  *       r = p on the support of q leaves a deficit, the tokens with q = 0
  *       (other than x0) take it in proportion to p, the rule of R2.
+ *   R11 tolerance of the proxy-denominator chain (R8): the proxy K = R - r
+ *       is a difference that cancels on tokens just below the level, and a
+ *       later rejection may divide it by a small budget, so an fp32
+ *       evaluation of the chain can be far from the fp64 one on a few
+ *       tokens.  For such rows the oracle also returns a first-order forward
+ *       error bound per token of the final distribution (out_dist_err): the
+ *       absolute errors of R and D are carried through every rejection
+ *       (min, R - m, r = m + mu t, K, the budget Z = D(x0) - R(x0), the
+ *       level's response to Z and the normaliser), starting from the
+ *       rounding of fp32 tempered softmax values; it is test infrastructure
+ *       that widens the parity tolerance only where the arithmetic does.
  *   R6  the accept decision is taken in fp32, the kernel's precision
  *       (u * q(x) < R(x) with both operands rounded to fp32); the margin
  *       |u - R/q| is reported in fp64 for near-tie accounting.
@@ -250,11 +261,14 @@ static double lambda_level(const double* p, const double* q, int V, int x0, doub
   return lam;
 }
 
-/* GetProxy with the budget Z and the fill rule given (steps 2-4 below). */
-double oracle_get_proxy_z(const double* p, const double* q, int V, int x0, double Z, int fill,
-                          double* k, double* r) {
+/* GetProxy with the budget Z and the fill rule given (steps 2-4 below);
+ * *level_out / *mu_out (optional) receive the level of step 2 (INFINITY: the
+ * support of q saturated) and the fraction of the capacity filled in step 3. */
+static double get_proxy_full(const double* p, const double* q, int V, int x0, double Z, int fill,
+                             double* k, double* r, double* level_out, double* mu_out) {
   double* rr = r ? r : (double*)malloc(sizeof(double) * (size_t)V);
   const double level = fill == 1 ? lambda_level(p, q, V, x0, Z) : Z;
+  double mu = 0.0;
   double sum_r = 0.0;
   for (int i = 0; i < V; ++i) {
     /* step 2 at the level Z (R2), or at the level that meets Z (R10); with
@@ -270,6 +284,7 @@ double oracle_get_proxy_z(const double* p, const double* q, int V, int x0, doubl
   /* the capacity fill (R2; for R10 only the deficit that the level cannot
      meet, which leaves capacity on q = 0 tokens alone) */
   if (sum_cap > 0.0 && (fill != 1 || level == INFINITY)) {
+    mu = delta / sum_cap;
     for (int i = 0; i < V; ++i)
       if (i != x0) rr[i] += delta * (p[i] - rr[i]) / sum_cap;
   }
@@ -278,7 +293,14 @@ double oracle_get_proxy_z(const double* p, const double* q, int V, int x0, doubl
     k[x0] = q[x0];
   }
   if (!r) free(rr);
+  if (level_out) *level_out = level;
+  if (mu_out) *mu_out = mu;
   return Z;
+}
+
+double oracle_get_proxy_z(const double* p, const double* q, int V, int x0, double Z, int fill,
+                          double* k, double* r) {
+  return get_proxy_full(p, q, V, x0, Z, fill, k, r, NULL, NULL);
 }
 
 /* R <- norm(max(R - K, 0)).  Returns the normaliser (0: R left unchanged). */
@@ -318,10 +340,21 @@ int oracle_reject_ex(int mode, double* R, const double* q, int V, int x0,
   return oracle_reject_z(mode, 0, 0, R, q, V, x0, K, r, tmp, inv_err, norm_out);
 }
 
+static int reject_full(int mode, int z_rule, int fill, double* R, const double* q, int V, int x0,
+                       double* K, double* r, double* tmp, double* inv_err, double* norm_out,
+                       double* Z_out, double* level_out, double* mu_out);
+
 /* As oracle_reject_ex with the ResiSpec budget chosen by z_rule (R1 / R7)
  * and the fill of step 3 by fill (0: R2, 1: R10). */
 int oracle_reject_z(int mode, int z_rule, int fill, double* R, const double* q, int V, int x0,
                     double* K, double* r, double* tmp, double* inv_err, double* norm_out) {
+  return reject_full(mode, z_rule, fill, R, q, V, x0, K, r, tmp, inv_err, norm_out, NULL, NULL,
+                     NULL);
+}
+
+static int reject_full(int mode, int z_rule, int fill, double* R, const double* q, int V, int x0,
+                       double* K, double* r, double* tmp, double* inv_err, double* norm_out,
+                       double* Z_out, double* level_out, double* mu_out) {
   if (norm_out) *norm_out = 1.0;
   if (mode == OR_MODE_SPECINFER) {
     double changed = residual_from(R, q, V, tmp);
@@ -338,8 +371,9 @@ int oracle_reject_z(int mode, int z_rule, int fill, double* R, const double* q, 
     return changed > 0.0;
   }
   const double Z = oracle_budget(R, q, V, x0, z_rule);
+  if (Z_out) *Z_out = Z;
   if (!(Z > 0.0)) return 0;
-  oracle_get_proxy_z(R, q, V, x0, Z, fill, K, r);
+  get_proxy_full(R, q, V, x0, Z, fill, K, r, level_out, mu_out);
   double e = 0.0;
   if (inv_err) {
     double sr = 0.0, sk = 0.0;
@@ -404,6 +438,86 @@ int oracle_sample(const double* R, int V, double u, double* margin) {
 }
 
 /* ------------------------------------------------------------------ */
+/* First-order absolute error bounds of an fp32 evaluation (R11).  Units:
+ * probabilities; EPS is fp32's unit roundoff. */
+static const double ERR_EPS = 5.9604644775390625e-08; /* 2^-24 */
+
+/* Rounding of an fp32 tempered softmax value 2^a / S, a = log2(v / max v):
+ * the exponent's argument is rounded relative to |a|, plus a few roundings
+ * of the exponential and the normaliser. */
+static void err_init(const double* v, int V, double* e) {
+  double mx = 0.0;
+  for (int i = 0; i < V; ++i)
+    if (v[i] > mx) mx = v[i];
+  for (int i = 0; i < V; ++i)
+    e[i] = v[i] > 0.0 ? v[i] * ERR_EPS * (4.0 + 0.7 * fabs(log2(v[i] / mx))) : 0.0;
+}
+
+/* Bounds of m = min(level D, R) and t = R - m at one token (R > 0, not x0). */
+static void err_min(double R, double D, double eR, double eD, double level, double* m,
+                    double* em, double* t, double* et) {
+  const double lD = level == INFINITY ? (D > 0.0 ? INFINITY : 0.0) : level * D;
+  const double le = level == INFINITY ? 0.0 : level * eD;
+  *m = fmin(lD, R);
+  if (fabs(R - lD) <= eR + le + ERR_EPS * R)
+    *em = fmax(eR, le) + ERR_EPS * R; /* either side of the min */
+  else
+    *em = (lD < R) ? le + ERR_EPS * *m : eR;
+  *t = R - *m;
+  *et = eR + *em + ERR_EPS * *t;
+}
+
+/* Carries the bounds (eR, eD) of R and D through one ResiSpec rejection of
+ * x0 (R, D before; r, K after; budget Z, level, fill fraction mu) and leaves
+ * the bounds of R' = r / sum r and D' = K in (eR, eD). */
+static void err_reject(const double* R, const double* D, const double* r, const double* K, int V,
+                       int x0, double Z, double level, double mu, double* eR, double* eD) {
+  double S = 0.0, slope = 0.0, sum_t = 0.0, sum_em = 0.0, sum_et = 0.0;
+  for (int i = 0; i < V; ++i) {
+    S += r[i];
+    if (i == x0 || R[i] == 0.0) continue;
+    double m, em, t, et;
+    err_min(R[i], D[i], eR[i], eD[i], level, &m, &em, &t, &et);
+    sum_t += t;
+    sum_em += em;
+    sum_et += et;
+    if (level != INFINITY && level * D[i] < R[i]) slope += D[i];
+  }
+  if (!(S > 0.0)) return;
+  const double eZ = eD[x0] + eR[x0] + ERR_EPS * Z;
+  /* mu = (Z - sum m) / sum t: its numerator may cancel */
+  const double emu = mu > 0.0 && sum_t > 0.0
+                         ? (eZ + sum_em + ERR_EPS * Z) / sum_t + mu * sum_et / sum_t
+                         : 0.0;
+  double er_sum = 0.0;
+  for (int i = 0; i < V; ++i) {
+    double er, eK;
+    if (i == x0 || R[i] == 0.0) {
+      er = 0.0; /* taken out exactly; a rejected token stays at 0 */
+      eK = (i == x0) ? eD[i] : 0.0;
+    } else {
+      double m, em, t, et;
+      err_min(R[i], D[i], eR[i], eD[i], level, &m, &em, &t, &et);
+      er = em + mu * et + emu * t + ERR_EPS * r[i];
+      eK = (1.0 - mu) * et + emu * t + ERR_EPS * K[i];
+    }
+    eR[i] = er; /* bound of r for now */
+    eD[i] = eK;
+    er_sum += er;
+  }
+  /* the level's response to an error in Z moves the tokens below it
+     together: relative dZ / (mass below the level) on them, dZ / Z on all */
+  const double below = (level == INFINITY) ? 0.0 : level * slope;
+  for (int i = 0; i < V; ++i) {
+    const double Rn = r[i] / S;
+    double e = eR[i] / S + Rn * (er_sum / S + eZ / Z);
+    if (i != x0 && R[i] > 0.0 && below > 0.0 && level != INFINITY && level * D[i] < R[i])
+      e += Rn * eZ / below;
+    eR[i] = e;
+  }
+}
+
+/* ------------------------------------------------------------------ */
 typedef struct {
   int32_t B, N, V, D;
   int32_t dtype;
@@ -445,6 +559,8 @@ typedef struct {
   double* out_draft_margin; /* [B] smallest relative CDF margin of those draws */
   int32_t fill;            /* ResiSpec fill of step 3: 0 capacity (R2), 1 level (R10) */
   int32_t pad2_;
+  double* out_dist_err;    /* [B, V] forward error bound of out_dist for rows with
+                              the proxy denominator (R11); 0 elsewhere */
 } oracle_args;
 
 typedef struct {
@@ -463,7 +579,7 @@ static int tree_is_bad(const int32_t* parents, int N) {
 static void verify_sequence(const oracle_args* a, int lb, int tree_bad,
                             double* z, double* p, double* q, double* R,
                             double* K, double* r, double* tmp, double* Dbuf,
-                            int32_t* kids) {
+                            double* eR, double* eD, double* Rb, int32_t* kids) {
   const int V = a->V, N = a->N, D = a->D;
   const int32_t* parents = a->parents + (size_t)(a->parents_stride * lb);
   if (a->parents_stride) tree_bad = tree_is_bad(parents, N);
@@ -508,6 +624,7 @@ static void verify_sequence(const oracle_args* a, int lb, int tree_bad,
       int y = oracle_sample(p, V, u, &smargin);
       if (toks) toks[depth] = y;
       if (a->out_dist) memcpy(a->out_dist + (size_t)lb * V, p, sizeof(double) * V);
+      if (a->out_dist_err) memset(a->out_dist_err + (size_t)lb * V, 0, sizeof(double) * V);
       break;
     }
     load_row(a->draft, a->dtype, seq_off + (size_t)row * V, V, z);
@@ -528,6 +645,11 @@ static void verify_sequence(const oracle_args* a, int lb, int tree_bad,
     if (a->denom_update && a->mode == OR_MODE_RESISPEC) {
       memcpy(Dbuf, q, sizeof(double) * V);
       Dn = Dbuf;                      /* becomes each rejection's proxy (R8) */
+    }
+    const int track = a->out_dist_err != NULL && Dn == Dbuf; /* R11 */
+    if (track) {
+      err_init(p, V, eR);
+      err_init(q, V, eD);
     }
     cond = 1.0;
     int accepted = -1;
@@ -556,11 +678,15 @@ static void verify_sequence(const oracle_args* a, int lb, int tree_bad,
         break;
       }
       rejects += 1;
-      double norm = 1.0;
-      if (!oracle_reject_z(a->mode, a->z_rule, a->fill, R, Dn, V, x, K, r, tmp, inv_ptr, &norm))
+      double norm = 1.0, Zj = 0.0, level = 0.0, mu = 0.0;
+      if (track) memcpy(Rb, R, sizeof(double) * V);
+      if (!reject_full(a->mode, a->z_rule, a->fill, R, Dn, V, x, K, r, tmp, inv_ptr, &norm, &Zj,
+                       &level, &mu)) {
         status |= OR_INFO_DEGENERATE;
-      else if (Dn == Dbuf)
+      } else if (Dn == Dbuf) {
+        if (track) err_reject(Rb, Dbuf, r, K, V, x, Zj, level, mu, eR, eD);
         memcpy(Dbuf, K, sizeof(double) * V);
+      }
       cond /= norm;
     }
     if (accepted < 0) {
@@ -568,6 +694,12 @@ static void verify_sequence(const oracle_args* a, int lb, int tree_bad,
       int y = oracle_sample(R, V, u, &smargin);
       if (toks) toks[depth] = y;
       if (a->out_dist) memcpy(a->out_dist + (size_t)lb * V, R, sizeof(double) * V);
+      if (a->out_dist_err) {
+        if (track)
+          memcpy(a->out_dist_err + (size_t)lb * V, eR, sizeof(double) * V);
+        else
+          memset(a->out_dist_err + (size_t)lb * V, 0, sizeof(double) * V);
+      }
       break;
     }
     if (depth >= D) {
@@ -603,11 +735,12 @@ static void* worker(void* arg) {
   worker_ctx* w = (worker_ctx*)arg;
   const oracle_args* a = w->a;
   size_t V = (size_t)(a->V > 0 ? a->V : 1);
-  double* buf = (double*)malloc(sizeof(double) * V * 8);
+  double* buf = (double*)malloc(sizeof(double) * V * 11);
   int32_t* kids = (int32_t*)malloc(sizeof(int32_t) * (size_t)(a->N > 0 ? a->N : 1));
   for (int lb = w->tid; lb < a->B; lb += w->nthreads)
     verify_sequence(a, lb, w->tree_bad, buf, buf + V, buf + 2 * V, buf + 3 * V,
-                    buf + 4 * V, buf + 5 * V, buf + 6 * V, buf + 7 * V, kids);
+                    buf + 4 * V, buf + 5 * V, buf + 6 * V, buf + 7 * V, buf + 8 * V,
+                    buf + 9 * V, buf + 10 * V, kids);
   free(kids);
   free(buf);
   return NULL;

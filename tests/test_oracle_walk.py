@@ -447,3 +447,98 @@ def test_oracle_drafted_candidates_follow_q():
     # an accepted candidate is emitted as drafted
     acc = out["accept_len"] >= 1
     np.testing.assert_array_equal(out["tokens"][acc, 0], d[acc, out["nodes"][acc, 0]])
+
+
+# ------------------------------------------------------------ fp32 error bound of proxy chains
+
+
+def _fp32_softmax(z, T):
+    """Tempered softmax as an fp32 evaluation: a = fp32(z c - M) (one
+    rounding, as a fused multiply-add), 2^a in fp32, fp32 sum and divide."""
+    c = np.float32(1.4426950408889634 / np.float32(T))
+    z = z.astype(np.float32)
+    M = np.float32(z.max() * c)
+    a = (z.astype(np.float64) * np.float64(c) - np.float64(M)).astype(np.float32)
+    e = np.exp2(a).astype(np.float32)
+    return (e / e.sum(dtype=np.float32)).astype(np.float32)
+
+
+def _fp32_proxy_chain(zt, zd, xs, fill):
+    """The proxy-denominator chain of rejections of xs in fp32 arithmetic:
+    the level is solved exactly on the fp32 values, every elementwise step
+    is rounded to fp32."""
+    f = np.float32
+    R, D = _fp32_softmax(zt, 1.0), _fp32_softmax(zd, 1.0)
+    rejected = []
+    for x0 in xs:
+        Z = f(D[x0] - R[x0])
+        if not Z > 0:
+            continue
+        off = np.ones(R.size, bool)
+        off[x0] = False
+        off[rejected] = False
+        R64, D64 = R.astype(np.float64), D.astype(np.float64)
+        lam = Z
+        if fill:
+            lam = en.level_by_bisection(np.where(off, R64, 0.0), D64, x0, float(Z))
+        if np.isfinite(lam):
+            m = np.minimum((f(lam) * D).astype(f), R)
+        else:
+            m = np.where(D > 0, R, f(0))
+        m = np.where(off, m, f(0))
+        t = np.where(off, (R - m).astype(f), f(0))
+        mu = f(0)
+        if not fill or not np.isfinite(lam):
+            mu = f(min(max((Z - m.sum(dtype=f)) / t.sum(dtype=f), 0), 1)) if t.sum() > 0 else f(0)
+        r = (m + mu * t).astype(f)
+        K = ((f(1) - mu) * t).astype(f)
+        K[x0] = D[x0]       # K = R - r = 0 at the earlier rejected tokens
+        R = (r / r.sum(dtype=f)).astype(f)
+        D = K
+        rejected.append(x0)
+    return R.astype(np.float64)
+
+
+@pytest.mark.parametrize("fill", [0, 1])
+def test_proxy_chain_error_bound_covers_fp32(fill):
+    """Reading R11: the oracle's per-token error bound of a proxy-denominator
+    row covers an fp32 evaluation of the same rejections, token by token,
+    on rows built to put tokens next to the level (R close to lam D), where
+    the proxy K = R - r cancels."""
+    rng = np.random.default_rng(31 + fill)
+    V, k = 1500, 4
+    worst_ratio, rows = 0.0, 0
+    for trial in range(40):
+        zt = rng.normal(0, 2.0, V).astype(np.float32)
+        zd = (0.7 * zt + 0.7 * rng.normal(0, 2.0, V)).astype(np.float32)
+        xs = list(rng.choice(V, size=k, p=sp_softmax(zd.astype(np.float64))))
+        if trial % 3 == 0:
+            xs[1] = xs[0]   # a duplicate rejection
+        zt[xs] = -np.inf    # candidates the target excludes: every test rejects
+        cand = np.asarray([xs], np.int32)
+        target = np.broadcast_to(zt, (k + 1, V)).copy()
+        draft = np.broadcast_to(zd, (k + 1, V)).copy()
+        o = oracle.verify(target, draft, W.tree_single(k), cand, 1.0, 5, seq_stride=0,
+                          want_dist=True, denom_update=True, fill=fill, want_dist_err=True,
+                          decide_fp64=True)
+        if o["accept_len"][0] != 0 or o["rejects"][0] != k:
+            continue
+        g = _fp32_proxy_chain(zt, zd, xs, fill)
+        diff = np.abs(g - o["dist"][0])
+        bound = o["dist_err"][0]
+        assert (diff <= bound + 1e-12).all(), (trial, diff.max(), bound[np.argmax(diff - bound)])
+        worst_ratio = max(worst_ratio, (diff / np.maximum(bound, 1e-300)).max())
+        rows += 1
+    assert rows >= 30
+    assert worst_ratio > 1e-2   # the bound is not vacuous on these rows
+
+
+def test_dist_err_is_zero_without_the_proxy_denominator():
+    V, k = 300, 3
+    rng = np.random.default_rng(4)
+    zt = rng.normal(0, 2, (k + 1, V)).astype(np.float32)
+    zd = rng.normal(0, 2, (k + 1, V)).astype(np.float32)
+    cand = rng.integers(0, V, (8, k)).astype(np.int32)
+    o = oracle.verify(zt, zd, W.tree_single(k), cand, 1.0, 5, seq_stride=0, want_dist=True,
+                      fill=1, want_dist_err=True)
+    assert (o["dist_err"] == 0).all()

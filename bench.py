@@ -54,6 +54,9 @@ def parse_args(argv=None):
                     help="ResiSpec budget: Algorithm 1's gap, or the Z_applied heuristic")
     ap.add_argument("--proxy-denominator", action="store_true",
                     help="ResiSpec variant: each rejection's proxy becomes the test denominator")
+    ap.add_argument("--fill", choices=["capacity", "level"], default="capacity",
+                    help="ResiSpec variant of GetProxy's deficit fill: in proportion to the "
+                         "capacity (default) or the draft raised to a level")
     ap.add_argument("--draft", action="store_true",
                     help="drafting mode: the kernel draws the visited nodes' children from q")
     ap.add_argument("--pool", type=int, default=0, help="input sets rotated between steps (0 = auto)")
@@ -195,18 +198,26 @@ def rows_visited(nodes, accept_len, haschild):
     return rows
 
 
-def cpu_oracle_rate(w, target_h, draft_h, parents, cand_h, seq_ids, mode, seconds, seed0):
+def oracle_variant(args) -> dict:
+    """The oracle's switches for the verification rule the run measures."""
+    return dict(z_rule=1 if args.z_rule == "applied" else 0, denom_update=args.proxy_denominator,
+                fill=1 if args.fill == "level" else 0, draft_children=args.draft)
+
+
+def cpu_oracle_rate(w, target_h, draft_h, parents, cand_h, seq_ids, mode, seconds, seed0,
+                    variant=None):
     """Time the fp64 oracle as it stands on this host's cores over a bounded
     sample; returns (nodes/s, threads, sample description)."""
     import oracle
+    variant = variant or {}
     S = cand_h.shape[0]
     threads = min(os.cpu_count() or 1, S)
     oracle.verify(target_h[:1], draft_h[:1], parents, cand_h[:1], w.temperature, seed0,
-                  mode=mode, max_depth=w.max_depth, seq_ids=seq_ids[:1], nthreads=1)
+                  mode=mode, max_depth=w.max_depth, seq_ids=seq_ids[:1], nthreads=1, **variant)
     reps, t0 = 0, time.perf_counter()
     while True:
         oracle.verify(target_h, draft_h, parents, cand_h, w.temperature, seed0 + reps, mode=mode,
-                      max_depth=w.max_depth, seq_ids=seq_ids, nthreads=threads)
+                      max_depth=w.max_depth, seq_ids=seq_ids, nthreads=threads, **variant)
         reps += 1
         el = time.perf_counter() - t0
         if el >= seconds or reps >= 200:
@@ -292,7 +303,7 @@ def run_reference(args):
     def step(i):
         oracle.verify(inp["target"], inp["draft"], inp["parents"], inp["cand"], w.temperature,
                       args.seed + i, mode=mode, max_depth=w.max_depth, seq_ids=seq_ids,
-                      nthreads=threads)
+                      nthreads=threads, **oracle_variant(args))
 
     for i in range(max(0, args.warmup)):
         step(i)
@@ -357,14 +368,15 @@ def run_ours(args):
     status = torch.zeros((1,), dtype=torch.int32, device=dev)
     kernel = None if args.kernel == "auto" else args.kernel
     z_rule = rs.Z_RULE_APPLIED if args.z_rule == "applied" else rs.Z_RULE_ALG1
+    fill = rs.FILL_LEVEL if args.fill == "level" else rs.FILL_CAPACITY
     kw = dict(max_depth=D, mode=mode, cluster_size=args.cluster_size,
               block_threads=args.block_threads, status=status, kernel=kernel, z_rule=z_rule,
-              proxy_denominator=args.proxy_denominator)
+              proxy_denominator=args.proxy_denominator, fill=fill)
     stream = torch.cuda.current_stream(dev)
     plan = rs.plan(B, N, V, D, w.dtype, cluster_size=args.cluster_size,
                    block_threads=args.block_threads,
                    kernel="stream" if (args.draft and kernel is None) else kernel,
-                   z_rule=z_rule, proxy_denominator=args.proxy_denominator)
+                   z_rule=z_rule, proxy_denominator=args.proxy_denominator, fill=fill)
 
     drafted = torch.empty((B, N), dtype=torch.int32, device=dev) if args.draft else None
 
@@ -420,7 +432,7 @@ def run_ours(args):
             "tree": list(w.tree[1]) if w.tree[0] == "levels" else list(w.tree[1:]),
             "logits": f"{w.gen} slope {w.slope} scale {w.scale} rho {w.rho}",
             "temperature": w.temperature, "mode": args.mode, "z_rule": args.z_rule,
-            "proxy_denominator": args.proxy_denominator, "draft": args.draft,
+            "proxy_denominator": args.proxy_denominator, "fill": args.fill, "draft": args.draft,
             "parallelism": f"replicas{world}" if world > 1 else "single",
             "launch": {k: plan[k] for k in ("kernel_name", "cluster_size", "block_threads",
                                             "smem_bytes", "slice_elems", "uses_tma",
@@ -462,7 +474,7 @@ def run_ours(args):
             rs.verify(dbuf["target"], dbuf["draft"], dbuf["parents"], dbuf["cand"],
                       w.temperature, args.seed + i, out_tokens=d_tok, out_accept_len=d_len,
                       max_depth=D, mode=mode, stream=stream, kernel=kernel, z_rule=z_rule,
-                      proxy_denominator=args.proxy_denominator)
+                      proxy_denominator=args.proxy_denominator, fill=fill)
             h_tok.copy_(d_tok, non_blocking=True)
             h_len.copy_(d_len, non_blocking=True)
 
@@ -513,7 +525,7 @@ def _finish_cpu(result, args, sets, w, mode, world, dev):
     pa = s0["parents_np"][:S] if w.per_sequence_tree else s0["parents_np"]
     rate, threads, sample = cpu_oracle_rate(w, th, dh, pa, ch,
                                             np.arange(S, dtype=np.int32), omode,
-                                            args.cpu_seconds, args.seed)
+                                            args.cpu_seconds, args.seed, oracle_variant(args))
     result["cpu_baseline"] = {"value": rate, "unit": "nodes/s", "cores": threads,
                               "kind": "oracle", "sample": sample}
     return result

@@ -116,6 +116,23 @@ typedef struct {
                                       q; candidates stay draws from q.  Streaming
                                       kernel only (with RESISPEC_FLAG_RESIDENT:
                                       RESISPEC_E_ARG); no effect in SPECINFER mode */
+#define RESISPEC_FLAG_LEVEL_FILL 64 /* RESISPEC mode variant of GetProxy's step 3
+                                      (Algorithm 1; the paper fixes only that the
+                                      deficit goes to tokens below their capacity):
+                                      r = min(lam q, R) off x0 with the level lam
+                                      at which sum r = Z, instead of the default
+                                      fill in proportion to the capacity R - r.
+                                      lam is found by Newton steps from lam = Z on
+                                      the concave, piecewise linear sum (one more
+                                      pass over the rows per step, typically 2 to
+                                      6 steps); the residual is normalised by the
+                                      mass reached (a deficit left below 2^-22 Z
+                                      acts as a relative rounding).  When the
+                                      support of q cannot hold Z (no level
+                                      exists) that support is saturated and the
+                                      default rule places the rest.  Streaming
+                                      kernel only (with RESISPEC_FLAG_RESIDENT:
+                                      RESISPEC_E_ARG); no effect in SPECINFER mode */
 
 /* Kernels.  Both compute the same verification; they differ in where a
  * visited node's rows live between the passes of a visit.

@@ -39,8 +39,11 @@ FLAG_RESIDENT = 4
 FLAG_STREAM = 8
 FLAG_Z_APPLIED = 16
 FLAG_PROXY_DENOM = 32
+FLAG_LEVEL_FILL = 64
 Z_RULE_ALG1 = 0       # ResiSpec budget Z = q(x0) - R(x0) (Algorithm 1)
 Z_RULE_APPLIED = 1    # Z = max(Z*, |gap|) clamped to 1 - R(x0) (Sec. 5.3 heuristic)
+FILL_CAPACITY = 0     # GetProxy's deficit in proportion to the capacity R - r (default)
+FILL_LEVEL = 1        # r = min(lam q, R) at the level lam that meets the budget
 PHASES = ("setup", "norm", "norm_exchange", "test", "reject", "draw")
 KERNEL_RESIDENT = 0
 KERNEL_STREAM = 1
@@ -175,7 +178,7 @@ def _kernel_flags(kernel) -> int:
 def make_opts(mode=MODE_RESISPEC, cluster_size=0, block_threads=0, no_tma=False,
               seq_stride=None, status=None, out_nodes=None, out_dist=None,
               out_rejects=None, prefetch=False, kernel=None, z_rule=Z_RULE_ALG1,
-              proxy_denominator=False) -> Opts:
+              proxy_denominator=False, fill=FILL_CAPACITY) -> Opts:
     lib = load_library()
     o = Opts()
     lib.resispec_opts_default(ctypes.byref(o))
@@ -184,7 +187,8 @@ def make_opts(mode=MODE_RESISPEC, cluster_size=0, block_threads=0, no_tma=False,
     o.block_threads = int(block_threads)
     o.flags = ((FLAG_NO_TMA if no_tma else 0) | (FLAG_PREFETCH if prefetch else 0)
                | _kernel_flags(kernel) | (FLAG_Z_APPLIED if z_rule == Z_RULE_APPLIED else 0)
-               | (FLAG_PROXY_DENOM if proxy_denominator else 0))
+               | (FLAG_PROXY_DENOM if proxy_denominator else 0)
+               | (FLAG_LEVEL_FILL if fill == FILL_LEVEL else 0))
     o.seq_stride = -1 if seq_stride is None else int(seq_stride)
     o.status = None if status is None else status.data_ptr()
     o.out_nodes = None if out_nodes is None else out_nodes.data_ptr()
@@ -213,7 +217,7 @@ def verify(target, draft, tree_parents, cand_tokens, temperature, seed, *, max_d
            out_dist=None, out_rejects=None, status=None, cluster_size=0, block_threads=0,
            no_tma=False, seq_stride=None, stream=None, prefetch=False, kernel=None,
            z_rule=Z_RULE_ALG1, proxy_denominator=False, out_phase=None,
-           out_candidates=None):
+           out_candidates=None, fill=FILL_CAPACITY):
     """Verify a batch of draft trees on the GPU.
 
     target, draft: CUDA tensors [B, N+1, V] (float32 or bfloat16); with
@@ -227,6 +231,9 @@ def verify(target, draft, tree_parents, cand_tokens, temperature, seed, *, max_d
     ``proxy_denominator``: after each ResiSpec rejection the accept tests
     and the next GetProxy use that rejection's proxy in place of q (the
     paper's EAGLE integration; streaming kernel).
+    ``fill``: how GetProxy fills the deficit, FILL_CAPACITY (in proportion to
+    the remaining capacity) or FILL_LEVEL (the draft raised to the level
+    that meets the budget; streaming kernel).
     ``out_phase``: optional int64 CUDA tensor [B, len(PHASES)] receiving the
     SM cycles each sequence spent per phase (selects the streaming kernel).
     ``out_candidates``: drafting mode, an int32 CUDA tensor [B, N] that
@@ -271,7 +278,7 @@ def verify(target, draft, tree_parents, cand_tokens, temperature, seed, *, max_d
     if seq_stride is None and target.numel() != B * (N + 1) * V:
         raise ValueError("target must be [B, N+1, V] (or pass seq_stride)")
     o = make_opts(mode, cluster_size, block_threads, no_tma, seq_stride, status, out_nodes,
-                  out_dist, out_rejects, prefetch, kernel, z_rule, proxy_denominator)
+                  out_dist, out_rejects, prefetch, kernel, z_rule, proxy_denominator, fill)
     o.parents_stride = N if per_seq_tree else 0
     if out_phase is not None:
         _need_cuda("out_phase", out_phase)

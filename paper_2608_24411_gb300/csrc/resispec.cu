@@ -269,7 +269,8 @@ int make_plan(const resispec_dims& d, const resispec_opts& o, int dev, int sms,
   if (o.seq_stride < -1) return RESISPEC_E_ARG;
   if (o.parents_stride < 0) return RESISPEC_E_ARG;
   const bool force_res = (o.flags & RESISPEC_FLAG_RESIDENT) != 0;
-  const bool variant = (o.flags & (RESISPEC_FLAG_Z_APPLIED | RESISPEC_FLAG_PROXY_DENOM)) != 0 ||
+  const bool variant = (o.flags & (RESISPEC_FLAG_Z_APPLIED | RESISPEC_FLAG_PROXY_DENOM |
+                                   RESISPEC_FLAG_LEVEL_FILL)) != 0 ||
                        o.out_phase_cycles != nullptr || o.out_candidates != nullptr;
   const bool force_str = (o.flags & RESISPEC_FLAG_STREAM) != 0 || variant;
   if (force_res && force_str) return RESISPEC_E_ARG;
@@ -457,6 +458,7 @@ int resispec_verify_ex(const void* target_logits, const void* draft_logits,
   prm.prefetch = (o.flags & RESISPEC_FLAG_PREFETCH) != 0;
   prm.z_applied = (o.flags & RESISPEC_FLAG_Z_APPLIED) != 0;
   prm.denom_update = (o.flags & RESISPEC_FLAG_PROXY_DENOM) != 0;
+  prm.level_fill = (o.flags & RESISPEC_FLAG_LEVEL_FILL) != 0;
 
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   cudaError_t e;

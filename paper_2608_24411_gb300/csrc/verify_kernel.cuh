@@ -84,6 +84,7 @@ struct VerifyParams {
   int32_t prefetch;    // L2 prefetch of the first child's rows
   int32_t z_applied;   // ResiSpec budget max(Z*, gap) clamped to 1 - R(x0) (streaming kernel)
   int32_t denom_update;  // ResiSpec: each rejection's proxy becomes the test denominator (streaming)
+  int32_t level_fill;  // ResiSpec: GetProxy's deficit raises the draft to a level (streaming)
 };
 
 struct __align__(16) Slot {
@@ -189,13 +190,14 @@ __device__ __forceinline__ bool wait_bar(uint32_t bar, uint32_t parity) {
 // received partials.  Every CTA combines identical partials in identical
 // lanes, so all CTAs obtain the same bits.
 //   NORM: (a0, a1) and (a2, a3) are (reference, scaled sum) pairs of the
-//         target and draft rows; SUM: a0, a1 are sums (a2, a3 unused).
+//         target and draft rows; SUM: a0, a1 are sums, and a2, a3 too when
+//         NSUM = 4 (otherwise they are unused).
 //   H.pubv holds the values published by the owner thread of a token; every
 //   CTA reads them from the slot of the owner CTA `owner` (-1: none).
 //   flags are OR-ed; `mn` is min-reduced over the cluster's CTAs (each CTA
 //   passes its own value; the result is left in H.bc[9]).
 // out[0..3]: reduced partials, out[4..7]: published values.
-template <int NWARPS, bool NORM>
+template <int NWARPS, bool NORM, int NSUM = 2>
 __device__ __forceinline__ void exchange(Head& H, float a0, float a1, float a2, float a3,
                                          int flags, int owner, int& xp, uint32_t& xph,
                                          uint32_t rank, uint32_t C, float (&out)[8],
@@ -208,6 +210,8 @@ __device__ __forceinline__ void exchange(Head& H, float a0, float a1, float a2, 
   } else {
     a0 = group_sum<5>(a0);
     a1 = group_sum<5>(a1);
+    if constexpr (NSUM > 2) a2 = group_sum<5>(a2);
+    if constexpr (NSUM > 3) a3 = group_sum<5>(a3);
   }
   flags = __reduce_or_sync(0xffffffffu, flags);
   if (lane == 0) {
@@ -232,6 +236,8 @@ __device__ __forceinline__ void exchange(Head& H, float a0, float a1, float a2, 
     } else {
       a0 = group_sum<4>(a0);
       a1 = group_sum<4>(a1);
+      if constexpr (NSUM > 2) a2 = group_sum<4>(a2);
+      if constexpr (NSUM > 3) a3 = group_sum<4>(a3);
     }
     const int p = xp;
     if (lane < (int)C) {
@@ -264,6 +270,8 @@ __device__ __forceinline__ void exchange(Head& H, float a0, float a1, float a2, 
     } else {
       a0 = group_sum<4>(a0);
       a1 = group_sum<4>(a1);
+      if constexpr (NSUM > 2) a2 = group_sum<4>(a2);
+      if constexpr (NSUM > 3) a3 = group_sum<4>(a3);
     }
     if (lane == 0) {
       H.bc[0] = a0; H.bc[1] = a1; H.bc[2] = a2; H.bc[3] = a3;

@@ -1032,13 +1032,17 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
       // one pass: the residual so far and the sums of the new map, in
       // unnormalised units (k: the new map's scalar).  The rejected tokens
       // get no special case here; their terms are taken out below.
-      const float kq = __fdiv_rn(resi ? __fmul_rn(Z, dsc) : K.invSd, K.sig);
+      float kq = __fdiv_rn(resi ? __fmul_rn(Z, dsc) : K.invSd, K.sig);
       // s1: sum of min(k D~, R~) (ResiSpec) or of the capacity t (SpecInfer);
-      // s2: sum of t (ResiSpec); both as pairs of lanes.  D~ is q~ unless the
-      // proxies replace the denominator (then the chain leaves it in q[]).
-      float2 s1p = make_float2(0.f, 0.f), s2p = make_float2(0.f, 0.f);
-      auto rej_pass = [&](auto kind_c) {
+      // s2: sum of t (ResiSpec), or in a level pass the sum of R~ where
+      // D~ > 0 (s1 for an unbounded k); s3 (level pass): the sum of D~ where
+      // k D~ < R~, the slope of s1 in k.  All as pairs of lanes.  D~ is q~
+      // unless the proxies replace the denominator (then the chain leaves it
+      // in q[]).
+      float2 s1p, s2p, s3p;
+      auto rej_pass = [&](auto kind_c, auto level_c) {
         constexpr int KIND = decltype(kind_c)::value;
+        constexpr bool LEVEL = decltype(level_c)::value;
         const float2 c2 = dup2(K.c), nMt = dup2(-K.Mt), nMd = dup2(-K.Md), kq2 = dup2(kq),
                      nkq = dup2(-kq);
         stream_pass<THREADS, BF16>(ring, src, [&](const unsigned char* rt, const unsigned char* rd,
@@ -1058,7 +1062,13 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
 #pragma unroll
             for (int j = 0; j < 4; ++j) {
               m[j] = min_part2(kq2, q[j], Rv[j]);
-              t[j] = __ffma2_rn(m[j], dup2(-1.f), Rv[j]);
+              if constexpr (LEVEL) {
+                s3p.x += m[j].x < Rv[j].x ? q[j].x : 0.f;
+                s3p.y += m[j].y < Rv[j].y ? q[j].y : 0.f;
+                t[j] = make_float2(q[j].x > 0.f ? Rv[j].x : 0.f, q[j].y > 0.f ? Rv[j].y : 0.f);
+              } else {
+                t[j] = __ffma2_rn(m[j], dup2(-1.f), Rv[j]);
+              }
             }
             s1p = __fadd2_rn(s1p, __fadd2_rn(__fadd2_rn(m[0], m[1]), __fadd2_rn(m[2], m[3])));
             s2p = __fadd2_rn(s2p, __fadd2_rn(__fadd2_rn(t[0], t[1]), __fadd2_rn(t[2], t[3])));
@@ -1071,41 +1081,96 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
           return false;
         });
       };
-      if (chain == kChainResiDenom) rej_pass(std::integral_constant<int, kChainResiDenom>{});
-      else if (chain == kChainResi) rej_pass(std::integral_constant<int, kChainResi>{});
-      else rej_pass(std::integral_constant<int, kChainSpec>{});
-      float s1 = __fadd_rn(s1p.x, s1p.y), s2 = __fadd_rn(s2p.x, s2p.y);
-      if (resi) {
-        // The token just rejected (r(x0) = 0) and the earlier rejected ones
-        // (R = 0 there) add nothing: the thread that summed each such token
-        // of this slice subtracts the terms the pass gave it, recomputed
-        // bit for bit (each distinct token once).
-        for (int t = -1; t < nm; ++t) {
-          const int y = t < 0 ? x : S2.rej[t];
-          const int yk = t < 0 ? i : S2.rejk[t];
-          if (y < lo || y >= lo + nloc) continue;
-          if ((((y - lo) % G::CE) / VEC) % THREADS != tid) continue;
-          bool seen = t >= 0 && y == x;
-          for (int t2 = 0; t2 < t && !seen; ++t2) seen = S2.rej[t2] == y;
-          if (seen) continue;
-          float Dy = exp_of(S2.kzd[yk], K.c, K.Md);
-          const float py = exp_of(S2.kzt[yk], K.c, K.Mt);
-          const float Ry = chain == kChainResiDenom ? apply_chain<kChainResiDenom>(S2, nm, py, Dy)
-                                                    : apply_chain<kChainResi>(S2, nm, py, Dy);
-          const float my = fminf(__fmul_rn(kq, Dy), Ry);
-          s1 = __fsub_rn(s1, my);
-          s2 = __fsub_rn(s2, __fmaf_rn(my, -1.f, Ry));
+      // The level fill (r = min(lam q, R) with sum r = Z) moves k by Newton
+      // steps from k = Z: s1 is concave and piecewise linear in k, so every
+      // step stays at or below the level and the steps end on its piece.
+      // The loop stops when the deficit is below 2^-22 Z, when a step no
+      // longer moves k in fp32, or after kLevelSteps passes; the residual is
+      // then normalised by the mass reached, so what is left of the deficit
+      // scales every token by the same relative amount (as a rounding
+      // would) instead of moving mass between tokens.  When even an
+      // unbounded level falls short of Z (the first level pass's s2 < Z: the
+      // support of the denominator cannot hold the budget) no level exists:
+      // one plain pass at k = FLT_MAX saturates that support and the default
+      // fill places the rest on the tokens outside it.  Every CTA sees the
+      // same exchanged sums, so all take the same steps.
+      constexpr int kLevelSteps = 24;
+      const bool level = resi && P.level_fill != 0;
+      bool timed_out = false, saturate = false;
+      float s1, s2, s3;
+      for (int step = 0;; ++step) {
+        const bool lpass = level && !saturate;
+        s1p = s2p = s3p = make_float2(0.f, 0.f);
+        if (chain == kChainResiDenom) {
+          if (lpass) rej_pass(std::integral_constant<int, kChainResiDenom>{}, std::true_type{});
+          else rej_pass(std::integral_constant<int, kChainResiDenom>{}, std::false_type{});
+        } else if (chain == kChainResi) {
+          if (lpass) rej_pass(std::integral_constant<int, kChainResi>{}, std::true_type{});
+          else rej_pass(std::integral_constant<int, kChainResi>{}, std::false_type{});
+        } else {
+          rej_pass(std::integral_constant<int, kChainSpec>{}, std::false_type{});
         }
+        s1 = __fadd_rn(s1p.x, s1p.y);
+        s2 = __fadd_rn(s2p.x, s2p.y);
+        s3 = __fadd_rn(s3p.x, s3p.y);
+        if (resi) {
+          // The token just rejected (r(x0) = 0) and the earlier rejected ones
+          // (R = 0 there) add nothing: the thread that summed each such token
+          // of this slice subtracts the terms the pass gave it, recomputed
+          // bit for bit (each distinct token once).
+          for (int t = -1; t < nm; ++t) {
+            const int y = t < 0 ? x : S2.rej[t];
+            const int yk = t < 0 ? i : S2.rejk[t];
+            if (y < lo || y >= lo + nloc) continue;
+            if ((((y - lo) % G::CE) / VEC) % THREADS != tid) continue;
+            bool seen = t >= 0 && y == x;
+            for (int t2 = 0; t2 < t && !seen; ++t2) seen = S2.rej[t2] == y;
+            if (seen) continue;
+            float Dy = exp_of(S2.kzd[yk], K.c, K.Md);
+            const float py = exp_of(S2.kzt[yk], K.c, K.Mt);
+            const float Ry = chain == kChainResiDenom
+                                 ? apply_chain<kChainResiDenom>(S2, nm, py, Dy)
+                                 : apply_chain<kChainResi>(S2, nm, py, Dy);
+            const float my = fminf(__fmul_rn(kq, Dy), Ry);
+            s1 = __fsub_rn(s1, my);
+            if (!lpass) {
+              s2 = __fsub_rn(s2, __fmaf_rn(my, -1.f, Ry));
+            } else {
+              if (Dy > 0.f) s2 = __fsub_rn(s2, Ry);
+              if (my < Ry) s3 = __fsub_rn(s3, Dy);
+            }
+          }
+        }
+        if (lpass)
+          exchange<NW, false, 3>(H, s1, s2, s3, 0.f, 0, -1, xp, xph, rank, C, o, oflags);
+        else
+          exchange<NW, false>(H, s1, s2, 0.f, 0.f, 0, -1, xp, xph, rank, C, o, oflags);
+        mark(kPhaseTest);
+        if (oflags & kFlagTimeout) { timed_out = true; break; }
+        if (!level || saturate || step + 1 >= kLevelSteps) break;
+        float kn;
+        if (step == 0 && __fmul_rn(o[1], K.sig) < Z) {  // no level reaches Z
+          saturate = true;
+          kn = FLT_MAX;
+        } else {
+          // normalised: s1 o[0] sig, slope o[2] sig per unit of k
+          const float gap = __fsub_rn(Z, __fmul_rn(o[0], K.sig));
+          const float slope = __fmul_rn(o[2], K.sig);
+          if (!(gap > __fmul_rn(Z, 0x1p-22f)) || !(slope > 0.f)) break;
+          kn = __fadd_rn(kq, __fdiv_rn(gap, slope));
+          if (!(kn > kq)) break;
+        }
+        kq = kn;
+        mark(kPhaseRej);
       }
-      exchange<NW, false>(H, s1, s2, 0.f, 0.f, 0, -1, xp, xph, rank, C, o, oflags);
-      mark(kPhaseTest);
-      if (oflags & kFlagTimeout) { err |= kErrTimeout; break; }
+      if (timed_out) { err |= kErrTimeout; break; }
       bool has_map = false;
       float a = 0.f, lam = 0.f;
       if (resi) {
         const float S1 = __fmul_rn(o[0], K.sig), S2s = __fmul_rn(o[1], K.sig);
         const float delta = __fsub_rn(Z, S1);
-        lam = S2s > 0.f ? fminf(fmaxf(__fdiv_rn(delta, S2s), 0.f), 1.f) : 0.f;
+        lam = S2s > 0.f && (!level || saturate) ? fminf(fmaxf(__fdiv_rn(delta, S2s), 0.f), 1.f)
+                                                 : 0.f;
         const float norm = __fmaf_rn(lam, S2s, S1);
         if (norm > 0.f) {
           has_map = true;

@@ -120,6 +120,13 @@ def test_plan_without_device(lib):
     o = rs.make_opts(kernel="stream")
     o.flags |= rs.FLAG_RESIDENT                   # both kernels forced: argument error
     assert lib.resispec_plan(rs.Dims(1, 2, 10, 1, rs.F32), o, None) == rs.E_ARG
+    # the variants run on the streaming kernel only
+    for kw in (dict(z_rule=rs.Z_RULE_APPLIED), dict(proxy_denominator=True),
+               dict(fill=rs.FILL_LEVEL)):
+        assert rs.plan(1, 2, 64, 1, "f32", **kw)["kernel_name"] == "stream"
+        o = rs.make_opts(**kw)
+        o.flags |= rs.FLAG_RESIDENT
+        assert lib.resispec_plan(rs.Dims(1, 2, 64, 1, rs.F32), o, None) == rs.E_ARG
 
 
 def test_no_cpu_path():

@@ -35,7 +35,7 @@ def _check(inp, mode, seed, **kw):
     g = P.run_gpu(zt, zd, pa, ca, inp["temperature"], seed, D, mode=mode, **kw)
     o = P.run_oracle(inp["target"], inp["draft"], inp["parents"], inp["cand"],
                      inp["temperature"], seed, D, mode, z_rule=kw.get("z_rule", 0),
-                     denom_update=kw.get("proxy_denominator", False))
+                     denom_update=kw.get("proxy_denominator", False), fill=kw.get("fill", 0))
     n, near = P.compare(g, o)
     # near-tie differences are allowed but must stay rare
     assert near <= max(2, 0.002 * n), (near, n)
@@ -320,7 +320,7 @@ def _sampled_parity(w, seed, call_seed, rows, mode=rs.MODE_RESISPEC, batch=None,
     pa = inp["parents_np"][rows] if inp["parents_np"].ndim == 2 else inp["parents_np"]
     o = P.run_oracle(th, dh, pa, ch, w.temperature, call_seed, D, mode,
                      seq_ids=np.asarray(rows, np.int32), z_rule=kw.get("z_rule", 0),
-                     denom_update=kw.get("proxy_denominator", False))
+                     denom_update=kw.get("proxy_denominator", False), fill=kw.get("fill", 0))
     n, near = P.compare(g, o, rows=rows)
     assert near <= 1, near
     assert g["status"][0] & ~rs.INFO_DEGENERATE == 0
@@ -544,6 +544,103 @@ def test_gpu_proxy_denominator_million_draws_vs_enumerator():
     dist0, _ = en.single_position(p, q, k, en.MODE_RESISPEC)
     assert chisq_pvalue(counts, dist)[0] > 1e-4
     assert np.abs(dist - dist0).max() > 1e-3
+
+
+# ------------------------------------------------------------ level fill
+
+
+@pytest.mark.parametrize("wl", ["tree60-v32000", "chain8x4-v128256-b16", "dyntree60-v32000"])
+def test_parity_level_fill(wl):
+    """GetProxy's deficit raised to a level (r = min(lam q, R) with sum r =
+    Z): every sequence against the oracle's exact level, which must change
+    some walks against the default fill."""
+    w = W.WORKLOADS[wl]
+    inp = W.make_inputs_np(w, seed=17, batch=256 if wl != "chain8x4-v128256-b16" else 16)
+    g, o = _check(inp, rs.MODE_RESISPEC, seed=171, fill=rs.FILL_LEVEL)
+    o0 = P.run_oracle(inp["target"], inp["draft"], inp["parents"], inp["cand"],
+                      inp["temperature"], 171, int(inp["max_depth"]), rs.MODE_RESISPEC)
+    if wl != "chain8x4-v128256-b16":
+        assert ((o0["tokens"] != o["tokens"]).any(axis=1) | (o0["rejects"] != o["rejects"])).any()
+
+
+@pytest.mark.parametrize("other", [dict(proxy_denominator=True), dict(z_rule=rs.Z_RULE_APPLIED)])
+def test_parity_level_fill_with_other_variants(other):
+    """The level fill combined with the proxy denominator (the level is
+    taken against the current denominator) and with the Z_applied budget."""
+    w = W.WORKLOADS["tree60-v32000"]
+    inp = W.make_inputs_np(w, seed=19, batch=256)
+    _check(inp, rs.MODE_RESISPEC, seed=191, fill=rs.FILL_LEVEL, **other)
+
+
+@pytest.mark.parametrize("mode", MODES)
+def test_level_fill_wide_fanout(mode):
+    """128 children whose candidates the target all but excludes: up to 128
+    level searches at one node (SpecInfer: the flag has no effect)."""
+    V, kids = 3000, rs.MAX_FANOUT_STREAM
+    rng = np.random.default_rng(kids + 1)
+    zt = rng.normal(0, 2, (8, kids + 1, V)).astype(np.float32)
+    zd = rng.normal(0, 2, (8, kids + 1, V)).astype(np.float32)
+    cand = rng.integers(0, V, (8, kids)).astype(np.int32)
+    for b in range(8):
+        zt[b, 0, cand[b]] = -30.0
+    inp = {"target": zt, "draft": zd, "parents": np.full(kids, -1, np.int32), "cand": cand,
+           "temperature": 1.0, "max_depth": 1}
+    _check(inp, mode, seed=kids + 1, fill=rs.FILL_LEVEL)
+
+
+def test_level_fill_without_room_on_the_draft_support():
+    """Draft rows that exclude (-inf) half of the vocabulary, where the
+    target keeps most of its mass: the level saturates the draft's support
+    and the default fill places the rest, as in the oracle."""
+    V, k, B = 512, 4, 64
+    rng = np.random.default_rng(23)
+    zt = rng.normal(0, 1, (B, k + 1, V)).astype(np.float32)
+    zd = rng.normal(0, 1, (B, k + 1, V)).astype(np.float32)
+    zt[:, :, V // 2:] += 8.0
+    zd[:, :, V // 2:] = -np.inf
+    cand = rng.integers(0, V // 2, (B, k)).astype(np.int32)
+    for b in range(B):   # every candidate rejected: four shapings per sequence
+        zt[b, 0, cand[b]] = -30.0
+    # the first rejection at the root already finds no finite level
+    no_room = 0
+    for b in range(B):
+        p0, q0 = sp_softmax(zt[b, 0].astype(np.float64)), sp_softmax(zd[b, 0].astype(np.float64))
+        x0 = cand[b, 0]
+        no_room += p0[q0 > 0].sum() - p0[x0] < q0[x0] - p0[x0]
+    assert no_room > B // 2
+    inp = {"target": zt, "draft": zd, "parents": np.full(k, -1, np.int32), "cand": cand,
+           "temperature": 1.0, "max_depth": 1}
+    g, o = _check(inp, rs.MODE_RESISPEC, seed=231, fill=rs.FILL_LEVEL)
+    assert (o["rejects"] == k).all()
+    o0 = P.run_oracle(zt, zd, inp["parents"], cand, 1.0, 231, 1, rs.MODE_RESISPEC)
+    assert np.abs(o["dist"] - o0["dist"]).max() > 1e-5   # 30x the parity bound
+
+
+def test_parity_level_fill_binary5_full_size():
+    w = W.WORKLOADS["binary5-v151936-b64"]
+    _sampled_parity(w, seed=35, call_seed=1006, rows=[1, 22, 40, 61], fill=rs.FILL_LEVEL)
+
+
+def test_gpu_level_fill_million_draws_vs_enumerator():
+    """The level fill on the GPU follows its own enumerated law (the
+    enumerator finds the level by bisection)."""
+    import torch
+    V, k, n = 16, 3, 1_000_000
+    rng = np.random.default_rng(7)
+    zt = (2.0 * rng.standard_normal(V)).astype(np.float32)
+    zd = (0.8 * zt + 1.2 * rng.standard_normal(V)).astype(np.float32)
+    p, q = sp_softmax(zt.astype(np.float64)), sp_softmax(zd.astype(np.float64))
+    cand = rng.choice(V, size=(n, k), p=q).astype(np.int32)
+    toks, _ = rs.verify(P.to_device(np.broadcast_to(zt, (k + 1, V)).copy()),
+                        P.to_device(np.broadcast_to(zd, (k + 1, V)).copy()),
+                        torch.full((k,), -1, dtype=torch.int32, device="cuda"),
+                        torch.as_tensor(cand, device="cuda"), 1.0, 99, max_depth=1,
+                        seq_stride=0, fill=rs.FILL_LEVEL)
+    counts = np.bincount(toks[:, 0].cpu().numpy(), minlength=V)
+    dist, _ = en.single_position(p, q, k, en.MODE_RESISPEC, fill=1)
+    dist0, _ = en.single_position(p, q, k, en.MODE_RESISPEC)
+    assert chisq_pvalue(counts, dist)[0] > 1e-4
+    assert np.abs(dist - dist0).max() > 1e-3 and chisq_pvalue(counts, dist0)[0] < 1e-8
 
 
 @pytest.mark.parametrize("mode", MODES)

@@ -318,7 +318,9 @@ def run_reference(args):
         "ms_per_step": 1e3 * el / max(1, args.steps), "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
         "config": {"workload": w.name, "batch_per_step": S, "vocab": w.vocab,
-                   "nodes_per_seq": w.num_nodes, "mode": args.mode, "rho": w.rho},
+                   "nodes_per_seq": w.num_nodes, "mode": args.mode, "rho": w.rho,
+                   "z_rule": args.z_rule, "proxy_denominator": args.proxy_denominator,
+                   "fill": args.fill, "draft": args.draft},
         "cpu_baseline": {"value": value, "unit": "nodes/s", "cores": threads, "kind": "oracle",
                          "sample": f"{S} sequences of {w.name} per step (host inputs)"},
         "e2e": {"value": value, "unit": "nodes/s", "h2d_bytes_per_step": 0,

@@ -94,3 +94,22 @@ def test_rows_visited_per_sequence_trees():
     np.testing.assert_array_equal(bench.rows_visited(nodes, alen, hc), [3, 5])
     np.testing.assert_array_equal(bench.rows_visited(nodes, alen, bench.has_children(parents[0])),
                                   [3, 5])
+
+
+def test_reference_arm_times_the_variant_it_is_asked_for():
+    """The oracle legs verify with the same rule as the measured run."""
+    import argparse
+    import bench
+    ns = argparse.Namespace(z_rule="applied", proxy_denominator=True, fill="level", draft=False)
+    assert bench.oracle_variant(ns) == dict(z_rule=1, denom_update=True, fill=1,
+                                            draft_children=False)
+    ns = argparse.Namespace(z_rule="alg1", proxy_denominator=False, fill="capacity", draft=True)
+    assert bench.oracle_variant(ns) == dict(z_rule=0, denom_update=False, fill=0,
+                                            draft_children=True)
+    cmd = [sys.executable, os.path.join(ROOT, "bench.py"), "--impl", "reference", "--steps", "1",
+           "--warmup", "0", "--cpu-seqs", "4", "--workload", "tiny-chain-v64", "--fill", "level",
+           "--proxy-denominator"]
+    p = subprocess.run(cmd, cwd=ROOT, capture_output=True, text=True, timeout=300)
+    assert p.returncode == 0, p.stderr[-2000:]
+    d = json.loads([l for l in p.stdout.splitlines() if l.startswith("{")][-1])
+    assert d["config"]["fill"] == "level" and d["config"]["proxy_denominator"] is True

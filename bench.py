@@ -414,11 +414,13 @@ def run_ours(args):
     alg_bytes = 0
     emitted = 0
     accepted = 0
+    rows_read = 0
     for i in range(K):
         alen = outs[i][1].cpu().numpy()
         nodes = outs[i][2].cpu().numpy()[:, :D]
         rows = rows_visited(nodes, alen, haschild[(Wm + i) % pool])
         alg_bytes += int(rows.sum()) * V * es
+        rows_read += int(rows.sum())
         emitted += int((alen + 1).sum())
         accepted += int(alen.sum())
     mean_launch_s = (sum(launch_ms) / K) / 1e3
@@ -447,8 +449,13 @@ def run_ours(args):
                      "traffic": profiled_traffic(plan["kernel_name"], w.name, alg_bytes / K),
                      "peak_kind": peak_kind, "frac_of_8tbs": achieved_gbs / NOMINAL_HBM_GBS,
                      "alg_bytes_per_launch": alg_bytes / K,
-                     "mean_launch_us": mean_launch_s * 1e6},
+                     "mean_launch_us": mean_launch_s * 1e6,
+                     "median_launch_us": statistics.median(launch_ms) * 1e3},
         "tokens_per_s": sum_over_ranks(float(emitted)) / (elapsed_ms / 1e3),
+        # nodes whose rows were read (the root and every accepted node): one
+        # emitted token each, so equal to tokens_per_s
+        "visited_nodes_per_s": sum_over_ranks(float(emitted)) / (elapsed_ms / 1e3),
+        "rows_read_per_s": sum_over_ranks(float(rows_read)) / (elapsed_ms / 1e3),
         "mean_accept_len": accepted / (K * B),
         "gpu_launches": K,
         "wall_s": wall,

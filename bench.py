@@ -212,8 +212,13 @@ def cpu_oracle_rate(w, target_h, draft_h, parents, cand_h, seq_ids, mode, second
     variant = variant or {}
     S = cand_h.shape[0]
     threads = min(os.cpu_count() or 1, S)
-    oracle.verify(target_h[:1], draft_h[:1], parents, cand_h[:1], w.temperature, seed0,
-                  mode=mode, max_depth=w.max_depth, seq_ids=seq_ids[:1], nthreads=1, **variant)
+    # one thread on the first (at most two) sequences: the per-core rate
+    s1 = min(2, S)
+    p1 = parents[:s1] if np.asarray(parents).ndim == 2 else parents
+    t1 = time.perf_counter()
+    oracle.verify(target_h[:s1], draft_h[:s1], p1, cand_h[:s1], w.temperature, seed0,
+                  mode=mode, max_depth=w.max_depth, seq_ids=seq_ids[:s1], nthreads=1, **variant)
+    one_thread = s1 * w.num_nodes / (time.perf_counter() - t1)
     reps, t0 = 0, time.perf_counter()
     while True:
         oracle.verify(target_h, draft_h, parents, cand_h, w.temperature, seed0 + reps, mode=mode,
@@ -225,7 +230,27 @@ def cpu_oracle_rate(w, target_h, draft_h, parents, cand_h, seq_ids, mode, second
     nodes = reps * S * w.num_nodes
     sample = (f"{reps} calls x {S} sequences of {w.name} (rows copied to host), "
               f"{nodes} verified nodes in {el:.2f} s")
-    return nodes / el, threads, sample
+    return nodes / el, threads, sample, one_thread
+
+
+def cpu_model() -> str:
+    """The host CPU's model name (lscpu's, or /proc/cpuinfo's), else the
+    machine type."""
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        for line in out.splitlines():
+            if line.startswith("Model name:"):
+                return line.split(":", 1)[1].strip()
+    except (OSError, subprocess.SubprocessError):
+        pass
+    try:
+        for line in open("/proc/cpuinfo"):
+            if line.startswith("model name"):
+                return line.split(":", 1)[1].strip()
+    except OSError:
+        pass
+    import platform
+    return platform.machine()
 
 
 # ------------------------------------------------------------------ ranks
@@ -322,7 +347,8 @@ def run_reference(args):
                    "z_rule": args.z_rule, "proxy_denominator": args.proxy_denominator,
                    "fill": args.fill, "draft": args.draft},
         "cpu_baseline": {"value": value, "unit": "nodes/s", "cores": threads, "kind": "oracle",
-                         "sample": f"{S} sequences of {w.name} per step (host inputs)"},
+                         "sample": f"{S} sequences of {w.name} per step (host inputs)",
+                         "cpu_model": cpu_model(), "nproc": os.cpu_count()},
         "e2e": {"value": value, "unit": "nodes/s", "h2d_bytes_per_step": 0,
                 "d2h_bytes_per_step": 0},
     }
@@ -532,11 +558,12 @@ def _finish_cpu(result, args, sets, w, mode, world, dev):
     ch = s0["cand"].index_select(0, idx).cpu().numpy()
     omode = oracle.MODE_SPECINFER if mode == 1 else oracle.MODE_RESISPEC
     pa = s0["parents_np"][:S] if w.per_sequence_tree else s0["parents_np"]
-    rate, threads, sample = cpu_oracle_rate(w, th, dh, pa, ch,
-                                            np.arange(S, dtype=np.int32), omode,
-                                            args.cpu_seconds, args.seed, oracle_variant(args))
+    rate, threads, sample, one = cpu_oracle_rate(w, th, dh, pa, ch,
+                                                 np.arange(S, dtype=np.int32), omode,
+                                                 args.cpu_seconds, args.seed, oracle_variant(args))
     result["cpu_baseline"] = {"value": rate, "unit": "nodes/s", "cores": threads,
-                              "kind": "oracle", "sample": sample}
+                              "kind": "oracle", "sample": sample, "one_thread_value": one,
+                              "cpu_model": cpu_model(), "nproc": os.cpu_count()}
     return result
 
 

@@ -113,3 +113,19 @@ def test_reference_arm_times_the_variant_it_is_asked_for():
     assert p.returncode == 0, p.stderr[-2000:]
     d = json.loads([l for l in p.stdout.splitlines() if l.startswith("{")][-1])
     assert d["config"]["fill"] == "level" and d["config"]["proxy_denominator"] is True
+
+
+@pytest.mark.parametrize("wl", ["tiny-chain-v64", "dyntree60-v32000"])
+def test_cpu_oracle_rate_on_host_inputs(wl):
+    """The CPU-baseline leg of the GPU arm, on host copies of a workload
+    (one shared tree, and a tree per sequence)."""
+    import bench
+    import oracle
+    from paper_2608_24411_gb300 import workloads as W
+    w = W.WORKLOADS[wl]
+    inp = W.make_inputs_np(w, seed=0, batch=4)
+    rate, threads, sample, one = bench.cpu_oracle_rate(
+        w, inp["target"], inp["draft"], inp["parents"], inp["cand"],
+        np.arange(4, dtype=np.int32), oracle.MODE_RESISPEC, 0.05, 1, {"fill": 1})
+    assert rate > 0 and one > 0 and 1 <= threads <= 4 and "verified nodes" in sample
+    assert isinstance(bench.cpu_model(), str)

@@ -4,6 +4,7 @@
 
 namespace rs {
 const void* stream_entry_bf16(int threads) {
-  return threads == 512 ? (const void*)stream_kernel<512, true> : (const void*)stream_kernel<256, true>;
+  return threads == 512 ? (const void*)stream_kernel<512, true, false>
+                       : (const void*)stream_kernel<256, true, false>;
 }
 }  // namespace rs

@@ -4,6 +4,7 @@
 
 namespace rs {
 const void* stream_entry_f32(int threads) {
-  return threads == 512 ? (const void*)stream_kernel<512, false> : (const void*)stream_kernel<256, false>;
+  return threads == 512 ? (const void*)stream_kernel<512, false, false>
+                       : (const void*)stream_kernel<256, false, false>;
 }
 }  // namespace rs

@@ -8,4 +8,6 @@ const void* resident_entry_f32(int threads);
 const void* resident_entry_bf16(int threads);
 const void* stream_entry_f32(int threads);
 const void* stream_entry_bf16(int threads);
+const void* stream_var_entry_f32(int threads);   // with the optional paths
+const void* stream_var_entry_bf16(int threads);
 }  // namespace rs

@@ -44,6 +44,7 @@ constexpr int kAutoSliceBytes = 96 * 1024; // target on-chip bytes per CTA (two 
 
 struct Plan {
   int kernel = RESISPEC_KERNEL_RESIDENT;
+  int var = 0;  // streaming kernel with the optional paths compiled in
   int C = 1;
   int threads = 512;
   int L = 8;
@@ -82,7 +83,7 @@ struct DeviceInfo {
 
 std::mutex g_mu;
 DeviceInfo g_dev[64];
-bool g_attr_set[64][8];
+bool g_attr_set[64][16];
 
 int query_device(int* dev_out, DeviceInfo* info) {
   int dev = 0;
@@ -117,19 +118,21 @@ int check_dims(const resispec_dims& d) {
 
 // Clusters of this shape that can be resident at once (0: the shape cannot
 // be launched).  Cached per device and shape.
-using OccKey = std::tuple<int, int, int, int, int, int>;  // dev, kernel, threads, bf16, C, smem
+using OccKey = std::tuple<int, int, int, int, int, int>;  // dev, kernel id, threads, bf16, C, smem
 std::map<OccKey, int> g_occ;
 
 template <int THREADS, bool BF16>
-const void* kernel_ptr(int kernel) {
+const void* kernel_ptr(int kernel, int var) {
+  if (kernel == RESISPEC_KERNEL_STREAM && var)
+    return BF16 ? rs::stream_var_entry_bf16(THREADS) : rs::stream_var_entry_f32(THREADS);
   if (kernel == RESISPEC_KERNEL_STREAM)
     return BF16 ? rs::stream_entry_bf16(THREADS) : rs::stream_entry_f32(THREADS);
   return BF16 ? rs::resident_entry_bf16(THREADS) : rs::resident_entry_f32(THREADS);
 }
 
 template <int THREADS, bool BF16>
-int query_clusters(int kernel, int C, int smem) {
-  const void* kern = kernel_ptr<THREADS, BF16>(kernel);
+int query_clusters(int kernel, int var, int C, int smem) {
+  const void* kern = kernel_ptr<THREADS, BF16>(kernel, var);
   if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, kMaxSmem) !=
           cudaSuccess ||
       cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) !=
@@ -157,8 +160,8 @@ int query_clusters(int kernel, int C, int smem) {
   return n;
 }
 
-int active_clusters(int dev, int kernel, int threads, bool bf16, int C, int smem) {
-  const OccKey key{dev, kernel, threads, bf16 ? 1 : 0, C, smem};
+int active_clusters(int dev, int kernel, int var, int threads, bool bf16, int C, int smem) {
+  const OccKey key{dev, kernel * 2 + (var ? 1 : 0), threads, bf16 ? 1 : 0, C, smem};
   {
     std::lock_guard<std::mutex> lk(g_mu);
     auto it = g_occ.find(key);
@@ -166,11 +169,11 @@ int active_clusters(int dev, int kernel, int threads, bool bf16, int C, int smem
   }
   int n;
   if (threads == 512)
-    n = bf16 ? query_clusters<512, true>(kernel, C, smem)
-             : query_clusters<512, false>(kernel, C, smem);
+    n = bf16 ? query_clusters<512, true>(kernel, var, C, smem)
+             : query_clusters<512, false>(kernel, var, C, smem);
   else
-    n = bf16 ? query_clusters<256, true>(kernel, C, smem)
-             : query_clusters<256, false>(kernel, C, smem);
+    n = bf16 ? query_clusters<256, true>(kernel, var, C, smem)
+             : query_clusters<256, false>(kernel, var, C, smem);
   std::lock_guard<std::mutex> lk(g_mu);
   g_occ[key] = n;
   return n;
@@ -190,7 +193,7 @@ int plan_resident(const resispec_dims& d, int cs, int dev, int sms, Plan* p) {
     for (int C = 1; C <= rs::kMaxCluster; ++C) {
       const int smem = smem_for(slice_for(V, C), p->npad);
       if (smem > kMaxSmem) continue;
-      const int n = active_clusters(dev, RESISPEC_KERNEL_RESIDENT, p->threads, bf16, C, smem);
+      const int n = active_clusters(dev, RESISPEC_KERNEL_RESIDENT, 0, p->threads, bf16, C, smem);
       if (n <= 0) continue;
       const int64_t score = std::min<int64_t>(d.batch, n) * C;
       if (score >= best_score) { best_score = score; best = C; }
@@ -206,7 +209,7 @@ int plan_resident(const resispec_dims& d, int cs, int dev, int sms, Plan* p) {
   p->L = slice_for(V, p->C);
   p->smem = smem_for(p->L, p->npad);
   if (p->smem > kMaxSmem) return RESISPEC_E_SHAPE;
-  p->active = dev >= 0 ? active_clusters(dev, RESISPEC_KERNEL_RESIDENT, p->threads, bf16, p->C,
+  p->active = dev >= 0 ? active_clusters(dev, RESISPEC_KERNEL_RESIDENT, 0, p->threads, bf16, p->C,
                                          p->smem)
                        : 0;
   return RESISPEC_OK;
@@ -228,7 +231,8 @@ int plan_stream(const resispec_dims& d, int cs, int dev, int sms, Plan* p) {
   if (p->smem > kMaxSmem) return RESISPEC_E_SHAPE;
   const int B = std::max(d.batch, 1);
   auto active_for = [&](int C) {
-    if (dev >= 0) return active_clusters(dev, RESISPEC_KERNEL_STREAM, p->threads, bf16, C, p->smem);
+    if (dev >= 0)
+      return active_clusters(dev, RESISPEC_KERNEL_STREAM, p->var, p->threads, bf16, C, p->smem);
     const int slots = (sms > 0 ? sms : 152) * (p->threads >= 512 ? 2 : 4);
     return C == 16 ? 14 * slots / 304 : slots / C;
   };
@@ -274,6 +278,7 @@ int make_plan(const resispec_dims& d, const resispec_opts& o, int dev, int sms,
                        o.out_phase_cycles != nullptr || o.out_candidates != nullptr;
   const bool force_str = (o.flags & RESISPEC_FLAG_STREAM) != 0 || variant;
   if (force_res && force_str) return RESISPEC_E_ARG;
+  p->var = variant ? 1 : 0;
   p->threads = o.block_threads ? o.block_threads : 512;
   p->npad = round_up(d.num_nodes + 1, 16);
   const int V = d.vocab;
@@ -312,9 +317,9 @@ int make_plan(const resispec_dims& d, const resispec_opts& o, int dev, int sms,
 template <int THREADS, bool BF16>
 cudaError_t launch_verify(const Plan& pl, const rs::VerifyParams& prm, cudaStream_t stream,
                           int dev) {
-  const void* kern = kernel_ptr<THREADS, BF16>(pl.kernel);
-  const int slot = (pl.kernel == RESISPEC_KERNEL_STREAM ? 4 : 0) + (THREADS == 512 ? 2 : 0) +
-                   (BF16 ? 1 : 0);
+  const void* kern = kernel_ptr<THREADS, BF16>(pl.kernel, pl.var);
+  const int slot = (pl.var ? 8 : 0) + (pl.kernel == RESISPEC_KERNEL_STREAM ? 4 : 0) +
+                   (THREADS == 512 ? 2 : 0) + (BF16 ? 1 : 0);
   {
     std::lock_guard<std::mutex> lk(g_mu);
     if (!g_attr_set[dev][slot]) {

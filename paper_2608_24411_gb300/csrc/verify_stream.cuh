@@ -681,7 +681,11 @@ __device__ bool stream_sample(Head& H, const StreamHead& S2, float* F, unsigned 
 }
 
 // ---------------------------------------------------------------- kernel
-template <int THREADS, bool BF16>
+// VAR: the instance that carries the optional paths (Z_applied, proxy
+// denominator, level fill, drafting, phase counters).  The default instance
+// compiles them out: their code, even untaken, costs the hot loops
+// instruction-cache misses.
+template <int THREADS, bool BF16, bool VAR>
 __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
     stream_kernel(const VerifyParams P) {
   using G = StreamGeom<THREADS, BF16>;
@@ -710,8 +714,8 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
   const int lo = (int)rank * L;
   const int nloc = max(0, min(V, lo + L) - lo);
   const bool resi = P.mode == 0;
-  const int chain = !resi ? kChainSpec : (P.denom_update ? kChainResiDenom : kChainResi);
-  const bool drafting = P.draft_out != nullptr;
+  const int chain = !resi ? kChainSpec : ((VAR && P.denom_update) ? kChainResiDenom : kChainResi);
+  const bool drafting = VAR && P.draft_out != nullptr;
   const bool bf16 = BF16;
 
   int err = 0;
@@ -819,7 +823,7 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
   };
 
   // optional phase counters (thread 0 of every CTA; rank 0 writes them)
-  const bool prof = P.out_phase != nullptr;
+  const bool prof = VAR && P.out_phase != nullptr;
   auto mark = [&](int ph) {
     if (prof && tid == 0) {
       const unsigned long long now = clock64();
@@ -860,7 +864,7 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
     float mt = kNoRef, md = kNoRef;
     float2 st2 = make_float2(0.f, 0.f), sd2 = make_float2(0.f, 0.f);
     float dmin = INFINITY;  // Z_applied: smallest z_t - z_d of the slice
-    const bool zapp = P.z_applied != 0 && resi;
+    const bool zapp = VAR && P.z_applied != 0 && resi;
     // (child t is found by walking t siblings; the loaded logits stay in
     // registers until the pass ends, so no warp waits for them; the draws
     // are computed by the last threads)
@@ -1095,7 +1099,7 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
       // fill places the rest on the tokens outside it.  Every CTA sees the
       // same exchanged sums, so all take the same steps.
       constexpr int kLevelSteps = 24;
-      const bool level = resi && P.level_fill != 0;
+      const bool level = VAR && resi && P.level_fill != 0;
       bool timed_out = false, saturate = false;
       float s1, s2, s3;
       for (int step = 0;; ++step) {

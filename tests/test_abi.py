@@ -135,3 +135,25 @@ def test_no_cpu_path():
     with pytest.raises(ValueError):
         rs.verify(t, t, torch.zeros(1, dtype=torch.int32), torch.zeros((1, 1), dtype=torch.int32),
                   1.0, 0, max_depth=1)
+
+
+def test_binding_constants_match_the_header():
+    """Every RESISPEC_* constant the header defines has the same value in the
+    Python binding (flags, status bits, phases, limits, kernels, ABI)."""
+    text = open(HEADER).read()
+    defs = dict((n, int(v)) for n, v in re.findall(r"^#define (RESISPEC_[A-Z0-9_]+) (\d+)", text,
+                                                   flags=re.M))
+    assert len(defs) >= 25
+    phase = {"SETUP": "setup", "NORM": "norm", "NORM_X": "norm_exchange", "TEST": "test",
+             "REJECT": "reject", "DRAW": "draw"}
+    for name, value in defs.items():
+        short = name[len("RESISPEC_"):]
+        if short == "PHASES":
+            assert len(rs.PHASES) == value
+        elif short.startswith("PHASE_"):
+            assert rs.PHASES.index(phase[short[len("PHASE_"):]]) == value, name
+        elif short == "ABI_VERSION":
+            assert rs.load_library().resispec_abi_version() == value
+        else:
+            assert hasattr(rs, short), f"binding lacks {short}"
+            assert getattr(rs, short) == value, name

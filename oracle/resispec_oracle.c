@@ -32,7 +32,7 @@
  *     accept-test uniform of candidate node c; word 1 of the block of row r
  *     is the residual/bonus uniform of the node whose logits are row r.
  *
- * Readings of points the paper leaves open (each also listed in the design doc):
+ * Readings of points the paper leaves open:
  *   R1  budget Z = q(x0) - R(x0) with R the current residual (Algorithm 1
  *       calls GetProxy(R, Q, x_i)); positive on every rejection.
  *   R2  the deficit is water-filled in proportion to the remaining capacity

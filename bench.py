@@ -510,6 +510,10 @@ def run_ours(args):
         h_len = torch.empty((B,), dtype=torch.int32).pin_memory()
         d_tok = torch.empty((B, D + 1), dtype=torch.int32, device=dev)
         d_len = torch.empty((B,), dtype=torch.int32, device=dev)
+        # drafting: the kernel writes the drafted children here (the same work
+        # as the timed steps)
+        e2e_kw = {"out_candidates": torch.empty((B, N), dtype=torch.int32, device=dev)} \
+            if args.draft else {}
         h2d = sum(t.numel() * t.element_size() for t in host.values())
         d2h = h_tok.numel() * 4 + h_len.numel() * 4
         E = max(1, args.e2e_steps)
@@ -520,7 +524,7 @@ def run_ours(args):
             rs.verify(dbuf["target"], dbuf["draft"], dbuf["parents"], dbuf["cand"],
                       w.temperature, args.seed + i, out_tokens=d_tok, out_accept_len=d_len,
                       max_depth=D, mode=mode, stream=stream, kernel=kernel, z_rule=z_rule,
-                      proxy_denominator=args.proxy_denominator, fill=fill)
+                      proxy_denominator=args.proxy_denominator, fill=fill, **e2e_kw)
             h_tok.copy_(d_tok, non_blocking=True)
             h_len.copy_(d_len, non_blocking=True)
 

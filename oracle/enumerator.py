@@ -20,6 +20,9 @@ oracle and vectorised over the vocabulary:
   integration, App. C): after each rejection the denominator D used by the
   accept tests and by the next GetProxy becomes that rejection's K; the
   candidates are still drawn from the draft q.
+* RESISPEC with the Z_applied budget (``z_rule=1``, the Sec. 5.3 heuristic):
+  Z = max(Z*, |q(x0) - R(x0)|) with Z* the smallest R/q over q > 0, at most
+  1 - R(x0).
 * RESISPEC with the level fill (``fill=1``): r = min(lam q, R) off x0 with
   the level lam >= Z that makes sum r = Z, found here by bisection on the
   nondecreasing function lam -> sum min(lam q, R) (the C oracle solves it
@@ -65,9 +68,17 @@ def level_by_bisection(R, q, x0, Z, iters=200):
     return hi
 
 
-def proxy_resispec(R, q, x0, fill=0):
+def budget(R, q, x0, z_rule=0):
+    gap = q[x0] - R[x0]
+    if z_rule == 0:
+        return gap
+    zstar = np.min(R[q > 0] / q[q > 0])
+    return min(max(zstar, abs(gap)), 1.0 - R[x0])
+
+
+def proxy_resispec(R, q, x0, fill=0, z_rule=0):
     """Returns (K, r, Z) of GetProxy(R, q, x0)."""
-    Z = q[x0] - R[x0]
+    Z = budget(R, q, x0, z_rule)
     lam = Z if fill == 0 else level_by_bisection(R, q, x0, Z)
     r = np.minimum(lam * q, R) if np.isfinite(lam) else np.where(q > 0, R, 0.0)
     r[x0] = 0.0
@@ -81,8 +92,8 @@ def proxy_resispec(R, q, x0, fill=0):
     return K, r, Z
 
 
-def shape_resispec(R, q, x0, fill=0):
-    K, r, Z = proxy_resispec(R, q, x0, fill)
+def shape_resispec(R, q, x0, fill=0, z_rule=0):
+    K, r, Z = proxy_resispec(R, q, x0, fill, z_rule)
     if not Z > 0:
         return R.copy()
     d = np.maximum(R - K, 0.0)
@@ -90,8 +101,9 @@ def shape_resispec(R, q, x0, fill=0):
     return R.copy() if not s > 0 else d / s
 
 
-def shape(mode, R, q, x0, fill=0):
-    return shape_specinfer(R, q) if mode == MODE_SPECINFER else shape_resispec(R, q, x0, fill)
+def shape(mode, R, q, x0, fill=0, z_rule=0):
+    return (shape_specinfer(R, q) if mode == MODE_SPECINFER
+            else shape_resispec(R, q, x0, fill, z_rule))
 
 
 def accept_prob(R, D, x):
@@ -101,11 +113,11 @@ def accept_prob(R, D, x):
     return 1.0 if R[x] > 0 else 0.0
 
 
-def reject_step(mode, R, D, x, denom_update, fill=0):
+def reject_step(mode, R, D, x, denom_update, fill=0, z_rule=0):
     """(R', D') after candidate x is rejected."""
     if mode == MODE_SPECINFER or not denom_update:
-        return shape(mode, R, D, x, fill), D
-    K, r, Z = proxy_resispec(R, D, x, fill)
+        return shape(mode, R, D, x, fill, z_rule), D
+    K, r, Z = proxy_resispec(R, D, x, fill, z_rule)
     if not Z > 0:
         return R.copy(), D
     d = np.maximum(R - K, 0.0)
@@ -115,7 +127,7 @@ def reject_step(mode, R, D, x, denom_update, fill=0):
     return d / s, K
 
 
-def single_position(p, q, k, mode, denom_update=False, fill=0):
+def single_position(p, q, k, mode, denom_update=False, fill=0, z_rule=0):
     """Exact distribution of the emitted token when k i.i.d. candidates from q
     are tested in order against the residual chain starting at p, with the
     residual sample after k rejections (``denom_update``: the test
@@ -140,7 +152,7 @@ def single_position(p, q, k, mode, denom_update=False, fill=0):
             out[x] += q[x] * a
             acc[depth] += weight * q[x] * a
             if a < 1.0:
-                R2, D2 = reject_step(mode, R, D, x, denom_update, fill)
+                R2, D2 = reject_step(mode, R, D, x, denom_update, fill, z_rule)
                 out += q[x] * (1.0 - a) * rec(R2, D2, m - 1, weight * q[x] * (1.0 - a),
                                               depth + 1)
         return out

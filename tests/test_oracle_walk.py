@@ -542,3 +542,45 @@ def test_dist_err_is_zero_without_the_proxy_denominator():
     o = oracle.verify(zt, zd, W.tree_single(k), cand, 1.0, 5, seq_stride=0, want_dist=True,
                       fill=1, want_dist_err=True)
     assert (o["dist_err"] == 0).all()
+
+
+@pytest.mark.parametrize("fill", [0, 1])
+def test_oracle_z_applied_matches_enumerator(fill):
+    """The Z_applied budget (Sec. 5.3 heuristic, reading R7): oracle draws
+    against the law the enumerator derives with its own budget rule.  (By
+    Theorem 2 every budget up to Z* reaches the ideal proxy, so this law is
+    close to Algorithm 1's; the budgets themselves are compared below.)"""
+    V, k, n = 8, 3, 400_000
+    zt, zd = _pq(45, V, scale=1.5, rho=0.4)
+    target, draft, cand = _single_position_draws(7, V, k, n, zt, zd)
+    out = oracle.verify(target, draft, W.tree_single(k), cand, 1.0, seed=2468,
+                        mode=oracle.MODE_RESISPEC, seq_stride=0, z_rule=1, fill=fill)
+    assert (out["status"] & ~oracle.INFO_DEGENERATE == 0).all()
+    p = sp_softmax(zt.astype(np.float64))
+    q = sp_softmax(zd.astype(np.float64))
+    dist, acc = en.single_position(p, q, k, oracle.MODE_RESISPEC, fill=fill, z_rule=1)
+    pv, nb = chisq_pvalue(np.bincount(out["tokens"][:, 0], minlength=V), dist)
+    assert pv > 1e-4, (pv, nb)
+    which = np.where(out["accept_len"] > 0, out["nodes"][:, 0], k)
+    pv2, _ = chisq_pvalue(np.bincount(which, minlength=k + 1), np.append(acc, 1 - acc.sum()))
+    assert pv2 > 1e-4
+
+
+def test_z_applied_budget_matches_enumerator():
+    """The oracle's Z_applied budget against the enumerator's own, on rows
+    where the capacity bound Z* exceeds the gap (the heuristic's case) and
+    where it does not."""
+    rng = np.random.default_rng(46)
+    above = 0
+    for _ in range(300):
+        V = int(rng.integers(2, 30))
+        R = rng.dirichlet(np.full(V, 3.0))
+        q = rng.dirichlet(np.full(V, 3.0))
+        x0 = int(np.argmax(q - R))
+        if not q[x0] > R[x0]:
+            continue
+        zo, ze = oracle.budget(R, q, x0, z_rule=1), en.budget(R, q, x0, z_rule=1)
+        assert zo == pytest.approx(ze, rel=1e-14, abs=1e-16)
+        assert oracle.budget(R, q, x0) == pytest.approx(en.budget(R, q, x0), abs=1e-16)
+        above += zo > q[x0] - R[x0] + 1e-12
+    assert above > 30

@@ -157,3 +157,35 @@ def test_binding_constants_match_the_header():
         else:
             assert hasattr(rs, short), f"binding lacks {short}"
             assert getattr(rs, short) == value, name
+
+
+def test_header_is_c_and_library_links_from_c(tmp_path, lib):
+    """include/resispec.h compiles as C11 and a C program links against the
+    library and calls it (no device work: the ABI version and a synchronous
+    argument error)."""
+    import shutil
+    import subprocess
+    gcc = shutil.which("gcc")
+    if gcc is None:
+        pytest.skip("no C compiler")
+    src = tmp_path / "c_abi.c"
+    src.write_text(r'''
+#include <stdio.h>
+#include <stdint.h>
+#include "resispec.h"
+int main(void) {
+  resispec_opts o;
+  resispec_opts_default(&o);
+  resispec_dims d = {1, 2, 10, 1, RESISPEC_F32};
+  int rc = resispec_verify_ex(0, 0, 0, 0, 1.0f, 0, 0, 0, d, &o, 0);
+  printf("%d %d %d\n", resispec_abi_version(), rc == RESISPEC_E_ARG, o.seq_stride == -1);
+  return 0;
+}
+''')
+    libdir = os.path.dirname(rs._build.LIB)
+    exe = tmp_path / "c_abi"
+    subprocess.run([gcc, "-std=c11", "-Wall", "-Werror", "-I", os.path.join(ROOT, "include"),
+                    str(src), "-o", str(exe), "-L", libdir, "-lresispec",
+                    f"-Wl,-rpath,{libdir}"], check=True)
+    out = subprocess.run([str(exe)], capture_output=True, text=True, check=True).stdout.split()
+    assert out == ["3", "1", "1"]

@@ -28,6 +28,9 @@ import numpy as np
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
 _SRC = os.path.join(_HERE, "resispec_oracle.c")
+# tolerance machinery for proxy-denominator rows, kept apart from the walk
+_SRC_ERR = os.path.join(_HERE, "fp32_error_bound.c")
+_SOURCES = (_SRC, _SRC_ERR, os.path.join(_HERE, "fp32_error_bound.h"))
 _LIBDIR = os.path.join(_HERE, "_lib")
 _LIB = os.path.join(_LIBDIR, "libresispec_oracle.so")
 
@@ -53,11 +56,11 @@ def build(force: bool = False) -> str:
     """Compile the oracle with gcc (no -ffast-math, no FMA contraction)."""
     os.makedirs(_LIBDIR, exist_ok=True)
     if (not force and os.path.exists(_LIB)
-            and os.path.getmtime(_LIB) >= os.path.getmtime(_SRC)):
+            and all(os.path.getmtime(_LIB) >= os.path.getmtime(f) for f in _SOURCES)):
         return _LIB
     tmp = _LIB + f".tmp{os.getpid()}"
     cmd = ["gcc", "-O2", "-std=c11", "-fPIC", "-shared", "-pthread",
-           "-ffp-contract=off", "-fno-fast-math", "-o", tmp, _SRC, "-lm"]
+           "-ffp-contract=off", "-fno-fast-math", "-o", tmp, _SRC, _SRC_ERR, "-lm"]
     subprocess.run(cmd, check=True)
     os.replace(tmp, _LIB)
     return _LIB
@@ -129,6 +132,12 @@ def load():
             lib.oracle_sample.argtypes = [ctypes.c_void_p, ctypes.c_int,
                                           ctypes.c_double, ctypes.c_void_p]
             lib.oracle_sample.restype = ctypes.c_int
+            lib.oracle_fp32err_init.argtypes = [ctypes.c_void_p, ctypes.c_int, ctypes.c_void_p]
+            lib.oracle_fp32err_init.restype = None
+            lib.oracle_fp32err_reject.argtypes = [ctypes.c_void_p] * 4 + [
+                ctypes.c_int, ctypes.c_int, ctypes.c_double, ctypes.c_double, ctypes.c_double,
+                ctypes.c_void_p, ctypes.c_void_p]
+            lib.oracle_fp32err_reject.restype = None
             lib.oracle_args_size.restype = ctypes.c_int
             if lib.oracle_args_size() != ctypes.sizeof(_Args):
                 raise RuntimeError("oracle_args layout mismatch")
@@ -203,6 +212,26 @@ def reject(mode: int, R, q, x0: int, check: bool = True, z_rule: int = 0,
     return R, bool(changed), float(err[0])
 
 
+def fp32_error_init(v):
+    """Bounds of the rounding of fp32 tempered softmax values v (tolerance
+    machinery of proxy-denominator rows, ``fp32_error_bound.c``)."""
+    v = _f64(v)
+    e = np.zeros_like(v)
+    load().oracle_fp32err_init(v.ctypes.data, v.size, e.ctypes.data)
+    return e
+
+
+def fp32_error_reject(R, D, r, K, x0, Z, level, mu, eR, eD):
+    """One rejection's propagation of the bounds (eR, eD) of R and D
+    (``fp32_error_bound.c``); returns the bounds of R' = r / sum r and D' = K."""
+    R, D, r, K = _f64(R), _f64(D), _f64(r), _f64(K)
+    eR, eD = _f64(eR).copy(), _f64(eD).copy()
+    load().oracle_fp32err_reject(R.ctypes.data, D.ctypes.data, r.ctypes.data, K.ctypes.data,
+                                 R.size, int(x0), float(Z), float(level), float(mu),
+                                 eR.ctypes.data, eD.ctypes.data)
+    return eR, eD
+
+
 def sample(R, u: float):
     """Inverse-CDF draw -> (token, relative margin)."""
     R = _f64(R)
@@ -214,7 +243,7 @@ def sample(R, u: float):
 # ---------------------------------------------------------------- full walk
 def verify(target, draft, parents, cand, temperature, seed, *, mode=MODE_RESISPEC,
            max_depth=None, seq_stride=None, seq_ids=None, nthreads=None,
-           check_invariants=False, decide_fp64=False, want_dist=False, z_rule=0,
+           check_invariants=False, decide_fp64=True, want_dist=False, z_rule=0,
            denom_update=False, draft_children=False, fill=0, want_dist_err=False):
     """Run the oracle walk.
 
@@ -223,6 +252,9 @@ def verify(target, draft, parents, cand, temperature, seed, *, mode=MODE_RESISPE
     one set of rows across all B sequences, in which case ``cand`` gives B).
     ``parents``: int32 [N] (one tree for every sequence) or [B, N] (a tree
     per sequence); ``cand``: int32 [B, N].
+    ``decide_fp64``: every accept test is the paper's u < R(x)/D(x) in fp64
+    (Algorithm 1); False takes it as u * D(x) < R(x) on values rounded to
+    fp32, a diagnostic of how a single-precision evaluation decides.
     ``want_dist_err``: also return "dist_err" [B, V], a first-order bound of
     the error of an fp32 evaluation of "dist" for rows whose test
     denominator is the proxy (``denom_update``; reading R11), 0 elsewhere.

@@ -81,15 +81,19 @@
  *       level's response to Z and the normaliser), starting from the
  *       rounding of fp32 tempered softmax values; it is test infrastructure
  *       that widens the parity tolerance only where the arithmetic does.
- *   R6  the accept decision is taken in fp32, the kernel's precision
- *       (u * q(x) < R(x) with both operands rounded to fp32); the margin
- *       |u - R/q| is reported in fp64 for near-tie accounting.
+ *   R6  the accept decision is the paper's test u < R(x) / D(x) in fp64
+ *       (decide_fp64 = 1, what the Python wrapper passes by default);
+ *       decide_fp64 = 0 takes it as u * D(x) < R(x) on operands rounded to
+ *       fp32, a diagnostic only.  The margin |u - R/D| is reported in fp64
+ *       for near-tie accounting.
  */
 #include <math.h>
 #include <pthread.h>
 #include <stdint.h>
 #include <stdlib.h>
 #include <string.h>
+
+#include "fp32_error_bound.h"
 
 #define OR_MODE_RESISPEC 0
 #define OR_MODE_SPECINFER 1
@@ -438,91 +442,11 @@ int oracle_sample(const double* R, int V, double u, double* margin) {
 }
 
 /* ------------------------------------------------------------------ */
-/* First-order absolute error bounds of an fp32 evaluation (R11).  Units:
- * probabilities; EPS is fp32's unit roundoff. */
-static const double ERR_EPS = 5.9604644775390625e-08; /* 2^-24 */
-
-/* Rounding of an fp32 tempered softmax value 2^a / S, a = log2(v / max v):
- * the exponent's argument is rounded relative to |a|, plus a few roundings
- * of the exponential and the normaliser. */
-static void err_init(const double* v, int V, double* e) {
-  double mx = 0.0;
-  for (int i = 0; i < V; ++i)
-    if (v[i] > mx) mx = v[i];
-  for (int i = 0; i < V; ++i)
-    e[i] = v[i] > 0.0 ? v[i] * ERR_EPS * (4.0 + 0.7 * fabs(log2(v[i] / mx))) : 0.0;
-}
-
-/* Bounds of m = min(level D, R) and t = R - m at one token (R > 0, not x0). */
-static void err_min(double R, double D, double eR, double eD, double level, double* m,
-                    double* em, double* t, double* et) {
-  const double lD = level == INFINITY ? (D > 0.0 ? INFINITY : 0.0) : level * D;
-  const double le = level == INFINITY ? 0.0 : level * eD;
-  *m = fmin(lD, R);
-  if (fabs(R - lD) <= eR + le + ERR_EPS * R)
-    *em = fmax(eR, le) + ERR_EPS * R; /* either side of the min */
-  else
-    *em = (lD < R) ? le + ERR_EPS * *m : eR;
-  *t = R - *m;
-  *et = eR + *em + ERR_EPS * *t;
-}
-
-/* Carries the bounds (eR, eD) of R and D through one ResiSpec rejection of
- * x0 (R, D before; r, K after; budget Z, level, fill fraction mu) and leaves
- * the bounds of R' = r / sum r and D' = K in (eR, eD). */
-static void err_reject(const double* R, const double* D, const double* r, const double* K, int V,
-                       int x0, double Z, double level, double mu, double* eR, double* eD) {
-  double S = 0.0, slope = 0.0, sum_t = 0.0, sum_em = 0.0, sum_et = 0.0;
-  for (int i = 0; i < V; ++i) {
-    S += r[i];
-    if (i == x0 || R[i] == 0.0) continue;
-    double m, em, t, et;
-    err_min(R[i], D[i], eR[i], eD[i], level, &m, &em, &t, &et);
-    sum_t += t;
-    sum_em += em;
-    sum_et += et;
-    if (level != INFINITY && level * D[i] < R[i]) slope += D[i];
-  }
-  if (!(S > 0.0)) return;
-  const double eZ = eD[x0] + eR[x0] + ERR_EPS * Z;
-  /* mu = (Z - sum m) / sum t: its numerator may cancel */
-  const double emu = mu > 0.0 && sum_t > 0.0
-                         ? (eZ + sum_em + ERR_EPS * Z) / sum_t + mu * sum_et / sum_t
-                         : 0.0;
-  double er_sum = 0.0;
-  for (int i = 0; i < V; ++i) {
-    double er, eK;
-    if (i == x0 || R[i] == 0.0) {
-      er = 0.0; /* taken out exactly; a rejected token stays at 0 */
-      eK = (i == x0) ? eD[i] : 0.0;
-    } else {
-      double m, em, t, et;
-      err_min(R[i], D[i], eR[i], eD[i], level, &m, &em, &t, &et);
-      er = em + mu * et + emu * t + ERR_EPS * r[i];
-      eK = (1.0 - mu) * et + emu * t + ERR_EPS * K[i];
-    }
-    eR[i] = er; /* bound of r for now */
-    eD[i] = eK;
-    er_sum += er;
-  }
-  /* the level's response to an error in Z moves the tokens below it
-     together: relative dZ / (mass below the level) on them, dZ / Z on all */
-  const double below = (level == INFINITY) ? 0.0 : level * slope;
-  for (int i = 0; i < V; ++i) {
-    const double Rn = r[i] / S;
-    double e = eR[i] / S + Rn * (er_sum / S + eZ / Z);
-    if (i != x0 && R[i] > 0.0 && below > 0.0 && level != INFINITY && level * D[i] < R[i])
-      e += Rn * eZ / below;
-    eR[i] = e;
-  }
-}
-
-/* ------------------------------------------------------------------ */
 typedef struct {
   int32_t B, N, V, D;
   int32_t dtype;
   int32_t mode;
-  int32_t decide_fp64; /* 1: literal fp64 test u < R/D instead of R6 */
+  int32_t decide_fp64; /* 1: the fp64 test u < R/D (R6); 0: fp32 diagnostic */
   int32_t check_invariants;
   int32_t nthreads;
   int32_t pad_;
@@ -648,8 +572,8 @@ static void verify_sequence(const oracle_args* a, int lb, int tree_bad,
     }
     const int track = a->out_dist_err != NULL && Dn == Dbuf; /* R11 */
     if (track) {
-      err_init(p, V, eR);
-      err_init(q, V, eD);
+      fp32err_init(p, V, eR);
+      fp32err_init(q, V, eD);
     }
     cond = 1.0;
     int accepted = -1;
@@ -684,7 +608,7 @@ static void verify_sequence(const oracle_args* a, int lb, int tree_bad,
                        &level, &mu)) {
         status |= OR_INFO_DEGENERATE;
       } else if (Dn == Dbuf) {
-        if (track) err_reject(Rb, Dbuf, r, K, V, x, Zj, level, mu, eR, eD);
+        if (track) fp32err_reject(Rb, Dbuf, r, K, V, x, Zj, level, mu, eR, eD);
         memcpy(Dbuf, K, sizeof(double) * V);
       }
       cond /= norm;

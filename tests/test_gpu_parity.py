@@ -36,7 +36,8 @@ def _check(inp, mode, seed, **kw):
     o = P.run_oracle(inp["target"], inp["draft"], inp["parents"], inp["cand"],
                      inp["temperature"], seed, D, mode, z_rule=kw.get("z_rule", 0),
                      denom_update=kw.get("proxy_denominator", False), fill=kw.get("fill", 0))
-    n, near = P.compare(g, o)
+    rep = P.compare(g, o)
+    n, near = rep["sequences"], rep["mismatch_in_ties"]
     # near-tie differences are allowed but must stay rare
     assert near <= max(2, 0.002 * n), (near, n)
     assert g["status"][0] & ~rs.INFO_DEGENERATE == 0
@@ -321,8 +322,8 @@ def _sampled_parity(w, seed, call_seed, rows, mode=rs.MODE_RESISPEC, batch=None,
     o = P.run_oracle(th, dh, pa, ch, w.temperature, call_seed, D, mode,
                      seq_ids=np.asarray(rows, np.int32), z_rule=kw.get("z_rule", 0),
                      denom_update=kw.get("proxy_denominator", False), fill=kw.get("fill", 0))
-    n, near = P.compare(g, o, rows=rows)
-    assert near <= 1, near
+    rep = P.compare(g, o, rows=rows)
+    assert rep["mismatch_in_ties"] <= 1, rep
     assert g["status"][0] & ~rs.INFO_DEGENERATE == 0
     assert (g["accept_len"] >= 0).all()
     del inp
@@ -348,21 +349,37 @@ def test_parity_binary5_specinfer_full_size(kernel):
                     kernel=kernel)
 
 
+def _spread_rows(B, n):
+    """n sequence indices spread over a batch of B (first and last included)."""
+    return sorted({int(round(i * (B - 1) / (n - 1))) for i in range(n)})
+
+
+@pytest.mark.parametrize("B", [32, 128])
+@pytest.mark.parametrize("k", [2, 4, 8, 16])
+def test_parity_single_position_v256000(k, B):
+    """Single position with k candidates, V = 256000 bf16, at the batch and
+    in the launch shape the benchmark times; 8 sampled sequences."""
+    w = W.WORKLOADS[f"single-k{k}-v256000-b{B}"]
+    _sampled_parity(w, seed=40 + k + B, call_seed=77 + k, rows=_spread_rows(B, 8))
+
+
 @pytest.mark.parametrize("kernel", KERNELS)
-@pytest.mark.parametrize("k", [2, 16])
-def test_parity_single_position_v256000(k, kernel):
-    w = W.WORKLOADS[f"single-k{k}-v256000-b32"]
-    _sampled_parity(w, seed=40 + k, call_seed=77, rows=[0, 7, 15, 31], kernel=kernel)
+def test_parity_single_position_v256000_kernels(kernel):
+    w = W.WORKLOADS["single-k16-v256000-b32"]
+    _sampled_parity(w, seed=45, call_seed=79, rows=[0, 7, 15, 31], kernel=kernel)
 
 
-def test_parity_single_position_v256000_b128():
-    """B = 128, k = 16, in the launch shape the benchmark times."""
-    w = W.WORKLOADS["single-k16-v256000-b128"]
-    _sampled_parity(w, seed=45, call_seed=79, rows=[0, 33, 64, 97, 127])
+@pytest.mark.parametrize("B", [32, 128])
+def test_parity_tree488_v256000(B):
+    """Tree [8, 4, 2, 2, 1, 1] (488 nodes), V = 256000 bf16, the whole batch
+    (B = 128: 64 GB of logits) in the launch shape the benchmark times;
+    6 sampled sequences."""
+    w = W.WORKLOADS[f"tree488-v256000-b{B}"]
+    _sampled_parity(w, seed=50 + B, call_seed=78, rows=_spread_rows(B, 6))
 
 
 @pytest.mark.parametrize("kernel", KERNELS)
-def test_parity_tree488_v256000(kernel):
+def test_parity_tree488_v256000_kernels(kernel):
     w = W.WORKLOADS["tree488-v256000-b32"]
     _sampled_parity(w, seed=50, call_seed=78, rows=[0, 5], batch=6, kernel=kernel)
 
@@ -703,7 +720,8 @@ def _check_drafting(inp, mode, seed, **kw):
                       inp["temperature"], seed, mode=mode, max_depth=D, want_dist=True,
                       draft_children=True)
     o["sample_margin"] = np.minimum(o["sample_margin"], o["draft_margin"])
-    n, near = P.compare(g, o)
+    rep = P.compare(g, o)
+    n, near = rep["sequences"], rep["mismatch_in_ties"]
     assert near <= max(2, 0.01 * n), (near, n)
     gd = drafted.cpu().numpy()
     clean = (o["accept_margin"] > P.ACCEPT_TIE) & (o["sample_margin"] > P.SAMPLE_TIE)

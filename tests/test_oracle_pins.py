@@ -373,3 +373,25 @@ def test_z_applied_equals_algorithm1_when_capacity_bound_is_below_gap():
         b = oracle.reject(oracle.MODE_RESISPEC, R, q, x0, z_rule=1)[0]
         np.testing.assert_array_equal(a, b)
     assert seen > 100
+
+
+def test_golden_fp32_error_bound_two_rejections():
+    """The fp32 error bound of proxy-denominator rows (reading R11,
+    oracle/fp32_error_bound.c) through two rejections, against the bound
+    worked by hand in tests/golden/fp32_error_bound_v3.json (inputs there are
+    exact GetProxy results, checked here against the oracle's GetProxy)."""
+    g = json.load(open(os.path.join(GOLDEN, "fp32_error_bound_v3.json")))
+    eps = 2.0 ** -24
+    eR = oracle.fp32_error_init(g["p"])
+    eD = oracle.fp32_error_init(g["q"])
+    np.testing.assert_allclose(eR / eps, g["eR_init"], rtol=1e-12)
+    np.testing.assert_allclose(eD / eps, g["eD_init"], rtol=1e-12)
+    for j, rj in enumerate(g["rejections"], start=1):
+        k, r, Z = oracle.get_proxy(rj["R"], rj["D"], rj["x0"])
+        np.testing.assert_allclose(r, rj["r"], atol=1e-15)
+        np.testing.assert_allclose(k, rj["K"], atol=1e-15)
+        assert abs(Z - rj["Z"]) < 1e-15
+        eR, eD = oracle.fp32_error_reject(rj["R"], rj["D"], rj["r"], rj["K"], rj["x0"], rj["Z"],
+                                          rj["level"], rj["mu"], eR, eD)
+        np.testing.assert_allclose(eR / eps, g[f"eR_after_{j}"], rtol=1e-9, atol=1e-9)
+        np.testing.assert_allclose(eD / eps, g[f"eD_after_{j}"], rtol=1e-9, atol=1e-9)

@@ -40,7 +40,7 @@
 extern "C" {
 #endif
 
-#define RESISPEC_ABI_VERSION 3
+#define RESISPEC_ABI_VERSION 4
 
 /* Synchronous return codes. */
 typedef enum {
@@ -139,13 +139,15 @@ typedef struct {
  *   RESIDENT: both rows of the sequence's vocabulary slice stay in the
  *     shared memory of the cluster's CTAs as fp32 (8 bytes per vocabulary
  *     entry per sequence), so only as many sequences as fit on chip run at
- *     once.  Any fan-out.
+ *     once.  Any fan-out.  RESISPEC mode only (SPECINFER with
+ *     RESISPEC_FLAG_RESIDENT: RESISPEC_E_ARG).
  *   STREAM: nothing but per-sequence scalars stays on chip; every pass
  *     streams the rows from global memory (the passes after a visit's first
- *     read them from L2).  All sequences of a large batch run at once.
- *     Fan-out up to RESISPEC_MAX_FANOUT_STREAM children per node.
- * The automatic choice takes RESIDENT when the whole batch fits on chip at
- * once, else STREAM. */
+ *     read them from L2, or from shared memory when a CTA's slice fits its
+ *     copy ring).  All sequences of a large batch run at once.  Fan-out up
+ *     to RESISPEC_MAX_FANOUT_STREAM children per node.
+ * The automatic choice is STREAM (measured as fast or faster at every batch
+ * size); RESIDENT runs when RESISPEC_FLAG_RESIDENT asks for it. */
 #define RESISPEC_KERNEL_RESIDENT 0
 #define RESISPEC_KERNEL_STREAM 1
 
@@ -223,8 +225,12 @@ typedef struct {
   int32_t block_threads;   /* threads per CTA */
   int32_t smem_bytes;      /* dynamic shared memory per CTA */
   int32_t slice_elems;     /* vocabulary entries per CTA */
-  int32_t uses_tma;        /* 1 if rows are fetched with bulk copies */
-  int32_t reserved;        /* 0 */
+  int32_t uses_tma;        /* 1 if rows are fetched with bulk (TMA) copies: the
+                              resident kernel on 16-byte aligned rows */
+  int32_t vector_loads;    /* 1 if rows move in 16-byte vectors (bulk copies in
+                              the resident kernel, per-thread asynchronous
+                              16-byte copies in the streaming kernel), 0 if
+                              element by element (rows not 16-byte aligned) */
   int32_t active_clusters; /* clusters of this shape resident at once on the
                               current device (0 without a device) */
 } resispec_plan_info;

@@ -84,7 +84,7 @@ class Opts(ctypes.Structure):
 class PlanInfo(ctypes.Structure):
     _fields_ = [(n, ctypes.c_int32) for n in (
         "kernel", "cluster_size", "block_threads", "smem_bytes", "slice_elems", "uses_tma",
-        "reserved", "active_clusters")]
+        "vector_loads", "active_clusters")]
 
 
 class ResispecError(RuntimeError):

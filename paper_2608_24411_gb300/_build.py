@@ -12,7 +12,8 @@ HEADER = os.path.join(os.path.dirname(HERE), "include", "resispec.h")
 UNITS = ("resispec.cu", "kern_resident_f32.cu", "kern_resident_bf16.cu", "kern_stream_f32.cu",
          "kern_stream_bf16.cu", "kern_stream_var_f32.cu", "kern_stream_var_bf16.cu")
 SOURCES = [os.path.join(CSRC, f) for f in UNITS + ("kernels.h", "verify_kernel.cuh",
-                                                   "verify_stream.cuh", "philox.cuh", "ptx.cuh")]
+                                                   "verify_stream.cuh", "specinfer.cuh",
+                                                   "dfloat.cuh", "philox.cuh", "ptx.cuh")]
 
 
 def nvcc() -> str:

@@ -76,6 +76,8 @@ struct VerifyParams {
   int64_t parents_stride;  // elements between sequences' trees (0: one tree)
   uint64_t seed;
   float scale_log2;    // log2(e) / T
+  float scale_log2_lo; // log2(e) / T - scale_log2, rounded (SpecInfer instance)
+  float exp2_tab[65][2];  // 2^(j / 64), j = -32 .. 32, as double-floats (SpecInfer instance)
   int32_t B, N, V, D;
   int32_t slice;       // L, elements per CTA (multiple of 8)
   int32_t npad;        // padded node count of the tree arrays
@@ -109,7 +111,8 @@ static_assert(sizeof(Head) <= kHeadBytes, "head too large");
 
 // ---------------------------------------------------------------- residual map
 // kScale: R = w * sc with the per-thread scale sc (sc = 1 once R is materialised
-// and no map is pending); kResi: GetProxy residual; kSpec: Eq. recur.
+// and no map is pending); kResi: GetProxy residual; kSpec: the streaming
+// kernel's SpecInfer residual (its sampler masses only).
 enum : int { kScale = 0, kResi = 1, kSpec = 2 };
 
 struct Pending {
@@ -128,25 +131,19 @@ __device__ __forceinline__ float apply_map(const Pending& P, float w, float qq, 
                                            float sc) {
   if constexpr (KIND == kScale) {
     return __fmul_rn(w, sc);
-  } else if constexpr (KIND == kResi) {
+  } else {
     // GetProxy: r = min(Z q, R) + lambda (R - min(Z q, R)) off x0, r(x0) = 0;
     // R' = r / sum r.
     if (idx == P.x0) return 0.f;
     const float m = fminf(__fmul_rn(P.Z, qq), w);
     return __fmul_rn(__fmaf_rn(P.lam, __fsub_rn(w, m), m), P.a);
-  } else {
-    // Eq. recur: R' = (R - q)_+ / sum.
-    return __fmul_rn(fmaxf(__fsub_rn(w, qq), 0.f), P.a);
   }
 }
 
 __device__ __forceinline__ float apply_any(const Pending& P, float w, float qq, int idx,
                                            float sc) {
-  switch (P.kind) {
-    case kScale: return apply_map<kScale>(P, w, qq, idx, sc);
-    case kResi: return apply_map<kResi>(P, w, qq, idx, sc);
-    default: return apply_map<kSpec>(P, w, qq, idx, sc);
-  }
+  return P.kind == kScale ? apply_map<kScale>(P, w, qq, idx, sc)
+                          : apply_map<kResi>(P, w, qq, idx, sc);
 }
 
 // 2^(m - M) / S for a stored reference m in log2 units (0 when m = -inf).
@@ -164,8 +161,6 @@ __device__ __forceinline__ float group_sum(float v) {
   for (int o = 1 << (LEVELS - 1); o; o >>= 1) v = __fadd_rn(v, __shfl_xor_sync(0xffffffffu, v, o));
   return v;
 }
-
-__device__ __forceinline__ float warp_sum(float v) { return group_sum<5>(v); }
 
 // (reference, sum of 2^(z c - reference)) pairs, references in log2 units:
 // the common reference is the warp maximum (one redux), each lane rescales
@@ -511,11 +506,11 @@ struct RowNorm {
 };
 
 // One rejection pass: materialise R_j = map(W) into W and accumulate the
-// sums of rejection j (ResiSpec: sum min(Z q, R) and sum (R - min(Z q, R))
-// over x != x0; SpecInfer: sum (R - q)_+), publishing token xn's values.
+// sums of rejection j (sum min(Z q, R) and sum (R - min(Z q, R)) over
+// x != x0), publishing token xn's values.
 // Per-element index tests are needed only in the (at most three) vectors
 // that hold x0, xn or the previous map's x0.
-template <int VEC, int KIND, bool RESI, bool CHECK>
+template <int VEC, int KIND, bool CHECK>
 __device__ __forceinline__ void reject_vector(float (&w)[VEC], const float (&q)[VEC], int base,
                                               const Pending& P, float at, float bt, float mt,
                                               float md, int x0, float Z, int xn, float& t1,
@@ -533,19 +528,15 @@ __device__ __forceinline__ void reject_vector(float (&w)[VEC], const float (&q)[
     }
     if (CHECK && idx == xn) { pubv[0] = R; pubv[1] = mt; pubv[2] = q[j]; pubv[3] = md; }
     w[j] = R;
-    if constexpr (RESI) {
-      if (!CHECK || idx != x0) {
-        const float m = fminf(__fmul_rn(Z, qq), R);
-        t1 += m;
-        t2 += __fsub_rn(R, m);
-      }
-    } else {
-      t1 += fmaxf(__fsub_rn(R, qq), 0.f);
+    if (!CHECK || idx != x0) {
+      const float m = fminf(__fmul_rn(Z, qq), R);
+      t1 += m;
+      t2 += __fsub_rn(R, m);
     }
   }
 }
 
-template <int THREADS, bool BF16, int KIND, bool RESI>
+template <int THREADS, bool BF16, int KIND>
 __device__ __forceinline__ void reject_pass(float* W, const float* Q, int L, int lo,
                                             const Pending& P, float at, float bt, float mt,
                                             float md, int x0, float Z, int xn, float* pubv,
@@ -567,11 +558,11 @@ __device__ __forceinline__ void reject_pass(float* W, const float* Q, int L, int
     }
     float t1 = 0.f, t2 = 0.f;
     if (g == s0 || g == s1 || g == s2)
-      reject_vector<VEC, KIND, RESI, true>(w, q, lo + g * VEC, P, at, bt, mt, md, x0, Z, xn, t1,
-                                           t2, pubv);
+      reject_vector<VEC, KIND, true>(w, q, lo + g * VEC, P, at, bt, mt, md, x0, Z, xn, t1, t2,
+                                     pubv);
     else
-      reject_vector<VEC, KIND, RESI, false>(w, q, lo + g * VEC, P, at, bt, mt, md, x0, Z, xn,
-                                            t1, t2, pubv);
+      reject_vector<VEC, KIND, false>(w, q, lo + g * VEC, P, at, bt, mt, md, x0, Z, xn, t1, t2,
+                                      pubv);
     s1sum += t1;
     s2sum += t2;
 #pragma unroll
@@ -583,20 +574,16 @@ __device__ __forceinline__ void reject_pass(float* W, const float* Q, int L, int
   s2out = s2sum;
 }
 
-// A ResiSpec pass follows either the normaliser scale or a ResiSpec map; a
-// SpecInfer pass either the scale or a SpecInfer map.
-template <int THREADS, bool BF16, bool RESI>
+// A rejection pass follows either the normaliser scale or a ResiSpec map.
+template <int THREADS, bool BF16>
 __device__ __forceinline__ void reject_pass_any(float* W, const float* Q, int L, int lo,
                                                 const Pending& P, float at, float bt, float mt,
                                                 float md, int x0, float Z, int xn, float* pubv,
                                                 float& s1, float& s2) {
-  constexpr int MAPPED = RESI ? kResi : kSpec;
   if (P.kind == kScale)
-    reject_pass<THREADS, BF16, kScale, RESI>(W, Q, L, lo, P, at, bt, mt, md, x0, Z, xn, pubv, s1,
-                                             s2);
+    reject_pass<THREADS, BF16, kScale>(W, Q, L, lo, P, at, bt, mt, md, x0, Z, xn, pubv, s1, s2);
   else
-    reject_pass<THREADS, BF16, MAPPED, RESI>(W, Q, L, lo, P, at, bt, mt, md, x0, Z, xn, pubv, s1,
-                                             s2);
+    reject_pass<THREADS, BF16, kResi>(W, Q, L, lo, P, at, bt, mt, md, x0, Z, xn, pubv, s1, s2);
 }
 
 // ---------------------------------------------------------------- sampler
@@ -809,6 +796,10 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 3)
   float* u_acc = reinterpret_cast<float*>(cand_s + P.npad);  // [r]: accept test of node r - 1
   float* u_fin = u_acc + P.npad;                             // [r]: final draw at row r
 
+  // Nothing is read before the preceding work on the stream has completed;
+  // the next launch may be scheduled from here on (it waits the same way).
+  grid_dependency_wait();
+  grid_launch_dependents();
   const int tid = threadIdx.x;
   const uint32_t rank = cluster_ctarank();
   const uint32_t C = cluster_nctarank();
@@ -938,60 +929,44 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 3)
       const int nxt = next_sib[cn];
       const int xn = nxt >= 0 ? cand_s[nxt] : -1;
       float s1 = 0.f, s2 = 0.f;
-      if (P.mode == 0) {
-        const float Z = __fsub_rn(qx, Rx);
-        if (!(Z > 0.f)) {
-          // degenerate rejection: keep R, fetch the next candidate's values
-          info |= kInfoDegenerate;
-          if (xn >= lo && xn < lo + nloc && ((xn - lo) / VEC) % THREADS == tid) {
-            H.pubv[0] = W[xn - lo];
-            H.pubv[1] = mref_t;
-            H.pubv[2] = Q[xn - lo];
-            H.pubv[3] = mref_d;
-          }
-          exchange<NW, false>(H, 0.f, 0.f, 0.f, 0.f, 0, owner_of(xn), xp, xph, rank, C, o,
-                              oflags);
-          if (oflags & kFlagTimeout) { err |= kErrTimeout; break; }
-          pub[0] = o[4]; pub[1] = o[5]; pub[2] = o[6]; pub[3] = o[7];
-          mass_kind = 0;
-          cn = nxt;
-          continue;
+      // ResiSpec rejection (Algorithm 1, GetProxy); SpecInfer runs on the
+      // streaming kernel
+      const float Z = __fsub_rn(qx, Rx);
+      if (!(Z > 0.f)) {
+        // degenerate rejection: keep R, fetch the next candidate's values
+        info |= kInfoDegenerate;
+        if (xn >= lo && xn < lo + nloc && ((xn - lo) / VEC) % THREADS == tid) {
+          H.pubv[0] = W[xn - lo];
+          H.pubv[1] = mref_t;
+          H.pubv[2] = Q[xn - lo];
+          H.pubv[3] = mref_d;
         }
-        reject_pass_any<THREADS, BF16, true>(W, Q, L, lo, Pm, at, bt, mref_t, mref_d, x, Z, xn,
-                                             H.pubv, s1, s2);
-        exchange<NW, false>(H, s1, s2, 0.f, 0.f, 0, owner_of(xn), xp, xph, rank, C, o,
+        exchange<NW, false>(H, 0.f, 0.f, 0.f, 0.f, 0, owner_of(xn), xp, xph, rank, C, o,
                             oflags);
         if (oflags & kFlagTimeout) { err |= kErrTimeout; break; }
-        const float S1 = o[0], S2 = o[1];
-        const float delta = __fsub_rn(Z, S1);
-        const float lam = S2 > 0.f ? fminf(fmaxf(__fdiv_rn(delta, S2), 0.f), 1.f) : 0.f;
-        const float norm = __fmaf_rn(lam, S2, S1);
-        if (norm > 0.f) {
-          Pm = Pending{kResi, x, __frcp_rn(norm), Z, lam};
-          mass_kind = 2;
-        } else {  // R_j is materialised in W: continue from it unchanged
-          Pm = Pending{kScale, -1, 1.f, 0.f, 0.f};
-          at = 1.f;
-          ident = true;
-          info |= kInfoDegenerate;
-          mass_kind = 0;
-        }
-      } else {
-        reject_pass_any<THREADS, BF16, false>(W, Q, L, lo, Pm, at, bt, mref_t, mref_d, x, 0.f,
-                                              xn, H.pubv, s1, s2);
-        exchange<NW, false>(H, s1, s2, 0.f, 0.f, 0, owner_of(xn), xp, xph, rank, C, o,
-                            oflags);
-        if (oflags & kFlagTimeout) { err |= kErrTimeout; break; }
-        if (o[0] > 0.f) {
-          Pm = Pending{kSpec, -1, __frcp_rn(o[0]), 0.f, 0.f};
-          mass_kind = 3;
-        } else {  // R_j is materialised in W: continue from it unchanged
-          Pm = Pending{kScale, -1, 1.f, 0.f, 0.f};
-          at = 1.f;
-          ident = true;
-          info |= kInfoDegenerate;
-          mass_kind = 0;
-        }
+        pub[0] = o[4]; pub[1] = o[5]; pub[2] = o[6]; pub[3] = o[7];
+        mass_kind = 0;
+        cn = nxt;
+        continue;
+      }
+      reject_pass_any<THREADS, BF16>(W, Q, L, lo, Pm, at, bt, mref_t, mref_d, x, Z, xn, H.pubv,
+                                     s1, s2);
+      exchange<NW, false>(H, s1, s2, 0.f, 0.f, 0, owner_of(xn), xp, xph, rank, C, o,
+                          oflags);
+      if (oflags & kFlagTimeout) { err |= kErrTimeout; break; }
+      const float S1 = o[0], S2 = o[1];
+      const float delta = __fsub_rn(Z, S1);
+      const float lam = S2 > 0.f ? fminf(fmaxf(__fdiv_rn(delta, S2), 0.f), 1.f) : 0.f;
+      const float norm = __fmaf_rn(lam, S2, S1);
+      if (norm > 0.f) {
+        Pm = Pending{kResi, x, __frcp_rn(norm), Z, lam};
+        mass_kind = 2;
+      } else {  // R_j is materialised in W: continue from it unchanged
+        Pm = Pending{kScale, -1, 1.f, 0.f, 0.f};
+        at = 1.f;
+        ident = true;
+        info |= kInfoDegenerate;
+        mass_kind = 0;
       }
       pub[0] = o[4]; pub[1] = o[5]; pub[2] = o[6]; pub[3] = o[7];
       cn = nxt;

@@ -34,6 +34,7 @@
 #pragma once
 #include <type_traits>
 
+#include "specinfer.cuh"
 #include "verify_kernel.cuh"
 
 namespace rs {
@@ -48,35 +49,38 @@ constexpr int kMaxKids = kMaxMaps;      // children per node the streaming kerne
 static_assert(2 * kMaxKids <= 256, "per-visit loads and draws use distinct threads of a CTA");
 constexpr int kErrFanout = 64;
 
-// Residual maps are kept in unnormalised units.  With p~ = 2^(z_t c - M_t)
-// and q~ = 2^(z_d c - M_d) (so p = p~ / S_t, q = q~ / S_d), the residual
-// after i maps is R_i = sigma_i R~_i, R~_0 = p~, sigma_0 = 1 / S_t, and map
-// i (Z_i, lambda_i, normaliser 1 / a_i) becomes, element-wise,
-//   ResiSpec:  m = min(k_i q~, R~), R~' = m + lambda_i (R~ - m),
-//   SpecInfer: R~' = (R~ - k_i q~)_+,
-// with k_i = Z_i / (S_d sigma_{i-1}) (ResiSpec) or 1 / (S_d sigma_{i-1})
-// (SpecInfer) and sigma_i = sigma_{i-1} a_i: every scale is folded into the
-// per-map scalar k_i and the running factor sigma.  The ResiSpec form keeps
+// ResiSpec residual maps are kept in unnormalised units.  With
+// p~ = 2^(z_t c - M_t) and q~ = 2^(z_d c - M_d) (so p = p~ / S_t,
+// q = q~ / S_d), the residual after i maps is R_i = sigma_i R~_i, R~_0 = p~,
+// sigma_0 = 1 / S_t, and map i (Z_i, lambda_i, normaliser 1 / a_i) becomes,
+// element-wise, m = min(k_i q~, R~), R~' = m + lambda_i (R~ - m), with
+// k_i = Z_i / (S_d sigma_{i-1}) and sigma_i = sigma_{i-1} a_i: every scale is
+// folded into the per-map scalar k_i and the running factor sigma.  (The
+// SpecInfer recurrence needs no list of maps: specinfer.cuh.)  The form keeps
 // m (its minimum taken directly) and R~ - m separate: folding the map into
 // R~ - (1 - lambda_i)(R~ - m) would round 1 - lambda_i, an error that the
 // renormalisation by a small Z_i magnifies wherever m + lambda_i (R~ - m)
 // is much smaller than R~.  Maps are applied two lanes per instruction.
 struct __align__(16) StreamHead {
-  float2 map[kMaxMaps];  // {k_i, lambda_i} of map i (SpecInfer: {-k_i, 0})
+  float2 map[kMaxMaps];  // {k_i, lambda_i} of map i
   float mdsc[kMaxMaps];  // scale of the test denominator's D~ after map i
-  int rej[kMaxMaps];     // tokens whose residual is 0 (ResiSpec maps)
+  int rej[kMaxMaps];     // rejected tokens (ResiSpec: their residual is 0)
   int16_t rejk[kMaxMaps];  // their child index in this visit
   float kzt[kMaxKids];   // raw target / draft logits of the children's tokens
   float kzd[kMaxKids];
   float kua[kMaxKids];   // their accept draws U(seed, b, child + 1, 0)
   float ufin;            // the visit's final draw U(seed, b, row, 1)
   int nmaps;
+  // Chunk records of the pass that defines the visit's final distribution
+  // (see ChunkRec): two floats per (chunk, warp), chunk-major.
+  float crec[2][256];
   // optional phase counters (clock64 cycles, thread 0): see kPhase*
   unsigned long long phc[kPhases];
   unsigned long long ph_last;
   int ph_cur;
 };
-constexpr int kStreamHeadBytes = 4096;
+constexpr int kStreamHeadBytes = 6144;
+constexpr int kMaxChunkRecs = 256;  // (chunk, warp) records per CTA
 static_assert(sizeof(StreamHead) <= kStreamHeadBytes, "stream head too large");
 
 template <int THREADS, bool BF16>
@@ -110,6 +114,7 @@ struct Src {
   int rows;
   int nloc;
   bool vec;       // 16-byte aligned rows: vector loads
+  bool held;      // every chunk of these rows is in ring stage k (slice <= S chunks)
 };
 
 template <bool BF16>
@@ -159,10 +164,22 @@ __device__ __forceinline__ void load_pairs(const unsigned char* row, float2 (&z)
   }
 }
 
+// Ring layout of a pass: a pass over both rows keeps S stages of SB bytes
+// (target row, then draft row); a pass over the target row alone keeps 2 S
+// stages of RB bytes, twice as many chunks in flight.  Chunk k of a pass
+// lives in stage k mod DEPTH.
+template <int THREADS, bool BF16, bool TWO>
+struct Lay {
+  using G = StreamGeom<THREADS, BF16>;
+  static constexpr int DEPTH = TWO ? G::S : 2 * G::S;
+  static constexpr uint32_t STRIDE = TWO ? G::SB : G::RB;
+};
+
 // Copies this thread's vectors of chunk k into ring stage `st` (the copies
-// of one chunk form one cp.async group).  Aligned rows: 16-byte
-// asynchronous copies; other rows: element loads stored synchronously.
-template <int THREADS, bool BF16>
+// of one chunk form one cp.async group): the target row, and the draft row
+// RB bytes further when TWO.  Aligned rows: 16-byte asynchronous copies;
+// other rows: element loads stored synchronously.
+template <int THREADS, bool BF16, bool TWO>
 __device__ __forceinline__ void copy_chunk(const Src& s, int k, unsigned char* st) {
   using G = StreamGeom<THREADS, BF16>;
   constexpr int VEC = G::VEC;
@@ -178,10 +195,10 @@ __device__ __forceinline__ void copy_chunk(const Src& s, int k, unsigned char* s
       // nloc is a multiple of VEC on this path: a vector is whole or absent
       if (e0 < s.nloc) {
         cp_async16(dt, s.t + (size_t)e0 * es);
-        if (s.rows == 2) cp_async16(dd, s.d + (size_t)e0 * es);
+        if constexpr (TWO) cp_async16(dd, s.d + (size_t)e0 * es);
       } else {
         *dt = ninf;
-        *dd = ninf;
+        if constexpr (TWO) *dd = ninf;
       }
     } else {
       uint32_t wt[4], wd[4];
@@ -194,9 +211,8 @@ __device__ __forceinline__ void copy_chunk(const Src& s, int k, unsigned char* s
             const int e = e0 + 2 * i + j;
             const bool in = e < s.nloc;
             lt[j] = in ? (uint32_t)__ldg(reinterpret_cast<const uint16_t*>(s.t) + e) : 0xff80u;
-            ld[j] = (in && s.rows == 2)
-                        ? (uint32_t)__ldg(reinterpret_cast<const uint16_t*>(s.d) + e)
-                        : 0xff80u;
+            ld[j] = (TWO && in) ? (uint32_t)__ldg(reinterpret_cast<const uint16_t*>(s.d) + e)
+                                : 0xff80u;
           }
           wt[i] = lt[0] | (lt[1] << 16);
           wd[i] = ld[0] | (ld[1] << 16);
@@ -205,42 +221,49 @@ __device__ __forceinline__ void copy_chunk(const Src& s, int k, unsigned char* s
           const bool in = e < s.nloc;
           wt[i] = in ? __float_as_uint(__ldg(reinterpret_cast<const float*>(s.t) + e))
                      : 0xff800000u;
-          wd[i] = (in && s.rows == 2)
-                      ? __float_as_uint(__ldg(reinterpret_cast<const float*>(s.d) + e))
-                      : 0xff800000u;
+          wd[i] = (TWO && in) ? __float_as_uint(__ldg(reinterpret_cast<const float*>(s.d) + e))
+                              : 0xff800000u;
         }
       }
       *dt = make_uint4(wt[0], wt[1], wt[2], wt[3]);
-      *dd = make_uint4(wd[0], wd[1], wd[2], wd[3]);
+      if constexpr (TWO) *dd = make_uint4(wd[0], wd[1], wd[2], wd[3]);
     }
   }
   cp_async_commit();
 }
 
-// Streams the slice chunk by chunk, S - 1 chunks ahead, calling
-// body(target_stage_row, draft_stage_row, k) with all threads; body returns
-// true (uniformly) to end the pass.  pre() runs once, after the first copies
-// are issued.  On return every copy of the pass has landed.
-template <int THREADS, bool BF16, class Pre, class Body>
-__device__ __forceinline__ void stream_pass_pre(unsigned char* ring, const Src& s, Pre&& pre,
-                                                Body&& body) {
+// Chunk k's stage when the slice is held in the ring (see Src::held).
+template <int THREADS, bool BF16>
+__device__ __forceinline__ unsigned char* held_stage(unsigned char* ring, const Src& s, int k) {
   using G = StreamGeom<THREADS, BF16>;
-  constexpr int S = G::S;
+  return ring + (size_t)k * (s.rows == 2 ? G::SB : G::RB);
+}
+
+// The pass proper for a given layout (see stream_pass_pre).
+template <int THREADS, bool BF16, bool TWO, class Pre, class Body>
+__device__ __forceinline__ void stream_pass_lay(unsigned char* ring, const Src& s, bool& primed,
+                                                Pre&& pre, Body&& body) {
+  using G = StreamGeom<THREADS, BF16>;
+  using Y = Lay<THREADS, BF16, TWO>;
+  constexpr int S = Y::DEPTH;
   const int NK = (s.nloc + G::CE - 1) / G::CE;
+  if (!primed) {
 #pragma unroll
-  for (int k = 0; k < S - 1; ++k) {
-    if (k < NK) copy_chunk<THREADS, BF16>(s, k, ring + k * G::SB);
-    else cp_async_commit();
+    for (int k = 0; k < S - 1; ++k) {
+      if (k < NK) copy_chunk<THREADS, BF16, TWO>(s, k, ring + k * Y::STRIDE);
+      else cp_async_commit();
+    }
   }
+  primed = false;
   pre();
   int slot = 0;
   for (int k = 0; k < NK; ++k) {
     const int kn = k + S - 1;
     const int nslot = slot == 0 ? S - 1 : slot - 1;  // (k + S - 1) % S
-    if (kn < NK) copy_chunk<THREADS, BF16>(s, kn, ring + nslot * G::SB);
+    if (kn < NK) copy_chunk<THREADS, BF16, TWO>(s, kn, ring + nslot * Y::STRIDE);
     else cp_async_commit();
     cp_async_wait<S - 1>();  // chunk k's copies (this thread's) have landed
-    const unsigned char* st = ring + slot * G::SB;
+    const unsigned char* st = ring + slot * Y::STRIDE;
     const bool stop = body(st, st + G::RB, k);
     slot = slot == S - 1 ? 0 : slot + 1;
     if (stop) break;
@@ -248,9 +271,72 @@ __device__ __forceinline__ void stream_pass_pre(unsigned char* ring, const Src& 
   cp_async_wait<0>();
 }
 
-template <int THREADS, bool BF16, class Body>
-__device__ __forceinline__ void stream_pass(unsigned char* ring, const Src& s, Body&& body) {
-  stream_pass_pre<THREADS, BF16>(ring, s, [] {}, body);
+// Streams the slice chunk by chunk, DEPTH - 1 chunks ahead (Lay), calling
+// body(target_stage_row, draft_stage_row, k) with all threads (the draft
+// pointer is meaningful only for passes over both rows); body returns true
+// (uniformly) to end the pass.  pre() runs once, after the first copies are
+// issued.  When `primed` is set the first chunks were issued earlier by
+// stream_prime over the same rows and are not issued again (the flag is
+// cleared).  On return every copy of the pass has landed.
+// ROWS: 2 or 1 when the caller knows s.rows (only that layout's loop is
+// compiled), 0 to dispatch on it.
+template <int THREADS, bool BF16, int ROWS = 0, class Pre, class Body>
+__device__ __forceinline__ void stream_pass_pre(unsigned char* ring, const Src& s, bool& primed,
+                                                Pre&& pre, Body&& body) {
+  using G = StreamGeom<THREADS, BF16>;
+  const int NK = (s.nloc + G::CE - 1) / G::CE;
+  if (s.held) {  // the rows stayed in the ring since the visit's first pass
+    pre();
+    for (int k = 0; k < NK; ++k) {
+      const unsigned char* st = held_stage<THREADS, BF16>(ring, s, k);
+      if (body(st, st + G::RB, k)) break;
+    }
+    return;
+  }
+  if (ROWS == 2 || (ROWS == 0 && s.rows == 2))
+    stream_pass_lay<THREADS, BF16, true>(ring, s, primed, pre, body);
+  else
+    stream_pass_lay<THREADS, BF16, false>(ring, s, primed, pre, body);
+}
+
+template <int THREADS, bool BF16, int ROWS = 0, class Body>
+__device__ __forceinline__ void stream_pass(unsigned char* ring, const Src& s, bool& primed,
+                                            Body&& body) {
+  stream_pass_pre<THREADS, BF16, ROWS>(ring, s, primed, [] {}, body);
+}
+
+// Issues the copies a pass over s starts with (its first DEPTH - 1 chunks,
+// into the ring stages it reads them from), so that they travel while the
+// CTA waits in a cluster exchange.  Every thread copies only into its own
+// slots, which its previous pass has finished reading, so no barrier is
+// needed.  The next pass over the same rows takes them (primed); any other
+// use of the ring first calls stream_drain.
+template <int THREADS, bool BF16>
+__device__ __forceinline__ void stream_prime(unsigned char* ring, const Src& s, bool& primed) {
+  using G = StreamGeom<THREADS, BF16>;
+  const int NK = (s.nloc + G::CE - 1) / G::CE;
+  if (s.rows == 2) {
+    using Y = Lay<THREADS, BF16, true>;
+#pragma unroll
+    for (int k = 0; k < Y::DEPTH - 1; ++k) {
+      if (k < NK) copy_chunk<THREADS, BF16, true>(s, k, ring + k * Y::STRIDE);
+      else cp_async_commit();
+    }
+  } else {
+    using Y = Lay<THREADS, BF16, false>;
+#pragma unroll
+    for (int k = 0; k < Y::DEPTH - 1; ++k) {
+      if (k < NK) copy_chunk<THREADS, BF16, false>(s, k, ring + k * Y::STRIDE);
+      else cp_async_commit();
+    }
+  }
+  primed = true;
+}
+
+// Waits for primed copies that no pass will take.
+__device__ __forceinline__ void stream_drain(bool& primed) {
+  if (primed) cp_async_wait<0>();
+  primed = false;
 }
 
 __device__ __forceinline__ float raw_logit(const void* base, size_t i, bool bf16) {
@@ -308,9 +394,9 @@ __device__ __forceinline__ float2 exp_sum8(const float2 (&z)[4], float2 c2, floa
 // One chunk of a thread's values (8 per row) into its online (reference,
 // sum) pairs; the sums are kept as pairs of lanes.
 template <bool TWO>
-__device__ __forceinline__ void norm_accumulate(const float2 (&zt)[4], const float2 (&zd)[4],
-                                                float c, float& mt, float2& st, float& md,
-                                                float2& sd) {
+__device__ __forceinline__ float2 norm_accumulate(const float2 (&zt)[4], const float2 (&zd)[4],
+                                                  float c, float& mt, float2& st, float& md,
+                                                  float2& sd) {
   const float vt = max8(zt);
   const bool rt = __fmaf_rn(vt, c, -mt) > 0.f;
   float vd = 0.f;
@@ -325,16 +411,40 @@ __device__ __forceinline__ void norm_accumulate(const float2 (&zt)[4], const flo
       if (rd) rebase2(vd, c, md, sd);
   }
   const float2 c2 = dup2(c);
-  st = __fadd2_rn(st, exp_sum8(zt, c2, dup2(-mt)));
+  const float2 part = exp_sum8(zt, c2, dup2(-mt));  // this chunk's target terms
+  st = __fadd2_rn(st, part);
   if constexpr (TWO) sd = __fadd2_rn(sd, exp_sum8(zd, c2, dup2(-md)));
+  return part;
 }
 
+// Chunk records: the pass that defines a visit's final distribution leaves,
+// per chunk of the slice and warp, the warp's share of that distribution's
+// mass, so that the final draw finds the chunk holding its threshold
+// without another pass over the slice.  The mass of chunk k is
+//   kind 1 (a leaf's normaliser: the bonus draw samples p):
+//     sum_w rec1[k, w] 2^(rec0[k, w] - a) b   (warp reference, warp sum;
+//                                              a = M_t, b = 1 / S_t)
+//   kind 2 (the last ResiSpec rejection: R~' = m + lambda t):
+//     sum_w (rec0[k, w] + a rec1[k, w]) b     (a = lambda, b = sigma)
+//   kind 3 (the last SpecInfer rejection): sum_w rec0[k, w] b   (b = 1 / T)
+// in fixed warp order (deterministic).  Records exist when the slice has at
+// most kMaxChunkRecs / NW chunks; kind 0: none (the draw runs a pass).
+struct ChunkRec {
+  int kind;
+  float a, b;
+};
+
 // Cluster-wide scalars of a visit after the normaliser.
+static_assert(sizeof(VerifyParams::exp2_tab) == sizeof(float) * 2 * kExp2Tab,
+              "exp2 table size");
+
 struct VisitScalars {
   float c;           // log2(e) / T
   float Mt, invSt;   // target: global reference, 1 / sum
   float Md, invSd;   // draft
   float sig;         // sigma of the current residual (R = sig R~; 1 / S_t before any map)
+  SpecConst sc;      // SpecInfer instance: the residual's threshold K and exponent constants
+  const float (*tab)[2];  // SpecInfer instance: 2^(j/64) as double-floats
 };
 
 // 2^(z c - M): p~ or q~ of one element from its raw logit.
@@ -342,19 +452,20 @@ __device__ __forceinline__ float exp_of(float z, float c, float M) {
   return ex2(__fmaf_rn(z, c, -M));
 }
 
-// The unnormalised residual R~ after the first nm maps, element-wise (no
-// rejected-token zeroing: the caller applies it).  ResiSpec map: GetProxy
-// residual r = min(Z q, R) + lambda (R - min(Z q, R)), R' = r / sum r;
-// SpecInfer map: R' = (R - q)_+ / sum (Eq. recur); in the units above.
-// The ResiSpec map's two parts from R~ and q~: m = min(k q~, R~) and the
-// capacity R~ - m.
+// The unnormalised ResiSpec residual R~ after the first nm maps,
+// element-wise (no rejected-token zeroing: the caller applies it): the
+// GetProxy residual r = min(Z q, R) + lambda (R - min(Z q, R)),
+// R' = r / sum r, in the units above.  The map's two parts from R~ and q~:
+// m = min(k q~, R~) and the capacity R~ - m.  (SpecInfer keeps no maps: its
+// residual is one threshold away from p, see specinfer.cuh.)
 __device__ __forceinline__ float2 min_part2(float2 k, float2 q, float2 R) {
   const float2 kq = __fmul2_rn(k, q);
   return make_float2(fminf(kq.x, R.x), fminf(kq.y, R.y));
 }
 
-// Kinds of residual chain: SpecInfer maps; ResiSpec maps with the draft q
-// as the test denominator D throughout (Algorithm 1); ResiSpec maps with the
+// Kinds of residual chain: SpecInfer (the threshold of specinfer.cuh, its
+// own kernel instance); ResiSpec maps with the draft q as the test
+// denominator D throughout (Algorithm 1); ResiSpec maps with the
 // proxy as the next denominator (the paper's EAGLE integration, App. C).
 // With the proxy update the map is written with the current denominator:
 // m = min(k D~, R~), t = R~ - m, R~' = m + lambda t, and the proxy off the
@@ -369,14 +480,10 @@ template <int KIND>
 __device__ __forceinline__ float apply_chain(const StreamHead& S2, int nm, float R, float& D) {
   for (int i = 0; i < nm; ++i) {
     const float2 mp = S2.map[i];
-    if constexpr (KIND == kChainSpec) {
-      R = fmaxf(__fmaf_rn(mp.x, D, R), 0.f);
-    } else {
-      const float m = fminf(__fmul_rn(mp.x, D), R);
-      const float t = __fmaf_rn(m, -1.f, R);
-      R = __fmaf_rn(mp.y, t, m);
-      if constexpr (KIND == kChainResiDenom) D = t;
-    }
+    const float m = fminf(__fmul_rn(mp.x, D), R);
+    const float t = __fmaf_rn(m, -1.f, R);
+    R = __fmaf_rn(mp.y, t, m);
+    if constexpr (KIND == kChainResiDenom) D = t;
   }
   return R;
 }
@@ -388,18 +495,13 @@ __device__ __forceinline__ void apply_chain_pairs(const StreamHead& S2, int nm, 
   for (int i = 0; i < nm; ++i) {
     const float2 mp = S2.map[i];
     const float2 k = dup2(mp.x);
-    if constexpr (KIND == kChainSpec) {
+    const float2 lam = dup2(mp.y);
 #pragma unroll
-      for (int j = 0; j < NP; ++j) R[j] = relu2(__ffma2_rn(k, D[j], R[j]));
-    } else {
-      const float2 lam = dup2(mp.y);
-#pragma unroll
-      for (int j = 0; j < NP; ++j) {
-        const float2 m = min_part2(k, D[j], R[j]);
-        const float2 t = __ffma2_rn(m, dup2(-1.f), R[j]);
-        R[j] = __ffma2_rn(lam, t, m);
-        if constexpr (KIND == kChainResiDenom) D[j] = t;
-      }
+    for (int j = 0; j < NP; ++j) {
+      const float2 m = min_part2(k, D[j], R[j]);
+      const float2 t = __ffma2_rn(m, dup2(-1.f), R[j]);
+      R[j] = __ffma2_rn(lam, t, m);
+      if constexpr (KIND == kChainResiDenom) D[j] = t;
     }
   }
 }
@@ -408,8 +510,7 @@ template <int NP>
 __device__ __forceinline__ void apply_chain_any(const StreamHead& S2, int chain, int nm,
                                                 float2 (&R)[NP], float2 (&D)[NP]) {
   if (chain == kChainResiDenom) apply_chain_pairs<NP, kChainResiDenom>(S2, nm, R, D);
-  else if (chain == kChainResi) apply_chain_pairs<NP, kChainResi>(S2, nm, R, D);
-  else apply_chain_pairs<NP, kChainSpec>(S2, nm, R, D);
+  else apply_chain_pairs<NP, kChainResi>(S2, nm, R, D);
 }
 
 // Zero the residual at rejected tokens (ResiSpec: r(x0) = 0 and the later
@@ -428,7 +529,7 @@ __device__ __forceinline__ void zero_rejected_vec(const StreamHead& S2, int nm, 
 // Final values (the distribution being sampled) of vector h of a thread's
 // chunk: p when no map is pending, else the residual, R = sig R~ (zero at
 // the rejected tokens).  base: its first token.
-template <int THREADS, bool BF16>
+template <int THREADS, bool BF16, bool SPEC>
 __device__ __forceinline__ void final_values(const StreamHead& S2, const VisitScalars& K,
                                              int chain, int nm, int base,
                                              const unsigned char* rt, const unsigned char* rd,
@@ -437,6 +538,16 @@ __device__ __forceinline__ void final_values(const StreamHead& S2, const VisitSc
   constexpr int NP = VEC / 2;
   float z[VEC];
   unpack_vec<BF16>(stage_vec(rt, h, THREADS), z);
+  if constexpr (SPEC) {
+    if (nm > 0) {  // SpecInfer residual (p~ - K q~)_+ / T (specinfer.cuh)
+      float zd[VEC];
+      unpack_vec<BF16>(stage_vec(rd, h, THREADS), zd);
+#pragma unroll
+      for (int j = 0; j < VEC; ++j)
+        v[j] = __fmul_rn(df_value(spec_residual(z[j], zd[j], K.sc, K.tab)), K.sig);
+      return;
+    }
+  }
   const float2 c2 = dup2(K.c);
   float2 R[NP];
 #pragma unroll
@@ -463,175 +574,213 @@ __device__ __forceinline__ void final_values(const StreamHead& S2, const VisitSc
     v[2 * j] = r.x;
     v[2 * j + 1] = r.y;
   }
-  if (chain != kChainSpec) zero_rejected_vec<VEC>(S2, nm, base, v);
+  zero_rejected_vec<VEC>(S2, nm, base, v);
 }
 
 // ---------------------------------------------------------------- sampler
-// Inverse-CDF draw inside one CTA from fixed-point masses (as the resident
-// kernel's sampler): chunk totals locate the chunk that holds the threshold
-// `tau` (mass units 2^-44); the chunk's values are written to shared memory
-// F as fp32 in token order; then NW contiguous warp segments, 32 lane ranges
-// and one lane's walk find the token.  If rounding leaves tau past the
-// slice's own total, the last token with positive mass is taken.  Returns
-// the token's offset in the slice (-1 if the slice has no mass).
-template <int THREADS, bool BF16>
-__device__ int stream_search(Head& H, const StreamHead& S2, float* F, unsigned char* ring,
-                             const Src& s, const VisitScalars& K, int chain, int lo,
-                             unsigned long long tau) {
+// Inverse-CDF draw inside one CTA: the smallest slice offset whose inclusive
+// mass prefix exceeds `tau` (mass units 2^-44).
+//   1. One pass over the slice sums the values of every warp's share of a
+//      chunk (fp32, a fixed butterfly order) and adds it, rounded to the
+//      fixed-point unit, into the chunk's total with one shared-memory
+//      atomic per warp and chunk (integer sums: the totals do not depend on
+//      the order of the atomics; no barrier inside the pass).  `ck` holds
+//      one total per chunk.
+//   2. One warp scans the chunk totals and finds the chunk that holds tau.
+//   3. That chunk's vectors are read again; a block-wide scan of their exact
+//      fixed-point masses in token order (vector h of thread t is token block
+//      h THREADS + t) finds the vector, and its thread walks its values.
+// The chunk totals carry the fp32 rounding of step 1 (about 1e-7 of the
+// mass), so they can place tau in a neighbouring chunk only when it lies
+// that close to a chunk boundary; if tau then falls past the chunk's exact
+// total (or rounding leaves it past the slice's total), the last token with
+// positive mass is taken.  Returns the token's offset in the slice (-1 if the
+// slice has no mass).
+constexpr int kMaxSearchChunks = 128;
+
+template <int THREADS, bool BF16, bool SPEC>
+__device__ int stream_search(Head& H, const StreamHead& S2, unsigned long long* ck,
+                             unsigned char* ring, const Src& s, const VisitScalars& K, int chain,
+                             int lo, unsigned long long tau, bool& primed, const ChunkRec& cr) {
   using G = StreamGeom<THREADS, BF16>;
   constexpr int VEC = G::VEC;
   constexpr int NW = THREADS / 32;
+  static_assert(G::VPT * NW <= 32, "one scan lane per warp segment");
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int nm = S2.nmaps;
-  if (threadIdx.x == 0) {
-    H.misc[0] = -1;  // chunk holding tau
-    H.misc[1] = -1;  // last chunk with mass
-    H.fixd[0] = 0;   // mass before the chunk
-  }
+  const int NK = (s.nloc + G::CE - 1) / G::CE;  // <= kMaxSearchChunks (slices <= 2^18)
+  for (int k = threadIdx.x; k < NK; k += THREADS) ck[k] = 0ull;
   __syncthreads();
-  unsigned long long run = 0;  // thread 0 only
-  stream_pass<THREADS, BF16>(ring, s, [&](const unsigned char* rt, const unsigned char* rd,
-                                           int k) -> bool {
-    unsigned long long acc = 0;
+  if (cr.kind != 0) {
+    // chunk totals from the records of the pass that defined the distribution
+    for (int k = threadIdx.x; k < NK; k += THREADS) {
+      float m = 0.f;
+      for (int w = 0; w < NW; ++w) {
+        const float r0 = S2.crec[0][k * NW + w], r1 = S2.crec[1][k * NW + w];
+        float v;
+        if (cr.kind == 1) v = __fmul_rn(__fmul_rn(r1, ex2(__fsub_rn(r0, cr.a))), cr.b);
+        else if (cr.kind == 2) v = __fmul_rn(__fmaf_rn(cr.a, r1, r0), cr.b);
+        else v = __fmul_rn(r0, cr.b);
+        m = __fadd_rn(m, v);
+      }
+      ck[k] = to_fix(m);
+    }
+  } else stream_pass<THREADS, BF16>(ring, s, primed, [&](const unsigned char* rt,
+                                                         const unsigned char* rd, int k) -> bool {
+    float2 acc2 = make_float2(0.f, 0.f);
 #pragma unroll
     for (int h = 0; h < G::VPT; ++h) {
       float v[VEC];
-      final_values<THREADS, BF16>(S2, K, chain, nm, lo + k * G::CE + (h * THREADS + (int)threadIdx.x) * VEC,
-                                  rt, rd, h, v);
+      final_values<THREADS, BF16, SPEC>(S2, K, chain, nm,
+                                        lo + k * G::CE + (h * THREADS + (int)threadIdx.x) * VEC,
+                                        rt, rd, h, v);
 #pragma unroll
-      for (int j = 0; j < VEC; ++j) acc += to_fix(v[j]);
+      for (int j = 0; j < VEC / 2; ++j) acc2 = __fadd2_rn(acc2, make_float2(v[2 * j], v[2 * j + 1]));
     }
-    acc = warp_sum_u64(acc);
-    if (lane == 0) H.seg[warp] = acc;
-    __syncthreads();
-    if (threadIdx.x == 0) {
-      unsigned long long m = 0;
-      for (int w = 0; w < NW; ++w) m += H.seg[w];
-      if (m > 0) H.misc[1] = k;
-      if (H.misc[0] < 0) {
-        if (run + m > tau) { H.misc[0] = k; H.fixd[0] = tau - run; }
-        else run += m;
-      }
+    const float acc = group_sum<5>(__fadd_rn(acc2.x, acc2.y));
+    if (lane == 0) {
+      const unsigned long long a = to_fix(acc);
+      if (a) atomicAdd(ck + k, a);
     }
-    __syncthreads();
-    return H.misc[0] >= 0;
+    return false;
   });
-  const int kfound = H.misc[0];
-  const int klast = H.misc[1];
-  if (kfound < 0 && klast < 0) return -1;
-  const bool force = kfound < 0;
-  const int ks = force ? klast : kfound;
-  const unsigned long long t = force ? 0ull : H.fixd[0];
-  // the chosen chunk's values in token order (this thread's vectors, copied
-  // again into ring stage 0)
-  copy_chunk<THREADS, BF16>(s, ks, ring);
-  cp_async_wait<0>();
+  __syncthreads();
+  if (warp == 0) {
+    // lanes hold chunks lane + 32 i; inclusive prefix over chunk order
+    unsigned long long run = 0;
+    int kfound = -1, klast = -1;
+    unsigned long long before = 0;
+    for (int base = 0; base < NK; base += 32) {
+      const int k = base + lane;
+      const unsigned long long m = k < NK ? ck[k] : 0ull;
+      unsigned long long incl = m;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const unsigned long long n = __shfl_up_sync(0xffffffffu, incl, o);
+        if (lane >= o) incl += n;
+      }
+      incl += run;
+      const unsigned cross = __ballot_sync(0xffffffffu, k < NK && incl > tau);
+      const unsigned pos = __ballot_sync(0xffffffffu, m > 0);
+      if (pos) klast = base + 31 - __clz(pos);
+      if (kfound < 0 && cross) {
+        const int l = __ffs(cross) - 1;
+        kfound = base + l;
+        before = __shfl_sync(0xffffffffu, incl - m, l);
+      }
+      run = __shfl_sync(0xffffffffu, incl, 31);
+    }
+    if (lane == 0) {
+      H.misc[0] = kfound >= 0 ? kfound : klast;
+      H.misc[3] = kfound < 0;  // threshold past the slice's total: last token with mass
+      H.fixd[0] = kfound >= 0 ? tau - before : 0ull;
+      H.misc[4] = -1;
+      H.misc[7] = -1;
+    }
+  }
+  __syncthreads();
+  const int ks = H.misc[0];
+  if (ks < 0) return -1;
+  const bool force = H.misc[3] != 0;
+  const unsigned long long t = H.fixd[0];
+  // the chosen chunk's values (this thread's vectors: held in the ring, or
+  // copied again into ring stage 0, which only this thread's copies write)
+  const unsigned char* stg = ring;
+  if (s.held) {
+    stg = held_stage<THREADS, BF16>(ring, s, ks);
+  } else {
+    stream_drain(primed);
+    if (s.rows == 2) copy_chunk<THREADS, BF16, true>(s, ks, ring);
+    else copy_chunk<THREADS, BF16, false>(s, ks, ring);
+    cp_async_wait<0>();
+  }
+  float v[G::VPT][VEC];
+  unsigned long long mv[G::VPT], ex[G::VPT];
+  int lastpos = -1;
 #pragma unroll
   for (int h = 0; h < G::VPT; ++h) {
-    float v[VEC];
     const int g = h * THREADS + (int)threadIdx.x;
-    final_values<THREADS, BF16>(S2, K, chain, nm, lo + ks * G::CE + g * VEC, ring, ring + G::RB, h,
-                                v);
+    final_values<THREADS, BF16, SPEC>(S2, K, chain, nm, lo + ks * G::CE + g * VEC, stg,
+                                      stg + G::RB, h, v[h]);
+    mv[h] = 0;
 #pragma unroll
-    for (int j = 0; j < VEC; ++j) F[g * VEC + j] = v[j];
+    for (int j = 0; j < VEC; ++j) {
+      mv[h] += to_fix(v[h][j]);
+      if (v[h][j] > 0.f && ks * G::CE + g * VEC + j < s.nloc) lastpos = g * VEC + j;
+    }
+    unsigned long long incl = mv[h];
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const unsigned long long n = __shfl_up_sync(0xffffffffu, incl, o);
+      if (lane >= o) incl += n;
+    }
+    ex[h] = incl - mv[h];
+    if (lane == 31) H.seg[h * NW + warp] = incl;
   }
   __syncthreads();
-  // warp segments of SEG elements over the chunk (zeros past the slice)
-  constexpr int SEG = G::CE / NW;
-  {
-    const int s0i = warp * SEG;
-    unsigned long long acc = 0;
-    for (int i = s0i + 4 * lane; i < s0i + SEG; i += 128) {
-      const float4 x = *reinterpret_cast<const float4*>(F + i);
-      acc += to_fix(x.x) + to_fix(x.y) + to_fix(x.z) + to_fix(x.w);
-    }
-    acc = warp_sum_u64(acc);
-    if (lane == 0) H.seg[warp] = acc;
-  }
-  __syncthreads();
-  if (threadIdx.x == 0) {
-    unsigned long long a = 0;
-    int wstar = -1, last = -1;
-    for (int w = 0; w < NW; ++w) {
-      const unsigned long long m = H.seg[w];
-      if (m > 0) last = w;
-      if (!force && wstar < 0) {
-        if (a + m > t) wstar = w;
-        else a += m;
-      }
-    }
-    const bool f2 = force || wstar < 0;
-    H.misc[3] = f2;
-    H.misc[2] = f2 ? max(last, 0) : wstar;
-    H.fixd[1] = f2 ? 0ull : t - a;
-    H.misc[4] = -1;
-  }
-  __syncthreads();
-  if (warp == H.misc[2]) {
-    constexpr int SUB = SEG / 32;
-    const int r0 = warp * SEG + lane * SUB, r1 = r0 + SUB;
-    unsigned long long m = 0;
-    int lastpos = -1;
-    for (int i = r0; i < r1; ++i) {
-      const float x = F[i];
-      m += to_fix(x);
-      if (x > 0.f) lastpos = i;
-    }
+  if (warp == 0) {  // exclusive prefix of the warp segments in token order
+    const unsigned long long m = lane < G::VPT * NW ? H.seg[lane] : 0ull;
     unsigned long long incl = m;
 #pragma unroll
     for (int o = 1; o < 32; o <<= 1) {
       const unsigned long long n = __shfl_up_sync(0xffffffffu, incl, o);
       if (lane >= o) incl += n;
     }
-    const unsigned long long tt = H.fixd[1];
-    const bool f2 = H.misc[3] != 0;
-    const unsigned cross = __ballot_sync(0xffffffffu, !f2 && incl > tt);
-    const unsigned pos = __ballot_sync(0xffffffffu, lastpos >= 0);
-    const int sel = cross ? __ffs(cross) - 1 : (pos ? 31 - __clz(pos) : 0);
-    if (lane == sel) {
-      int pick = -1;
-      if (cross) {
-        const unsigned long long tl = tt - (incl - m);
-        unsigned long long a = 0;
-        for (int i = r0; i < r1; ++i) {
-          a += to_fix(F[i]);
-          if (a > tl) { pick = i; break; }
+    __syncwarp();
+    if (lane < G::VPT * NW) H.seg[lane] = incl - m;
+  }
+  __syncthreads();
+  if (lastpos >= 0) atomicMax(&H.misc[7], lastpos);  // the chunk's last token with mass
+  if (!force) {
+#pragma unroll
+    for (int h = 0; h < G::VPT; ++h) {
+      const unsigned long long a0 = H.seg[h * NW + warp] + ex[h];
+      if (mv[h] > 0 && a0 <= t && t < a0 + mv[h]) {
+        unsigned long long a = a0;
+        int pick = (h * THREADS + (int)threadIdx.x) * VEC + VEC - 1;
+#pragma unroll
+        for (int j = 0; j < VEC; ++j) {
+          a += to_fix(v[h][j]);
+          if (a > t) { pick = (h * THREADS + (int)threadIdx.x) * VEC + j; break; }
         }
+        H.misc[4] = pick;
       }
-      if (pick < 0) pick = lastpos >= 0 ? lastpos : r0;
-      H.misc[4] = pick;
     }
   }
   __syncthreads();
-  const int pick = H.misc[4];
+  // no vector holds tau (forced, or tau past the chunk's exact total): the
+  // chunk's last token with positive mass
+  const int pick = H.misc[4] >= 0 ? H.misc[4] : H.misc[7];
   __syncthreads();
   return pick < 0 ? -1 : ks * G::CE + pick;
 }
 
 // Final draw of a visit: every CTA picks the CTA whose mass range holds
 // u * total (as the resident kernel's sampler); that CTA searches its slice.
-template <int THREADS, bool BF16>
-__device__ bool stream_sample(Head& H, const StreamHead& S2, float* F, unsigned char* ring,
-                              const VerifyParams& P, const Src& s_in, const VisitScalars& K, int chain, int mass_kind,
+template <int THREADS, bool BF16, bool SPEC>
+__device__ bool stream_sample(Head& H, StreamHead& S2, unsigned char* ring, const VerifyParams& P,
+                              const Src& s_in, const VisitScalars& K, int chain, int mass_kind,
                               const Pending& Pm, float u, int b, int depth, int lo,
-                              uint32_t rank, uint32_t C, int& xp, uint32_t& xph, bool& timeout) {
+                              uint32_t rank, uint32_t C, int& xp, uint32_t& xph, bool& timeout,
+                              bool& primed, const ChunkRec& cr) {
   using G = StreamGeom<THREADS, BF16>;
   constexpr int VEC = G::VEC;
   constexpr int NW = THREADS / 32;
   const int nm = S2.nmaps;
-  Src s = s_in;
-  s.rows = nm > 0 ? 2 : 1;
+  // the visit's rows, in the ring layout they were loaded with (a residual
+  // left unchanged by degenerate rejections still streams both rows)
+  const Src& s = s_in;
   if (P.out_dist || mass_kind == 0) {
     // every CTA: values of its slice (written out when asked) and their sum
     float* dist = P.out_dist ? P.out_dist + (size_t)b * P.V + lo : nullptr;
     float sum = 0.f;
-    stream_pass<THREADS, BF16>(ring, s, [&](const unsigned char* rt, const unsigned char* rd,
-                                             int k) -> bool {
+    stream_pass<THREADS, BF16>(ring, s, primed, [&](const unsigned char* rt,
+                                                    const unsigned char* rd, int k) -> bool {
 #pragma unroll
       for (int h = 0; h < G::VPT; ++h) {
         float v[VEC];
         const int e0 = k * G::CE + (h * THREADS + (int)threadIdx.x) * VEC;  // offset in the slice
-        final_values<THREADS, BF16>(S2, K, chain, nm, lo + e0, rt, rd, h, v);
+        final_values<THREADS, BF16, SPEC>(S2, K, chain, nm, lo + e0, rt, rd, h, v);
 #pragma unroll
         for (int j = 0; j < VEC; ++j) {
           sum += v[j];
@@ -675,9 +824,53 @@ __device__ bool stream_sample(Head& H, const StreamHead& S2, float* F, unsigned 
   if ((int)rank != cstar) return true;
   // A slice whose exchange mass is positive but whose every element rounds
   // to zero mass yields its first token.
-  const int pick = stream_search<THREADS, BF16>(H, S2, F, ring, s, K, chain, lo, tau);
+  // chunk totals of the search: the children's logit slots, unused by the draw
+  const int pick = stream_search<THREADS, BF16, SPEC>(
+      H, S2, reinterpret_cast<unsigned long long*>(S2.kzt), ring, s, K, chain, lo, tau, primed,
+      cr);
   if (threadIdx.x == 0) P.out_tokens[(size_t)b * (P.D + 1) + depth] = lo + max(pick, 0);
   return true;
+}
+
+// Cluster total of N double-float partials per thread (SpecInfer sums):
+// each CTA reduces its threads' values in a fixed order (warp butterflies,
+// then one warp over the warps' values), pushes the CTA's value through the
+// exchange (only thread 0 contributes, so the exchange's own fp32 sums add
+// zeros), and every CTA adds the received per-CTA values in rank order, so
+// that all CTAs obtain the same bits.
+template <int NW, int N>
+__device__ __forceinline__ bool df_exchange(Head& H, DF (&v)[N], DF (&tot)[N], int& xp,
+                                            uint32_t& xph, uint32_t rank, uint32_t C) {
+  static_assert(N <= 2 && N * NW <= 32, "two double-floats per warp in the segment slots");
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  DF* wdf = reinterpret_cast<DF*>(H.seg);
+#pragma unroll
+  for (int i = 0; i < N; ++i) {
+    v[i] = df_group_sum<5>(v[i]);
+    if (lane == 0) wdf[i * NW + warp] = v[i];
+  }
+  __syncthreads();
+  float a[4] = {0.f, 0.f, 0.f, 0.f};
+  if (warp == 0) {
+#pragma unroll
+    for (int i = 0; i < N; ++i) {
+      const DF c = df_group_sum<4>(lane < NW ? wdf[i * NW + lane] : df(0.f));
+      if (lane == 0) {
+        a[2 * i] = c.hi;
+        a[2 * i + 1] = c.lo;
+      }
+    }
+  }
+  float o[8];
+  int oflags;
+  exchange<NW, false, 2 * N>(H, a[0], a[1], a[2], a[3], 0, -1, xp, xph, rank, C, o, oflags);
+#pragma unroll
+  for (int i = 0; i < N; ++i) {
+    tot[i] = df(0.f);
+    for (uint32_t r = 0; r < C; ++r)
+      tot[i] = df_add(tot[i], DF{H.part[r][2 * i], H.part[r][2 * i + 1]});
+  }
+  return !(oflags & kFlagTimeout);
 }
 
 // ---------------------------------------------------------------- kernel
@@ -685,9 +878,9 @@ __device__ bool stream_sample(Head& H, const StreamHead& S2, float* F, unsigned 
 // denominator, level fill, drafting, phase counters).  The default instance
 // compiles them out: their code, even untaken, costs the hot loops
 // instruction-cache misses.
-template <int THREADS, bool BF16, bool VAR>
+template <int THREADS, bool BF16, bool VAR, bool SPEC>
 __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
-    stream_kernel(const VerifyParams P) {
+    stream_kernel(const __grid_constant__ VerifyParams P) {
   using G = StreamGeom<THREADS, BF16>;
   constexpr int NW = THREADS / 32;
   constexpr int VEC = G::VEC;
@@ -696,15 +889,15 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
   Head& H = *reinterpret_cast<Head*>(smem);
   StreamHead& S2 = *reinterpret_cast<StreamHead*>(smem + kHeadBytes);
   unsigned char* ring = smem + kHeadBytes + kStreamHeadBytes;  // S stages of SB bytes
-  // the sampler's chunk buffer (CE floats): ring stage 1, free once a pass
-  // has drained (the sampler copies its chunk into stage 0)
-  float* F = reinterpret_cast<float*>(ring + G::SB);
-  static_assert(G::CE * 4 <= G::SB, "sampler buffer exceeds a ring stage");
   int16_t* par = reinterpret_cast<int16_t*>(ring + G::RING);
   int16_t* first_child = par + P.npad;
   int16_t* next_sib = first_child + P.npad + 16;
   int32_t* cand_s = reinterpret_cast<int32_t*>(next_sib + P.npad);
 
+  // Nothing is read before the preceding work on the stream has completed;
+  // the next launch may be scheduled from here on (it waits the same way).
+  grid_dependency_wait();
+  grid_launch_dependents();
   const int tid = threadIdx.x;
   const uint32_t rank = cluster_ctarank();
   const uint32_t C = cluster_nctarank();
@@ -713,8 +906,9 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
   const int L = P.slice;
   const int lo = (int)rank * L;
   const int nloc = max(0, min(V, lo + L) - lo);
-  const bool resi = P.mode == 0;
-  const int chain = !resi ? kChainSpec : ((VAR && P.denom_update) ? kChainResiDenom : kChainResi);
+  // SPEC: the SpecInfer instance (Eq. recur, evaluated as in specinfer.cuh);
+  // the others run ResiSpec (Algorithm 1)
+  const int chain = SPEC ? kChainSpec : ((VAR && P.denom_update) ? kChainResiDenom : kChainResi);
   const bool drafting = VAR && P.draft_out != nullptr;
   const bool bf16 = BF16;
 
@@ -724,6 +918,11 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
   int node = -1, row = 0;
   uint32_t xph = 0;
   int xp = 0;
+  bool primed = false;  // the ring holds the first copies of the next pass (stream_prime)
+  const int lane = tid & 31, warp = tid >> 5;
+  // chunk records for the final draw (ChunkRec; not in the instance with the
+  // optional paths)
+  const bool rec_ok = !VAR && ((nloc + G::CE - 1) / G::CE) * NW <= kMaxChunkRecs;
 
   // Kernel setup: exchange barriers, the tree's child lists and the
   // candidates.  It runs while the first chunks of the root's rows are in
@@ -800,12 +999,20 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
     sq.rows = 1;
     sq.nloc = nloc;
     sq.vec = P.use_tma != 0;
+    sq.held = false;
     VisitScalars Kq = K;
     Kq.Mt = K.Md;
     Kq.invSt = K.invSd;
+    // chunk totals of the searches: the residual maps' slots (no map exists
+    // before the node's accept tests)
+    static_assert(sizeof(StreamHead::map) >= kMaxSearchChunks * sizeof(unsigned long long),
+                  "search chunk totals fit the map slots");
+    stream_drain(primed);
     for (int i = 0, cn = c1d; i < nk; ++i, cn = next_sib[cn]) {
       if (owner[i] != (int)rank) continue;
-      const int pick = stream_search<THREADS, BF16>(H, S2, F, ring, sq, Kq, chain, lo, tau[i]);
+      const int pick = stream_search<THREADS, BF16, SPEC>(
+          H, S2, reinterpret_cast<unsigned long long*>(S2.map), ring, sq, Kq, chain, lo, tau[i],
+          primed, ChunkRec{0, 0.f, 0.f});
       if (tid == 0) P.draft_out[(size_t)b * N + cn] = lo + max(pick, 0);
     }
     cluster_sync();  // every drawn token written (release / acquire at cluster scope)
@@ -848,12 +1055,14 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
     src.rows = need_draft ? 2 : 1;
     src.nloc = nloc;
     src.vec = P.use_tma != 0;
+    src.held = false;
 
     // Per-visit state in S2 is written by every thread with identical
     // values (each thread reads back its own writes), so no barrier is
     // needed to publish it; the barrier at the end of the previous visit
     // orders these writes after every read of the old values.
     S2.nmaps = 0;
+    stream_drain(primed);  // copies primed for the previous visit's rows
 
     mark(kPhaseNorm);
     // ---- tempered normaliser (S2): online (reference, sum) per row; while
@@ -864,7 +1073,8 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
     float mt = kNoRef, md = kNoRef;
     float2 st2 = make_float2(0.f, 0.f), sd2 = make_float2(0.f, 0.f);
     float dmin = INFINITY;  // Z_applied: smallest z_t - z_d of the slice
-    const bool zapp = VAR && P.z_applied != 0 && resi;
+    ChunkRec crec{0, 0.f, 0.f};  // records of this visit's final distribution
+    const bool zapp = VAR && !SPEC && P.z_applied != 0;
     // (child t is found by walking t siblings; the loaded logits stay in
     // registers until the pass ends, so no warp waits for them; the draws
     // are computed by the last threads)
@@ -875,7 +1085,7 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
     };
     bool have_kid = false;
     float kz_t = 0.f, kz_d = 0.f;
-    stream_pass_pre<THREADS, BF16>(ring, src,
+    stream_pass_pre<THREADS, BF16>(ring, src, primed,
         [&] {
           if (first) {
             setup();
@@ -899,7 +1109,7 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
             S2.ufin = uniform_draw(P.seed, (uint32_t)b, (uint32_t)row, 1);
           }
         },
-        [&](const unsigned char* rt, const unsigned char* rd, int) -> bool {
+        [&](const unsigned char* rt, const unsigned char* rd, int k) -> bool {
           if (err) return true;  // invalid tree (uniform over the cluster)
           float2 zt[4], zd[4];
           load_pairs<THREADS, BF16>(rt, zt);
@@ -908,11 +1118,29 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
             norm_accumulate<true>(zt, zd, P.scale_log2, mt, st2, md, sd2);
             if (zapp) dmin = fminf(dmin, dmin8(zt, zd));
           } else {
-            norm_accumulate<false>(zt, zd, P.scale_log2, mt, st2, md, sd2);
+            const float2 part = norm_accumulate<false>(zt, zd, P.scale_log2, mt, st2, md, sd2);
+            if (rec_ok) {
+              // a leaf: its bonus draw samples this row; record the warp's
+              // chunk mass against the warp's largest reference
+              const float mw = redux_max(mt);
+              const float sw =
+                  group_sum<5>(__fmul_rn(__fadd_rn(part.x, part.y), ex2(__fsub_rn(mt, mw))));
+              if (lane == 0) {
+                S2.crec[0][k * NW + warp] = mw;
+                S2.crec[1][k * NW + warp] = sw;
+              }
+            }
           }
           return false;
         });
     if (err) break;
+    // A slice of at most S chunks stays in the ring (chunk k in stage k; not
+    // in the instance with the optional paths, whose registers it exceeds):
+    // every later pass of the visit reads it from shared memory.  Otherwise
+    // the next pass over these rows (the first rejection's, or the draw's)
+    // starts its copies now, while the normaliser is exchanged.
+    src.held = !VAR && (nloc + G::CE - 1) / G::CE <= (src.rows == 2 ? G::S : 2 * G::S);
+    if (!src.held) stream_prime<THREADS, BF16>(ring, src, primed);
     const float st = __fadd_rn(st2.x, st2.y), sd = __fadd_rn(sd2.x, sd2.y);
     if (have_kid) {
       S2.kzt[tid] = kz_t;
@@ -953,6 +1181,14 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
     K.Md = o[2];
     K.invSd = need_draft ? __frcp_rn(o[3]) : 0.f;
     K.sig = K.invSt;
+    if constexpr (SPEC) {
+      K.sc = SpecConst{P.scale_log2, P.scale_log2_lo, K.Mt, K.Md, df(0.f)};
+      K.tab = P.exp2_tab;
+    }
+    // SpecInfer: the double-float normalisers (taken at the node's first
+    // rejection) and the current residual mass T
+    bool spec_norm = false;
+    DF spec_Sd = df(0.f), spec_T = df(0.f);
     if (drafting && need_draft) draft_children(c1, K, rbase);
     // Z_applied: Z* = min_{q>0} p / q = 2^(c min(z_t - z_d) - M_t + M_d) S_d / S_t,
     // valid while no map has zeroed a token (after one, Z* = 0)
@@ -966,9 +1202,11 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
     if (!need_draft) {
       // accepted leaf (or a root without children): bonus token from p
       bool to = false;
+      if (rec_ok) crec = ChunkRec{1, K.Mt, K.invSt};
       mark(kPhaseDraw);
-      if (!stream_sample<THREADS, BF16>(H, S2, F, ring, P, src, K, chain, mass_kind, Pm, S2.ufin,
-                                        b, depth, lo, rank, C, xp, xph, to))
+      if (!stream_sample<THREADS, BF16, SPEC>(H, S2, ring, P, src, K, chain, mass_kind, Pm,
+                                              S2.ufin, b, depth, lo, rank, C, xp, xph, to, primed,
+                                              crec))
         err |= kErrEmpty;
       if (to) err |= kErrTimeout;
       break;
@@ -986,7 +1224,9 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
       const float qt = exp_of(S2.kzd[i], K.c, K.Md);
       float qx = __fmul_rn(qt, K.invSd);
       float Rt = exp_of(S2.kzt[i], K.c, K.Mt);
-      if (chain == kChainResiDenom) {
+      if constexpr (SPEC) {
+        if (nm > 0) Rt = df_value(spec_residual(S2.kzt[i], S2.kzd[i], K.sc, K.tab));
+      } else if (chain == kChainResiDenom) {
         // The exact chain at x: a map that rejected x leaves R(x) = 0 and
         // the denominator's value there unchanged (K(x0) = D(x0)); a later
         // map then gives it R - r = 0.  D~ changes units at every map
@@ -1008,49 +1248,127 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
         }
         Rt = Rc;
         qx = __fmul_rn(D, dprev);
-      } else if (resi) {
+      } else {
         float D = qt;
         Rt = apply_chain<kChainResi>(S2, nm, Rt, D);
         for (int j = 0; j < nm; ++j)
           if (S2.rej[j] == x) Rt = 0.f;
-      } else {
-        float D = qt;
-        Rt = apply_chain<kChainSpec>(S2, nm, Rt, D);
       }
       const float Rx = __fmul_rn(Rt, K.sig);
       const float u = S2.kua[i];
       if (__fmul_rn(u, qx) < Rx) { accepted = cn; acc_tok = x; break; }
       rejects += 1;
-      float Z = 0.f;
-      if (resi) {
-        Z = __fsub_rn(qx, Rx);
-        if (zapp)  // max(Z*, |gap|), at most 1 - R(x0)
-          Z = fminf(fmaxf(nm == 0 ? zstar : 0.f, fabsf(Z)), __fsub_rn(1.f, Rx));
-        if (!(Z > 0.f)) {  // degenerate rejection: R is kept unchanged
-          info |= kInfoDegenerate;
-          continue;
+      if constexpr (SPEC) {
+        // ---- SpecInfer rejection (Eq. recur): R <- (R - q)_+ / S, kept as
+        // the threshold K of r~ = (p~ - K q~)_+ (specinfer.cuh).  The node's
+        // first rejection takes S_t and S_d in double-float (one pass);
+        // then K_1 = S_t / S_d, later K_{n+1} = K_n + T_n / S_d, and one pass
+        // sums T = sum r~ at the new K.
+        if (nm >= kMaxMaps) { err |= kErrFanout; break; }
+        mark(kPhaseRej);
+          const DF Kprev = K.sc.K;
+        if (!spec_norm) {
+          DF acc[2] = {df(0.f), df(0.f)};
+          stream_pass<THREADS, BF16, 2>(ring, src, primed, [&](const unsigned char* rt,
+                                                            const unsigned char* rd, int) -> bool {
+#pragma unroll
+            for (int h = 0; h < G::VPT; ++h) {
+              float zt[VEC], zd[VEC];
+              unpack_vec<BF16>(stage_vec(rt, h, THREADS), zt);
+              unpack_vec<BF16>(stage_vec(rd, h, THREADS), zd);
+#pragma unroll
+              for (int j = 0; j < VEC; ++j) {
+                acc[0] = df_add(acc[0], unnorm_df(zt[j], K.sc.c_hi, K.sc.c_lo, K.Mt, K.tab));
+                acc[1] = df_add(acc[1], unnorm_df(zd[j], K.sc.c_hi, K.sc.c_lo, K.Md, K.tab));
+              }
+            }
+            return false;
+          });
+          if (!src.held) stream_prime<THREADS, BF16>(ring, src, primed);
+          DF tot[2];
+          if (!df_exchange<NW, 2>(H, acc, tot, xp, xph, rank, C)) { err |= kErrTimeout; break; }
+          spec_norm = true;
+          spec_Sd = tot[1];
+          K.sc.K = df_div(tot[0], spec_Sd);
+        } else {
+          K.sc.K = df_add(K.sc.K, df_div(spec_T, spec_Sd));
         }
+        DF acc[1] = {df(0.f)};
+        // the last child's rejection defines the final distribution: its
+        // pass records it (ChunkRec kind 3)
+        const bool rec_last = rec_ok && next_sib[cn] < 0;
+        stream_pass<THREADS, BF16, 2>(ring, src, primed, [&](const unsigned char* rt,
+                                                          const unsigned char* rd, int k) -> bool {
+          float cr = 0.f;
+#pragma unroll
+          for (int h = 0; h < G::VPT; ++h) {
+            float zt[VEC], zd[VEC];
+            unpack_vec<BF16>(stage_vec(rt, h, THREADS), zt);
+            unpack_vec<BF16>(stage_vec(rd, h, THREADS), zd);
+#pragma unroll
+            for (int j = 0; j < VEC; ++j) {
+              const DF r = spec_residual(zt[j], zd[j], K.sc, K.tab);
+              acc[0] = df_add(acc[0], r);
+              cr = __fadd_rn(cr, r.hi);
+            }
+          }
+          if (rec_last) {
+            const float wr = group_sum<5>(cr);
+            if (lane == 0) S2.crec[0][k * NW + warp] = wr;
+          }
+          return false;
+        });
+        if (!src.held) stream_prime<THREADS, BF16>(ring, src, primed);
+        DF tot[1];
+        if (!df_exchange<NW, 1>(H, acc, tot, xp, xph, rank, C)) { err |= kErrTimeout; break; }
+        mark(kPhaseTest);
+        if (tot[0].hi > 0.f) {
+          spec_T = tot[0];
+          K.sig = __frcp_rn(df_value(spec_T));
+          // per-CTA masses of the residual for the draw: the exchange's
+          // per-CTA T (head part) times 1 / T
+          Pm = Pending{kSpec, x, K.sig, 0.f, 0.f};
+          mass_kind = 3;
+          if (rec_last) crec = ChunkRec{3, 0.f, K.sig};
+          S2.rej[nm] = x;
+          S2.nmaps = nm + 1;
+        } else {  // degenerate rejection: R is kept unchanged
+          K.sc.K = Kprev;
+          info |= kInfoDegenerate;
+          mass_kind = 0;
+        }
+        continue;
+      }
+      // ---- ResiSpec rejection (Algorithm 1, GetProxy)
+      float Z = __fsub_rn(qx, Rx);
+      if (zapp)  // max(Z*, |gap|), at most 1 - R(x0)
+        Z = fminf(fmaxf(nm == 0 ? zstar : 0.f, fabsf(Z)), __fsub_rn(1.f, Rx));
+      if (!(Z > 0.f)) {  // degenerate rejection: R is kept unchanged
+        info |= kInfoDegenerate;
+        continue;
       }
       if (nm >= kMaxMaps) { err |= kErrFanout; break; }
       mark(kPhaseRej);
       // one pass: the residual so far and the sums of the new map, in
       // unnormalised units (k: the new map's scalar).  The rejected tokens
       // get no special case here; their terms are taken out below.
-      float kq = __fdiv_rn(resi ? __fmul_rn(Z, dsc) : K.invSd, K.sig);
-      // s1: sum of min(k D~, R~) (ResiSpec) or of the capacity t (SpecInfer);
-      // s2: sum of t (ResiSpec), or in a level pass the sum of R~ where
+      float kq = __fdiv_rn(__fmul_rn(Z, dsc), K.sig);
+      // s1: sum of min(k D~, R~); s2: sum of t, or in a level pass the sum of R~ where
       // D~ > 0 (s1 for an unbounded k); s3 (level pass): the sum of D~ where
       // k D~ < R~, the slope of s1 in k.  All as pairs of lanes.  D~ is q~
       // unless the proxies replace the denominator (then the chain leaves it
       // in q[]).
       float2 s1p, s2p, s3p;
-      auto rej_pass = [&](auto kind_c, auto level_c) {
+      // the last child's rejection defines the final distribution when it
+      // leaves a map: its pass records it (ChunkRec kind 2)
+      const bool rec_last = rec_ok && next_sib[cn] < 0;
+      auto rej_pass = [&](auto kind_c, auto level_c, auto rec_c) {
         constexpr int KIND = decltype(kind_c)::value;
         constexpr bool LEVEL = decltype(level_c)::value;
-        const float2 c2 = dup2(K.c), nMt = dup2(-K.Mt), nMd = dup2(-K.Md), kq2 = dup2(kq),
-                     nkq = dup2(-kq);
-        stream_pass<THREADS, BF16>(ring, src, [&](const unsigned char* rt, const unsigned char* rd,
-                                                  int) -> bool {
+        constexpr bool REC = decltype(rec_c)::value;
+        const float2 c2 = dup2(K.c), nMt = dup2(-K.Mt), nMd = dup2(-K.Md), kq2 = dup2(kq);
+        stream_pass<THREADS, BF16, 2>(ring, src, primed, [&](const unsigned char* rt,
+                                                          const unsigned char* rd, int k) -> bool {
           float2 Rv[4], q[4];
           load_pairs<THREADS, BF16>(rt, Rv);  // -inf past the slice: 0
           load_pairs<THREADS, BF16>(rd, q);
@@ -1060,27 +1378,30 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
             q[j] = ex2x2(__ffma2_rn(q[j], c2, nMd));
           }
           float2 t[4];
-          if constexpr (KIND != kChainSpec) {
-            apply_chain_pairs<4, KIND>(S2, nm, Rv, q);
-            float2 m[4];
+          apply_chain_pairs<4, KIND>(S2, nm, Rv, q);
+          float2 m[4];
 #pragma unroll
-            for (int j = 0; j < 4; ++j) {
-              m[j] = min_part2(kq2, q[j], Rv[j]);
-              if constexpr (LEVEL) {
-                s3p.x += m[j].x < Rv[j].x ? q[j].x : 0.f;
-                s3p.y += m[j].y < Rv[j].y ? q[j].y : 0.f;
-                t[j] = make_float2(q[j].x > 0.f ? Rv[j].x : 0.f, q[j].y > 0.f ? Rv[j].y : 0.f);
-              } else {
-                t[j] = __ffma2_rn(m[j], dup2(-1.f), Rv[j]);
-              }
+          for (int j = 0; j < 4; ++j) {
+            m[j] = min_part2(kq2, q[j], Rv[j]);
+            if constexpr (LEVEL) {
+              s3p.x += m[j].x < Rv[j].x ? q[j].x : 0.f;
+              s3p.y += m[j].y < Rv[j].y ? q[j].y : 0.f;
+              t[j] = make_float2(q[j].x > 0.f ? Rv[j].x : 0.f, q[j].y > 0.f ? Rv[j].y : 0.f);
+            } else {
+              t[j] = __ffma2_rn(m[j], dup2(-1.f), Rv[j]);
             }
-            s1p = __fadd2_rn(s1p, __fadd2_rn(__fadd2_rn(m[0], m[1]), __fadd2_rn(m[2], m[3])));
-            s2p = __fadd2_rn(s2p, __fadd2_rn(__fadd2_rn(t[0], t[1]), __fadd2_rn(t[2], t[3])));
-          } else {
-            apply_chain_pairs<4, kChainSpec>(S2, nm, Rv, q);
-#pragma unroll
-            for (int j = 0; j < 4; ++j) t[j] = relu2(__ffma2_rn(nkq, q[j], Rv[j]));
-            s1p = __fadd2_rn(s1p, __fadd2_rn(__fadd2_rn(t[0], t[1]), __fadd2_rn(t[2], t[3])));
+          }
+          const float2 cm = __fadd2_rn(__fadd2_rn(m[0], m[1]), __fadd2_rn(m[2], m[3]));
+          const float2 ct = __fadd2_rn(__fadd2_rn(t[0], t[1]), __fadd2_rn(t[2], t[3]));
+          s1p = __fadd2_rn(s1p, cm);
+          s2p = __fadd2_rn(s2p, ct);
+          if constexpr (REC) {
+            const float wm = group_sum<5>(__fadd_rn(cm.x, cm.y));
+            const float wt = group_sum<5>(__fadd_rn(ct.x, ct.y));
+            if (lane == 0) {
+              S2.crec[0][k * NW + warp] = wm;
+              S2.crec[1][k * NW + warp] = wt;
+            }
           }
           return false;
         });
@@ -1099,25 +1420,33 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
       // fill places the rest on the tokens outside it.  Every CTA sees the
       // same exchanged sums, so all take the same steps.
       constexpr int kLevelSteps = 24;
-      const bool level = VAR && resi && P.level_fill != 0;
+      const bool level = VAR && P.level_fill != 0;
       bool timed_out = false, saturate = false;
       float s1, s2, s3;
       for (int step = 0;; ++step) {
         const bool lpass = level && !saturate;
         s1p = s2p = s3p = make_float2(0.f, 0.f);
         if (chain == kChainResiDenom) {
-          if (lpass) rej_pass(std::integral_constant<int, kChainResiDenom>{}, std::true_type{});
-          else rej_pass(std::integral_constant<int, kChainResiDenom>{}, std::false_type{});
-        } else if (chain == kChainResi) {
-          if (lpass) rej_pass(std::integral_constant<int, kChainResi>{}, std::true_type{});
-          else rej_pass(std::integral_constant<int, kChainResi>{}, std::false_type{});
+          if (lpass)
+            rej_pass(std::integral_constant<int, kChainResiDenom>{}, std::true_type{},
+                     std::false_type{});
+          else
+            rej_pass(std::integral_constant<int, kChainResiDenom>{}, std::false_type{},
+                     std::false_type{});
+        } else if (lpass) {
+          rej_pass(std::integral_constant<int, kChainResi>{}, std::true_type{}, std::false_type{});
+        } else if (!VAR && rec_last) {
+          rej_pass(std::integral_constant<int, kChainResi>{}, std::false_type{}, std::true_type{});
         } else {
-          rej_pass(std::integral_constant<int, kChainSpec>{}, std::false_type{});
+          rej_pass(std::integral_constant<int, kChainResi>{}, std::false_type{},
+                   std::false_type{});
         }
+        // the next pass over these rows starts its copies during the exchange
+        if (!src.held) stream_prime<THREADS, BF16>(ring, src, primed);
         s1 = __fadd_rn(s1p.x, s1p.y);
         s2 = __fadd_rn(s2p.x, s2p.y);
         s3 = __fadd_rn(s3p.x, s3p.y);
-        if (resi) {
+        {
           // The token just rejected (r(x0) = 0) and the earlier rejected ones
           // (R = 0 there) add nothing: the thread that summed each such token
           // of this slice subtracts the terms the pass gave it, recomputed
@@ -1170,7 +1499,7 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
       if (timed_out) { err |= kErrTimeout; break; }
       bool has_map = false;
       float a = 0.f, lam = 0.f;
-      if (resi) {
+      {
         const float S1 = __fmul_rn(o[0], K.sig), S2s = __fmul_rn(o[1], K.sig);
         const float delta = __fsub_rn(Z, S1);
         lam = S2s > 0.f && (!level || saturate) ? fminf(fmaxf(__fdiv_rn(delta, S2s), 0.f), 1.f)
@@ -1181,23 +1510,39 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
           a = __frcp_rn(norm);
           mass_kind = 2;
         }
-      } else {
-        const float Ssum = __fmul_rn(o[0], K.sig);
-        if (Ssum > 0.f) {
-          has_map = true;
-          a = __frcp_rn(Ssum);
-          mass_kind = 3;
-        }
+      }
+      if (has_map && !VAR && rec_last && !level) {
+        // The records hold every token's terms; the rejected tokens' residual
+        // is 0: thread 0 takes their terms out of their (chunk, warp) records
+        // in a fixed order (each distinct token once), recomputed as the pass
+        // computed them.
+        if (tid == 0)
+          for (int t = -1; t < nm; ++t) {
+            const int y = t < 0 ? x : S2.rej[t];
+            const int yk = t < 0 ? i : S2.rejk[t];
+            if (y < lo || y >= lo + nloc) continue;
+            bool seen = t >= 0 && y == x;
+            for (int t2 = 0; t2 < t && !seen; ++t2) seen = S2.rej[t2] == y;
+            if (seen) continue;
+            float Dy = exp_of(S2.kzd[yk], K.c, K.Md);
+            const float Ry = apply_chain<kChainResi>(S2, nm, exp_of(S2.kzt[yk], K.c, K.Mt), Dy);
+            const float my = fminf(__fmul_rn(kq, Dy), Ry);
+            const int off = y - lo;
+            const int r = (off / G::CE) * NW + ((off % G::CE) / VEC % THREADS) / 32;
+            S2.crec[0][r] = __fsub_rn(S2.crec[0][r], my);
+            S2.crec[1][r] = __fsub_rn(S2.crec[1][r], __fmaf_rn(my, -1.f, Ry));
+          }
+        crec = ChunkRec{2, lam, __fmul_rn(K.sig, a)};
       }
       if (has_map) {
         if (chain == kChainResiDenom)  // the proxy (1 - lambda) t~ becomes the denominator
           dsc = __fmul_rn(K.sig, __fsub_rn(1.f, lam));
         K.sig = __fmul_rn(K.sig, a);
-        // per-CTA masses of the new residual: (p0 + lambda p1) sig (ResiSpec)
-        // or p0 sig (SpecInfer) from this exchange's unnormalised partials
-        Pm = Pending{resi ? kResi : kSpec, x, K.sig, Z, lam};
+        // per-CTA masses of the new residual: (p0 + lambda p1) sig from this
+        // exchange's unnormalised partials
+        Pm = Pending{kResi, x, K.sig, Z, lam};
         // every thread, identical values (see the visit start)
-        S2.map[nm] = resi ? make_float2(kq, lam) : make_float2(-kq, 0.f);
+        S2.map[nm] = make_float2(kq, lam);
         S2.mdsc[nm] = dsc;
         S2.rej[nm] = x;
         S2.rejk[nm] = (int16_t)i;
@@ -1213,8 +1558,9 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
       // every child rejected: residual draw (Algorithm 1, last step)
       bool to = false;
       mark(kPhaseDraw);
-      if (!stream_sample<THREADS, BF16>(H, S2, F, ring, P, src, K, chain, mass_kind, Pm, S2.ufin,
-                                        b, depth, lo, rank, C, xp, xph, to))
+      if (!stream_sample<THREADS, BF16, SPEC>(H, S2, ring, P, src, K, chain, mass_kind, Pm,
+                                              S2.ufin, b, depth, lo, rank, C, xp, xph, to, primed,
+                                              crec))
         err |= kErrEmpty;
       if (to) err |= kErrTimeout;
       break;
@@ -1230,6 +1576,7 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
     __syncthreads();  // every read of this visit's S2 state precedes the next visit's writes
   }
 
+  stream_drain(primed);
   mark(kPhaseSetup);
   if (prof && rank == 0 && tid == 0)
     for (int k = 0; k < kPhases; ++k) P.out_phase[(size_t)b * kPhases + k] = (int64_t)S2.phc[k];

@@ -12,13 +12,9 @@ Parity rule (the tolerances of the verification hot path):
     are counted and reported;
   * the distribution of the final draw (for every sequence whose path
     matches) agrees within 1e-6 max-abs and 1e-5 L1 per row, and the GPU
-    row sums to 1 within 1e-6.
-    SpecInfer residuals are the one exception: each rejection divides
-    (R - q)_+ by its mass S_j, so an fp32 rounding of p or q (about 1e-7
-    relative, the floor of any fp32 normaliser) reaches the residual
-    multiplied by 1 / prod_j S_j.  Their rows use the same bounds scaled by
-    that factor, which the oracle reports per row ("cond"; 1 in every other
-    case).
+    row sums to 1 within 1e-6, in both modes (the kernel evaluates the
+    SpecInfer residual (p - C q)_+ / N with double-float sums and
+    exponentials where the residual's conditioning 1 / N demands them).
     Rows whose test denominator is the proxy (the EAGLE-integration
     variant) add, token by token, the oracle's first-order bound of the
     error of an fp32 evaluation of the chain ("dist_err"): the proxy
@@ -143,12 +139,13 @@ def compare(g, o, rows=None, check_dist=True, label=None):
         ok = same_path & ~errs
         if ok.any():
             diff = np.abs(gd[ok] - o["dist"][ok])
-            scale = np.maximum(1.0, o["cond"][ok])
             bar = o["dist_err"][ok] if "dist_err" in o else np.zeros_like(diff)
-            over = (diff - bar) / scale[:, None]
-            worst = over.max()
-            l1 = np.maximum(diff - bar, 0).sum(axis=1) / scale
-            rep.update(dist_rows=int(ok.sum()), dist_maxabs=float(worst), dist_l1=float(l1.max()))
+            worst = (diff - bar).max()
+            l1 = np.maximum(diff - bar, 0).sum(axis=1)
+            rep.update(dist_rows=int(ok.sum()), dist_maxabs=float(worst), dist_l1=float(l1.max()),
+                       dist_maxabs_raw=float(diff.max()),
+                       dist_l1_raw=float(diff.sum(axis=1).max()),
+                       cond_max=float(o["cond"][ok].max()))
             assert worst <= DIST_MAXABS, f"dist max-abs {worst:.3e} beyond the error bound"
             assert l1.max() <= DIST_L1, f"dist L1 {l1.max():.3e}"
             sums = gd[ok].sum(axis=1)
@@ -157,5 +154,7 @@ def compare(g, o, rows=None, check_dist=True, label=None):
     REPORTS.append(rep)
     print(f"parity {rep['label']}: {rep['sequences']} sequences, near ties {rep['near_tie']}, "
           f"mismatches in ties {rep['mismatch_in_ties']}, residual rows {rep['dist_rows']} "
-          f"(max-abs {rep['dist_maxabs']:.2e}, L1 {rep['dist_l1']:.2e})")
+          f"(max-abs {rep['dist_maxabs']:.2e}, L1 {rep['dist_l1']:.2e}; unscaled max-abs "
+          f"{rep.get('dist_maxabs_raw', 0.0):.2e}, L1 {rep.get('dist_l1_raw', 0.0):.2e}, "
+          f"largest 1/prod S {rep.get('cond_max', 1.0):.3g})")
     return rep

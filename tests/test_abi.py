@@ -5,6 +5,7 @@ import ctypes
 import os
 import re
 
+import numpy as np
 import pytest
 
 import paper_2608_24411_gb300 as rs
@@ -39,7 +40,7 @@ def test_library_exports_every_declared_symbol(lib):
     for n in declared_functions():
         assert hasattr(lib, n), n
     assert set(rs.EXPORTED) <= set(declared_functions())
-    assert lib.resispec_abi_version() == 3
+    assert lib.resispec_abi_version() == 4
 
 
 def test_opts_default_layout(lib):
@@ -85,7 +86,11 @@ def test_plan_without_device(lib):
     # clusters of 8; deep trees of 32 sequences in clusters of 8 (one wave)
     assert rs.plan(128, 16, 256000, 1, "bf16", kernel="stream")["cluster_size"] == 8
     assert rs.plan(32, 488, 256000, 6, "bf16", kernel="stream")["cluster_size"] == 8
-    assert p["uses_tma"] == 1
+    # the streaming kernel moves 16-byte vectors with per-thread asynchronous
+    # copies, not bulk (TMA) copies; the resident kernel uses bulk copies
+    assert p["uses_tma"] == 0 and p["vector_loads"] == 1
+    r = rs.plan(64, 62, 151936, 5, "f32", kernel="resident")
+    assert r["uses_tma"] == 1 and r["vector_loads"] == 1
     for B in (1, 7, 64, 128, 1000):
         p = rs.plan(B, 488, 256000, 6, "bf16", kernel="stream")
         assert p["smem_bytes"] <= 228 * 1024 // 2 - 1024
@@ -93,13 +98,14 @@ def test_plan_without_device(lib):
     assert p["kernel_name"] == "resident" and p["cluster_size"] in (8, 16)
     assert p["slice_elems"] * p["cluster_size"] >= 151936
     assert p["smem_bytes"] <= 227 * 1024
-    # a small batch that fits on chip stays resident
-    p = rs.plan(1, 60, 32000, 5, "bf16")
-    assert p["kernel_name"] == "resident"
+    # the automatic choice is the streaming kernel, also for a batch that
+    # would fit on chip; the resident kernel runs when asked for
+    assert rs.plan(1, 60, 32000, 5, "bf16")["kernel_name"] == "stream"
+    assert rs.plan(1, 60, 32000, 5, "bf16", kernel="resident")["kernel_name"] == "resident"
     p = rs.plan(1, 12, 64, 4, "f32", cluster_size=1)
     assert p["cluster_size"] == 1 and p["slice_elems"] == 64
     p = rs.plan(1, 12, 61, 4, "f32", cluster_size=2)
-    assert p["uses_tma"] == 0                      # 61 * 4 bytes per row: not 16-byte aligned
+    assert p["uses_tma"] == 0 and p["vector_loads"] == 0   # 61 * 4 bytes per row: not aligned
     p = rs.plan(1, 12, 64, 4, "bf16", no_tma=True)
     assert p["uses_tma"] == 0
     for V in (1, 7, 32000, 128256, 256000, rs.MAX_VOCAB):
@@ -120,6 +126,11 @@ def test_plan_without_device(lib):
     o = rs.make_opts(kernel="stream")
     o.flags |= rs.FLAG_RESIDENT                   # both kernels forced: argument error
     assert lib.resispec_plan(rs.Dims(1, 2, 10, 1, rs.F32), o, None) == rs.E_ARG
+    # SpecInfer runs on the streaming kernel only (its residual is evaluated
+    # from the raw logits, which the resident kernel does not keep)
+    assert rs.plan(1, 60, 32000, 5, "bf16", mode=rs.MODE_SPECINFER)["kernel_name"] == "stream"
+    o = rs.make_opts(mode=rs.MODE_SPECINFER, kernel="resident")
+    assert lib.resispec_plan(rs.Dims(1, 60, 32000, 5, rs.BF16), o, None) == rs.E_ARG
     # the variants run on the streaming kernel only
     for kw in (dict(z_rule=rs.Z_RULE_APPLIED), dict(proxy_denominator=True),
                dict(fill=rs.FILL_LEVEL)):
@@ -188,4 +199,102 @@ int main(void) {
                     str(src), "-o", str(exe), "-L", libdir, "-lresispec",
                     f"-Wl,-rpath,{libdir}"], check=True)
     out = subprocess.run([str(exe)], capture_output=True, text=True, check=True).stdout.split()
-    assert out == ["3", "1", "1"]
+    assert out == ["4", "1", "1"]
+
+
+@pytest.mark.gpu
+def test_c_program_verifies_a_batch_on_the_device(tmp_path, lib):
+    """A C program (no Python on its path) allocates device buffers with the
+    CUDA runtime, copies a batch in, calls resispec_verify and copies the
+    accepted tokens and accept lengths back; they match the fp64 oracle on
+    every sequence away from a near tie."""
+    import shutil
+    import subprocess
+    import oracle
+    from paper_2608_24411_gb300 import workloads as W
+    gcc = shutil.which("gcc")
+    cuda = "/usr/local/cuda"
+    if gcc is None or not os.path.exists(os.path.join(cuda, "include", "cuda_runtime_api.h")):
+        pytest.skip("no C compiler or CUDA headers")
+    w = W.WORKLOADS["tiny-chain-v64"]
+    B = 512
+    inp = W.make_inputs_np(w, seed=21, batch=B)
+    N, V, D = w.num_nodes, w.vocab, w.max_depth
+    seed = 2024
+    src = tmp_path / "c_verify.c"
+    src.write_text(r'''
+#include <stdio.h>
+#include <stdlib.h>
+#include <stdint.h>
+#include <cuda_runtime_api.h>
+#include "resispec.h"
+static void* slurp(const char* path, size_t n) {
+  void* p = malloc(n);
+  FILE* f = fopen(path, "rb");
+  if (!f || fread(p, 1, n, f) != n) { fprintf(stderr, "read %s\n", path); exit(2); }
+  fclose(f);
+  return p;
+}
+static void* to_device(const void* h, size_t n) {
+  void* d = 0;
+  if (cudaMalloc(&d, n) != cudaSuccess || cudaMemcpy(d, h, n, cudaMemcpyHostToDevice) != cudaSuccess) {
+    fprintf(stderr, "device copy failed\n"); exit(3);
+  }
+  return d;
+}
+int main(int argc, char** argv) {
+  const int B = atoi(argv[2]), N = atoi(argv[3]), V = atoi(argv[4]), D = atoi(argv[5]);
+  const float T = (float)atof(argv[6]);
+  const uint64_t seed = strtoull(argv[7], 0, 10);
+  char path[4096];
+  const size_t nlog = (size_t)B * (N + 1) * V * sizeof(float);
+  snprintf(path, sizeof path, "%s/target.bin", argv[1]);
+  void* t = to_device(slurp(path, nlog), nlog);
+  snprintf(path, sizeof path, "%s/draft.bin", argv[1]);
+  void* d = to_device(slurp(path, nlog), nlog);
+  snprintf(path, sizeof path, "%s/parents.bin", argv[1]);
+  int32_t* par = (int32_t*)to_device(slurp(path, N * 4), N * 4);
+  snprintf(path, sizeof path, "%s/cand.bin", argv[1]);
+  int32_t* cand = (int32_t*)to_device(slurp(path, (size_t)B * N * 4), (size_t)B * N * 4);
+  int32_t *tok = 0, *len = 0;
+  cudaMalloc((void**)&tok, (size_t)B * (D + 1) * 4);
+  cudaMalloc((void**)&len, (size_t)B * 4);
+  resispec_dims dims = {B, N, V, D, RESISPEC_F32};
+  int rc = resispec_verify(t, d, par, cand, T, seed, tok, len, dims, 0);
+  if (rc != RESISPEC_OK) { fprintf(stderr, "verify: %s\n", resispec_status_string(rc)); return 4; }
+  if (cudaDeviceSynchronize() != cudaSuccess) { fprintf(stderr, "sync failed\n"); return 5; }
+  int32_t* htok = (int32_t*)malloc((size_t)B * (D + 1) * 4);
+  int32_t* hlen = (int32_t*)malloc((size_t)B * 4);
+  cudaMemcpy(htok, tok, (size_t)B * (D + 1) * 4, cudaMemcpyDeviceToHost);
+  cudaMemcpy(hlen, len, (size_t)B * 4, cudaMemcpyDeviceToHost);
+  snprintf(path, sizeof path, "%s/out.bin", argv[1]);
+  FILE* f = fopen(path, "wb");
+  fwrite(htok, 4, (size_t)B * (D + 1), f);
+  fwrite(hlen, 4, (size_t)B, f);
+  fclose(f);
+  cudaFree(t); cudaFree(d); cudaFree(par); cudaFree(cand); cudaFree(tok); cudaFree(len);
+  return 0;
+}
+''')
+    for name in ("target", "draft"):
+        np.ascontiguousarray(inp[name], np.float32).tofile(tmp_path / f"{name}.bin")
+    np.ascontiguousarray(inp["parents"], np.int32).tofile(tmp_path / "parents.bin")
+    np.ascontiguousarray(inp["cand"], np.int32).tofile(tmp_path / "cand.bin")
+    libdir = os.path.dirname(rs._build.LIB)
+    cudalib = next((p for p in (os.path.join(cuda, "lib64"), os.path.join(cuda, "lib"))
+                    if os.path.exists(p)), os.path.join(cuda, "lib64"))
+    exe = tmp_path / "c_verify"
+    subprocess.run([gcc, "-std=c11", "-Wall", "-Werror", "-I", os.path.join(ROOT, "include"),
+                    "-I", os.path.join(cuda, "include"), str(src), "-o", str(exe),
+                    "-L", libdir, "-lresispec", "-L", cudalib, "-lcudart",
+                    f"-Wl,-rpath,{libdir}", f"-Wl,-rpath,{cudalib}"], check=True)
+    subprocess.run([str(exe), str(tmp_path), str(B), str(N), str(V), str(D), repr(w.temperature),
+                    str(seed)], check=True, timeout=120)
+    out = np.fromfile(tmp_path / "out.bin", dtype=np.int32)
+    toks, alen = out[: B * (D + 1)].reshape(B, D + 1), out[B * (D + 1):]
+    o = oracle.verify(inp["target"], inp["draft"], inp["parents"], inp["cand"], w.temperature,
+                      seed, max_depth=D)
+    clean = (o["accept_margin"] > 1e-5) & (o["sample_margin"] > 1e-6)
+    assert clean.sum() >= 0.99 * B
+    np.testing.assert_array_equal(alen[clean], o["accept_len"][clean])
+    np.testing.assert_array_equal(toks[clean], o["tokens"][clean])

@@ -129,3 +129,21 @@ def test_cpu_oracle_rate_on_host_inputs(wl):
         np.arange(4, dtype=np.int32), oracle.MODE_RESISPEC, 0.05, 1, {"fill": 1})
     assert rate > 0 and one > 0 and 1 <= threads <= 4 and "verified nodes" in sample
     assert isinstance(bench.cpu_model(), str)
+
+
+def test_parity_sample_counts_ties_and_mismatches():
+    """bench.parity_sample on hand-made outputs: a difference inside the tie
+    band is counted as such, one outside it separately, and the near-tie
+    counts follow the oracle's margins level by level."""
+    o = {"accept_len": np.array([1, 2, 0, 1]), "tokens": np.array([[5, 7, -1], [5, 6, 9], [3, -1, -1], [4, 4, -1]]),
+         "nodes": np.array([[0, -1], [0, 2], [-1, -1], [1, -1]]), "rejects": np.array([0, 1, 2, 1]),
+         "accept_margin": np.array([0.3, 5e-6, 0.2, 2e-8]), "sample_margin": np.array([0.1, 0.2, 5e-7, 0.4])}
+    g = {k: np.array(v, copy=True) for k, v in o.items() if k in ("accept_len", "tokens", "nodes", "rejects")}
+    g["tokens"][1, 2] = 8      # sequence 1 differs: accept margin 5e-6 is a near tie
+    g["tokens"][0, 1] = 3      # sequence 0 differs with no near tie
+    r = bench.parity_sample(g, o)
+    assert r["sequences"] == 4
+    assert r["mismatch_in_ties"] == 1 and r["mismatch_outside_ties"] == 1
+    assert r["near_tie"]["accept<=1e-05"] == 2 and r["near_tie"]["accept<=1e-06"] == 1
+    assert r["near_tie"]["accept<=1e-07"] == 1 and r["near_tie"]["sample<=1e-06"] == 1
+    assert r["near_tie"]["sample<=1e-07"] == 0

@@ -1,5 +1,7 @@
 """GPU parity: the CUDA verification path against the fp64 oracle on the
 same seeded inputs, through the C ABI (see tests/parity.py for the rule)."""
+import functools
+
 import numpy as np
 import pytest
 from scipy.special import softmax as sp_softmax
@@ -22,6 +24,14 @@ def built():
     rs.load_library()
 
 
+@functools.lru_cache(maxsize=2)
+def _inputs(name, seed, batch):
+    """make_inputs_np for a named workload, kept for the next test with the
+    same inputs (parametrized tests run next to each other); callers must
+    not modify the arrays."""
+    return W.make_inputs_np(W.WORKLOADS[name], seed=seed, batch=batch)
+
+
 def _np_inputs_to_gpu(inp):
     import torch
     return (P.to_device(inp["target"]), P.to_device(inp["draft"]),
@@ -29,9 +39,21 @@ def _np_inputs_to_gpu(inp):
             torch.as_tensor(inp["cand"], dtype=torch.int32, device="cuda"))
 
 
+def _refused_on_resident(zt, zd, pa, ca, T, seed, D, **kw):
+    """SpecInfer runs on the streaming kernel only: forcing the resident
+    kernel is an argument error, returned before any launch."""
+    with pytest.raises(rs.ResispecError) as e:
+        P.run_gpu(zt, zd, pa, ca, T, seed, D, mode=rs.MODE_SPECINFER, kernel="resident", **kw)
+    assert e.value.code == rs.E_ARG
+
+
 def _check(inp, mode, seed, **kw):
     zt, zd, pa, ca = _np_inputs_to_gpu(inp)
     D = int(inp["max_depth"])
+    if mode == rs.MODE_SPECINFER and kw.get("kernel") == "resident":
+        _refused_on_resident(zt, zd, pa, ca, inp["temperature"], seed, D,
+                             **{k: v for k, v in kw.items() if k != "kernel"})
+        return None, None
     g = P.run_gpu(zt, zd, pa, ca, inp["temperature"], seed, D, mode=mode, **kw)
     o = P.run_oracle(inp["target"], inp["draft"], inp["parents"], inp["cand"],
                      inp["temperature"], seed, D, mode, z_rule=kw.get("z_rule", 0),
@@ -76,7 +98,7 @@ def test_parity_tiny_chain_10000(mode, cluster, kernel):
 @pytest.mark.parametrize("mode", MODES)
 def test_parity_tree60_v32000(mode, kernel):
     w = W.WORKLOADS["tree60-v32000"]
-    inp = W.make_inputs_np(w, seed=1, batch=256)
+    inp = _inputs(w.name, 1, 256)
     _check(inp, mode, seed=11, kernel=kernel)
 
 
@@ -165,7 +187,7 @@ def test_wide_fanout(mode):
     candidate: every test rejects, the walk reaches the last child, 128
     residual maps) on both kernels; one child more: the streaming kernel
     reports ERR_FANOUT when the walk reaches the 129th child, the resident
-    kernel verifies."""
+    kernel verifies (ResiSpec; SpecInfer runs on the streaming kernel only)."""
     import torch
     V = 3000
     for kids in (rs.MAX_FANOUT_STREAM, rs.MAX_FANOUT_STREAM + 1):
@@ -312,6 +334,10 @@ def _sampled_parity(w, seed, call_seed, rows, mode=rs.MODE_RESISPEC, batch=None,
     import torch
     inp = W.make_inputs_torch(w, seed, "cuda", batch=batch, rho=rho)
     D = inp["max_depth"]
+    if mode == rs.MODE_SPECINFER and kernel == "resident":
+        _refused_on_resident(inp["target"], inp["draft"], inp["parents"], inp["cand"],
+                             w.temperature, call_seed, D, **kw)
+        return None
     g = P.run_gpu(inp["target"], inp["draft"], inp["parents"], inp["cand"], w.temperature,
                   call_seed, D, mode=mode, kernel=kernel, **kw)
     ridx = torch.as_tensor(rows, device="cuda")
@@ -387,8 +413,7 @@ def test_parity_tree488_v256000_kernels(kernel):
 # ------------------------------------------------------------ exactness on the GPU
 
 
-@pytest.mark.parametrize("kernel", KERNELS)
-def test_gpu_specinfer_million_draws_v32000(kernel):
+def test_gpu_specinfer_million_draws_v32000(kernel="stream"):
     """SpecInfer mode is distribution-exact: 1e6 GPU draws at V = 32000 (one
     shared set of rows, fresh candidates per draw) do not reject p."""
     import torch
@@ -500,7 +525,7 @@ def test_parity_z_applied_budget(V, dtype):
 
 def test_parity_z_applied_tree60():
     w = W.WORKLOADS["tree60-v32000"]
-    inp = W.make_inputs_np(w, seed=8, batch=256)
+    inp = _inputs(w.name, 8, 256)
     _check(inp, rs.MODE_RESISPEC, seed=88, z_rule=rs.Z_RULE_APPLIED)
 
 
@@ -511,7 +536,7 @@ def test_parity_proxy_denominator(wl):
     sequence against the oracle with the same rule, which must change some
     walks."""
     w = W.WORKLOADS[wl]
-    inp = W.make_inputs_np(w, seed=13, batch=256 if wl != "chain8x4-v128256-b16" else 16)
+    inp = _inputs(w.name, 13, 256 if wl != "chain8x4-v128256-b16" else 16)
     g, o = _check(inp, rs.MODE_RESISPEC, seed=131, proxy_denominator=True)
     o0 = P.run_oracle(inp["target"], inp["draft"], inp["parents"], inp["cand"],
                       inp["temperature"], 131, int(inp["max_depth"]), rs.MODE_RESISPEC)
@@ -572,7 +597,7 @@ def test_parity_level_fill(wl):
     Z): every sequence against the oracle's exact level, which must change
     some walks against the default fill."""
     w = W.WORKLOADS[wl]
-    inp = W.make_inputs_np(w, seed=17, batch=256 if wl != "chain8x4-v128256-b16" else 16)
+    inp = _inputs(w.name, 17, 256 if wl != "chain8x4-v128256-b16" else 16)
     g, o = _check(inp, rs.MODE_RESISPEC, seed=171, fill=rs.FILL_LEVEL)
     o0 = P.run_oracle(inp["target"], inp["draft"], inp["parents"], inp["cand"],
                       inp["temperature"], 171, int(inp["max_depth"]), rs.MODE_RESISPEC)
@@ -585,7 +610,7 @@ def test_parity_level_fill_with_other_variants(other):
     """The level fill combined with the proxy denominator (the level is
     taken against the current denominator) and with the Z_applied budget."""
     w = W.WORKLOADS["tree60-v32000"]
-    inp = W.make_inputs_np(w, seed=19, batch=256)
+    inp = _inputs(w.name, 19, 256)
     _check(inp, rs.MODE_RESISPEC, seed=191, fill=rs.FILL_LEVEL, **other)
 
 
@@ -736,7 +761,7 @@ def test_parity_drafting(wl, mode):
     from the node's draft distribution, then verifies them; tokens, accept
     lengths and drafted candidates against the oracle's drafting walk."""
     w = W.WORKLOADS[wl]
-    inp = W.make_inputs_np(w, seed=17, batch=256 if wl != "chain8x4-v128256-b16" else 16)
+    inp = _inputs(w.name, 17, 256 if wl != "chain8x4-v128256-b16" else 16)
     gd, _ = _check_drafting(inp, mode, seed=170 + mode)
     assert (gd[:, :1] >= 0).all()   # the root's first child is always drawn
 
@@ -756,3 +781,26 @@ def test_gpu_drafted_candidates_follow_q():
     d = drafted.cpu().numpy()
     assert (d[:, 0] >= 0).all()
     assert chisq_pvalue(np.bincount(d[:, 0], minlength=V), q)[0] > 1e-4
+
+
+def test_specinfer_residual_ill_conditioned():
+    """SpecInfer rows whose residual mass N = prod S_j is small: a draft
+    close to the target (rho 0.98) and 6 forced rejections of tokens the
+    target excludes (draft ranks 300-305) drive 1 / N into the thousands on
+    some rows, where the residual (p - C q)_+ / N magnifies any relative
+    error of its sums and exponentials by p / N; the kernel's double-float
+    evaluation meets the flat 1e-6 on every row."""
+    V, kids, B = 32000, 6, 64
+    rng = np.random.default_rng(77)
+    zt = (3.0 * rng.normal(0, 1, (B, kids + 1, V))
+          - np.log(rng.permuted(np.tile(np.arange(1, V + 1), (B, kids + 1, 1)), axis=2)))
+    zd = 0.98 * zt + np.sqrt(1 - 0.98 ** 2) * 3.0 * rng.normal(0, 1, zt.shape)
+    zt, zd = zt.astype(np.float32), zd.astype(np.float32)
+    cand = np.argsort(-zd[:, 0], axis=1)[:, 300:300 + kids].astype(np.int32)
+    for b in range(B):
+        zt[b, 0, cand[b]] = -30.0          # the target all but excludes them: every test rejects
+    inp = {"target": zt, "draft": zd, "parents": np.full(kids, -1, np.int32), "cand": cand,
+           "temperature": 1.0, "max_depth": 1}
+    g, o = _check(inp, rs.MODE_SPECINFER, seed=5, kernel="stream")
+    assert (o["rejects"] == kids).all()
+    assert o["cond"].max() > 1000.0, o["cond"].max()   # 1 / N: the conditioning under test

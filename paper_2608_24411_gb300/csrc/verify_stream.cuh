@@ -167,20 +167,25 @@ __device__ __forceinline__ void load_pairs(const unsigned char* row, float2 (&z)
 // Ring layout of a pass: a pass over both rows keeps S stages of SB bytes
 // (target row, then draft row); a pass over the target row alone keeps 2 S
 // stages of RB bytes, twice as many chunks in flight.  Chunk k of a pass
-// lives in stage k mod DEPTH.
-template <int THREADS, bool BF16, bool TWO>
-struct Lay {
+// lives in stage k mod depth.  The layout is chosen at run time, so each
+// pass body is compiled once.
+template <int THREADS, bool BF16>
+__device__ __forceinline__ int ring_depth(bool two) {
   using G = StreamGeom<THREADS, BF16>;
-  static constexpr int DEPTH = TWO ? G::S : 2 * G::S;
-  static constexpr uint32_t STRIDE = TWO ? G::SB : G::RB;
-};
+  return two ? G::S : 2 * G::S;
+}
+template <int THREADS, bool BF16>
+__device__ __forceinline__ uint32_t ring_stride(bool two) {
+  using G = StreamGeom<THREADS, BF16>;
+  return two ? G::SB : G::RB;
+}
 
 // Copies this thread's vectors of chunk k into ring stage `st` (the copies
 // of one chunk form one cp.async group): the target row, and the draft row
-// RB bytes further when TWO.  Aligned rows: 16-byte asynchronous copies;
+// RB bytes further when `two`.  Aligned rows: 16-byte asynchronous copies;
 // other rows: element loads stored synchronously.
-template <int THREADS, bool BF16, bool TWO>
-__device__ __forceinline__ void copy_chunk(const Src& s, int k, unsigned char* st) {
+template <int THREADS, bool BF16>
+__device__ __forceinline__ void copy_chunk(const Src& s, int k, unsigned char* st, bool two) {
   using G = StreamGeom<THREADS, BF16>;
   constexpr int VEC = G::VEC;
   constexpr int es = BF16 ? 2 : 4;
@@ -195,10 +200,10 @@ __device__ __forceinline__ void copy_chunk(const Src& s, int k, unsigned char* s
       // nloc is a multiple of VEC on this path: a vector is whole or absent
       if (e0 < s.nloc) {
         cp_async16(dt, s.t + (size_t)e0 * es);
-        if constexpr (TWO) cp_async16(dd, s.d + (size_t)e0 * es);
+        if (two) cp_async16(dd, s.d + (size_t)e0 * es);
       } else {
         *dt = ninf;
-        if constexpr (TWO) *dd = ninf;
+        if (two) *dd = ninf;
       }
     } else {
       uint32_t wt[4], wd[4];
@@ -211,7 +216,7 @@ __device__ __forceinline__ void copy_chunk(const Src& s, int k, unsigned char* s
             const int e = e0 + 2 * i + j;
             const bool in = e < s.nloc;
             lt[j] = in ? (uint32_t)__ldg(reinterpret_cast<const uint16_t*>(s.t) + e) : 0xff80u;
-            ld[j] = (TWO && in) ? (uint32_t)__ldg(reinterpret_cast<const uint16_t*>(s.d) + e)
+            ld[j] = (two && in) ? (uint32_t)__ldg(reinterpret_cast<const uint16_t*>(s.d) + e)
                                 : 0xff80u;
           }
           wt[i] = lt[0] | (lt[1] << 16);
@@ -221,12 +226,12 @@ __device__ __forceinline__ void copy_chunk(const Src& s, int k, unsigned char* s
           const bool in = e < s.nloc;
           wt[i] = in ? __float_as_uint(__ldg(reinterpret_cast<const float*>(s.t) + e))
                      : 0xff800000u;
-          wd[i] = (TWO && in) ? __float_as_uint(__ldg(reinterpret_cast<const float*>(s.d) + e))
+          wd[i] = (two && in) ? __float_as_uint(__ldg(reinterpret_cast<const float*>(s.d) + e))
                               : 0xff800000u;
         }
       }
       *dt = make_uint4(wt[0], wt[1], wt[2], wt[3]);
-      if constexpr (TWO) *dd = make_uint4(wd[0], wd[1], wd[2], wd[3]);
+      if (two) *dd = make_uint4(wd[0], wd[1], wd[2], wd[3]);
     }
   }
   cp_async_commit();
@@ -235,51 +240,17 @@ __device__ __forceinline__ void copy_chunk(const Src& s, int k, unsigned char* s
 // Chunk k's stage when the slice is held in the ring (see Src::held).
 template <int THREADS, bool BF16>
 __device__ __forceinline__ unsigned char* held_stage(unsigned char* ring, const Src& s, int k) {
-  using G = StreamGeom<THREADS, BF16>;
-  return ring + (size_t)k * (s.rows == 2 ? G::SB : G::RB);
+  return ring + (size_t)k * ring_stride<THREADS, BF16>(s.rows == 2);
 }
 
-// The pass proper for a given layout (see stream_pass_pre).
-template <int THREADS, bool BF16, bool TWO, class Pre, class Body>
-__device__ __forceinline__ void stream_pass_lay(unsigned char* ring, const Src& s, bool& primed,
-                                                Pre&& pre, Body&& body) {
-  using G = StreamGeom<THREADS, BF16>;
-  using Y = Lay<THREADS, BF16, TWO>;
-  constexpr int S = Y::DEPTH;
-  const int NK = (s.nloc + G::CE - 1) / G::CE;
-  if (!primed) {
-#pragma unroll
-    for (int k = 0; k < S - 1; ++k) {
-      if (k < NK) copy_chunk<THREADS, BF16, TWO>(s, k, ring + k * Y::STRIDE);
-      else cp_async_commit();
-    }
-  }
-  primed = false;
-  pre();
-  int slot = 0;
-  for (int k = 0; k < NK; ++k) {
-    const int kn = k + S - 1;
-    const int nslot = slot == 0 ? S - 1 : slot - 1;  // (k + S - 1) % S
-    if (kn < NK) copy_chunk<THREADS, BF16, TWO>(s, kn, ring + nslot * Y::STRIDE);
-    else cp_async_commit();
-    cp_async_wait<S - 1>();  // chunk k's copies (this thread's) have landed
-    const unsigned char* st = ring + slot * Y::STRIDE;
-    const bool stop = body(st, st + G::RB, k);
-    slot = slot == S - 1 ? 0 : slot + 1;
-    if (stop) break;
-  }
-  cp_async_wait<0>();
-}
-
-// Streams the slice chunk by chunk, DEPTH - 1 chunks ahead (Lay), calling
-// body(target_stage_row, draft_stage_row, k) with all threads (the draft
-// pointer is meaningful only for passes over both rows); body returns true
-// (uniformly) to end the pass.  pre() runs once, after the first copies are
-// issued.  When `primed` is set the first chunks were issued earlier by
-// stream_prime over the same rows and are not issued again (the flag is
-// cleared).  On return every copy of the pass has landed.
-// ROWS: 2 or 1 when the caller knows s.rows (only that layout's loop is
-// compiled), 0 to dispatch on it.
+// Streams the slice chunk by chunk, depth - 1 chunks ahead (the layout
+// above), calling body(target_stage_row, draft_stage_row, k) with all
+// threads (the draft pointer is meaningful only for passes over both rows);
+// body returns true (uniformly) to end the pass.  pre() runs once, after the
+// first copies are issued.  When `primed` is set the first chunks were
+// issued earlier by stream_prime over the same rows and are not issued again
+// (the flag is cleared).  On return every copy of the pass has landed.
+// ROWS: 2 or 1 when the caller knows s.rows, 0 to read it.
 template <int THREADS, bool BF16, int ROWS = 0, class Pre, class Body>
 __device__ __forceinline__ void stream_pass_pre(unsigned char* ring, const Src& s, bool& primed,
                                                 Pre&& pre, Body&& body) {
@@ -293,10 +264,32 @@ __device__ __forceinline__ void stream_pass_pre(unsigned char* ring, const Src& 
     }
     return;
   }
-  if (ROWS == 2 || (ROWS == 0 && s.rows == 2))
-    stream_pass_lay<THREADS, BF16, true>(ring, s, primed, pre, body);
-  else
-    stream_pass_lay<THREADS, BF16, false>(ring, s, primed, pre, body);
+  const bool two = ROWS == 2 || (ROWS == 0 && s.rows == 2);
+  const int S = ring_depth<THREADS, BF16>(two);
+  const uint32_t stride = ring_stride<THREADS, BF16>(two);
+  if (!primed) {
+    for (int k = 0; k < S - 1; ++k) {
+      if (k < NK) copy_chunk<THREADS, BF16>(s, k, ring + k * stride, two);
+      else cp_async_commit();
+    }
+  }
+  primed = false;
+  pre();
+  int slot = 0;
+  for (int k = 0; k < NK; ++k) {
+    const int kn = k + S - 1;
+    const int nslot = slot == 0 ? S - 1 : slot - 1;  // (k + S - 1) % S
+    if (kn < NK) copy_chunk<THREADS, BF16>(s, kn, ring + nslot * stride, two);
+    else cp_async_commit();
+    // chunk k's copies (this thread's) have landed
+    if (two) cp_async_wait<G::S - 1>();
+    else cp_async_wait<2 * G::S - 1>();
+    const unsigned char* st = ring + slot * stride;
+    const bool stop = body(st, st + G::RB, k);
+    slot = slot == S - 1 ? 0 : slot + 1;
+    if (stop) break;
+  }
+  cp_async_wait<0>();
 }
 
 template <int THREADS, bool BF16, int ROWS = 0, class Body>
@@ -305,7 +298,7 @@ __device__ __forceinline__ void stream_pass(unsigned char* ring, const Src& s, b
   stream_pass_pre<THREADS, BF16, ROWS>(ring, s, primed, [] {}, body);
 }
 
-// Issues the copies a pass over s starts with (its first DEPTH - 1 chunks,
+// Issues the copies a pass over s starts with (its first depth - 1 chunks,
 // into the ring stages it reads them from), so that they travel while the
 // CTA waits in a cluster exchange.  Every thread copies only into its own
 // slots, which its previous pass has finished reading, so no barrier is
@@ -315,20 +308,12 @@ template <int THREADS, bool BF16>
 __device__ __forceinline__ void stream_prime(unsigned char* ring, const Src& s, bool& primed) {
   using G = StreamGeom<THREADS, BF16>;
   const int NK = (s.nloc + G::CE - 1) / G::CE;
-  if (s.rows == 2) {
-    using Y = Lay<THREADS, BF16, true>;
-#pragma unroll
-    for (int k = 0; k < Y::DEPTH - 1; ++k) {
-      if (k < NK) copy_chunk<THREADS, BF16, true>(s, k, ring + k * Y::STRIDE);
-      else cp_async_commit();
-    }
-  } else {
-    using Y = Lay<THREADS, BF16, false>;
-#pragma unroll
-    for (int k = 0; k < Y::DEPTH - 1; ++k) {
-      if (k < NK) copy_chunk<THREADS, BF16, false>(s, k, ring + k * Y::STRIDE);
-      else cp_async_commit();
-    }
+  const bool two = s.rows == 2;
+  const int S = ring_depth<THREADS, BF16>(two);
+  const uint32_t stride = ring_stride<THREADS, BF16>(two);
+  for (int k = 0; k < S - 1; ++k) {
+    if (k < NK) copy_chunk<THREADS, BF16>(s, k, ring + k * stride, two);
+    else cp_async_commit();
   }
   primed = true;
 }
@@ -396,7 +381,7 @@ __device__ __forceinline__ float2 exp_sum8(const float2 (&z)[4], float2 c2, floa
 template <bool TWO>
 __device__ __forceinline__ float2 norm_accumulate(const float2 (&zt)[4], const float2 (&zd)[4],
                                                   float c, float& mt, float2& st, float& md,
-                                                  float2& sd) {
+                                                  float2& sd, float2& dpart) {
   const float vt = max8(zt);
   const bool rt = __fmaf_rn(vt, c, -mt) > 0.f;
   float vd = 0.f;
@@ -413,7 +398,10 @@ __device__ __forceinline__ float2 norm_accumulate(const float2 (&zt)[4], const f
   const float2 c2 = dup2(c);
   const float2 part = exp_sum8(zt, c2, dup2(-mt));  // this chunk's target terms
   st = __fadd2_rn(st, part);
-  if constexpr (TWO) sd = __fadd2_rn(sd, exp_sum8(zd, c2, dup2(-md)));
+  if constexpr (TWO) {
+    dpart = exp_sum8(zd, c2, dup2(-md));  // and its draft terms
+    sd = __fadd2_rn(sd, dpart);
+  }
   return part;
 }
 
@@ -690,8 +678,7 @@ __device__ int stream_search(Head& H, const StreamHead& S2, unsigned long long* 
     stg = held_stage<THREADS, BF16>(ring, s, ks);
   } else {
     stream_drain(primed);
-    if (s.rows == 2) copy_chunk<THREADS, BF16, true>(s, ks, ring);
-    else copy_chunk<THREADS, BF16, false>(s, ks, ring);
+    copy_chunk<THREADS, BF16>(s, ks, ring, s.rows == 2);
     cp_async_wait<0>();
   }
   float v[G::VPT][VEC];
@@ -923,6 +910,10 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
   // chunk records for the final draw (ChunkRec; not in the instance with the
   // optional paths)
   const bool rec_ok = !VAR && ((nloc + G::CE - 1) / G::CE) * NW <= kMaxChunkRecs;
+  // drafting: the normaliser records the draft row's chunk masses, from
+  // which every child's draw finds its chunk (ChunkRec kind 1 on q)
+  const bool rec_draft = VAR && P.draft_out != nullptr &&
+                         ((nloc + G::CE - 1) / G::CE) * NW <= kMaxChunkRecs;
 
   // Kernel setup: exchange barriers, the tree's child lists and the
   // candidates.  It runs while the first chunks of the root's rows are in
@@ -1012,7 +1003,7 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
       if (owner[i] != (int)rank) continue;
       const int pick = stream_search<THREADS, BF16, SPEC>(
           H, S2, reinterpret_cast<unsigned long long*>(S2.map), ring, sq, Kq, chain, lo, tau[i],
-          primed, ChunkRec{0, 0.f, 0.f});
+          primed, ChunkRec{rec_draft ? 1 : 0, K.Md, K.invSd});
       if (tid == 0) P.draft_out[(size_t)b * N + cn] = lo + max(pick, 0);
     }
     cluster_sync();  // every drawn token written (release / acquire at cluster scope)
@@ -1115,10 +1106,22 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
           load_pairs<THREADS, BF16>(rt, zt);
           if (need_draft) {
             load_pairs<THREADS, BF16>(rd, zd);
-            norm_accumulate<true>(zt, zd, P.scale_log2, mt, st2, md, sd2);
+            float2 dpart;
+            norm_accumulate<true>(zt, zd, P.scale_log2, mt, st2, md, sd2, dpart);
+            if (rec_draft) {
+              const float mw = redux_max(md);
+              const float sw =
+                  group_sum<5>(__fmul_rn(__fadd_rn(dpart.x, dpart.y), ex2(__fsub_rn(md, mw))));
+              if (lane == 0) {
+                S2.crec[0][k * NW + warp] = mw;
+                S2.crec[1][k * NW + warp] = sw;
+              }
+            }
             if (zapp) dmin = fminf(dmin, dmin8(zt, zd));
           } else {
-            const float2 part = norm_accumulate<false>(zt, zd, P.scale_log2, mt, st2, md, sd2);
+            float2 unused;
+            const float2 part =
+                norm_accumulate<false>(zt, zd, P.scale_log2, mt, st2, md, sd2, unused);
             if (rec_ok) {
               // a leaf: its bonus draw samples this row; record the warp's
               // chunk mass against the warp's largest reference

@@ -502,7 +502,8 @@ def run_ours(args):
             "launch": {k: plan[k] for k in ("kernel_name", "cluster_size", "block_threads",
                                             "smem_bytes", "slice_elems", "uses_tma",
                                             "vector_loads",
-                                            "active_clusters")},
+                                            "active_clusters")}
+                      | {"kernel_source_digest": kernel_source_digest()},
             "l2": f"rotating pool of {pool} input sets ({set_bytes / 1e9:.2f} GB each) "
                   f"between steps; each step's visited rows exceed L2 together",
         },

@@ -77,7 +77,7 @@ struct VerifyParams {
   uint64_t seed;
   float scale_log2;    // log2(e) / T
   float scale_log2_lo; // log2(e) / T - scale_log2, rounded (SpecInfer instance)
-  float exp2_tab[65][2];  // 2^(j / 64), j = -32 .. 32, as double-floats (SpecInfer instance)
+  float exp2_tab[64][2];  // 2^(j / 64), j = -32 .. 31, as double-floats (SpecInfer instance)
   int32_t B, N, V, D;
   int32_t slice;       // L, elements per CTA (multiple of 8)
   int32_t npad;        // padded node count of the tree arrays

@@ -63,7 +63,10 @@ constexpr int kErrFanout = 64;
 // is much smaller than R~.  Maps are applied two lanes per instruction.
 struct __align__(16) StreamHead {
   float2 map[kMaxMaps];  // {k_i, lambda_i} of map i
-  float mdsc[kMaxMaps];  // scale of the test denominator's D~ after map i
+  union {
+    float mdsc[kMaxMaps];     // scale of the test denominator's D~ after map i
+    float tab[kExp2Tab][2];   // SpecInfer instance: 2^(j/64) as double-floats
+  };
   int rej[kMaxMaps];     // rejected tokens (ResiSpec: their residual is 0)
   int16_t rejk[kMaxMaps];  // their child index in this visit
   float kzt[kMaxKids];   // raw target / draft logits of the children's tokens
@@ -83,15 +86,21 @@ constexpr int kStreamHeadBytes = 6144;
 constexpr int kMaxChunkRecs = 256;  // (chunk, warp) records per CTA
 static_assert(sizeof(StreamHead) <= kStreamHeadBytes, "stream head too large");
 
+// Eight logits per thread, chunk and row (one 16-byte vector of bf16, two
+// of fp32), and as many ring stages as fit 96 KB at 512 threads (6 for bf16,
+// 3 for fp32).  One fp32 vector per thread and 6 stages of 16 KB, more
+// copies in flight, measured 9 % slower on the fp32 workload: the pass
+// loop's fixed cost per chunk then falls on four elements instead of eight.
 template <int THREADS, bool BF16>
 struct StreamGeom {
   static constexpr int VEC = BF16 ? 8 : 4;            // elements per 16-byte vector
   static constexpr int VPT = BF16 ? 1 : 2;            // vectors per thread per chunk and row
-  static constexpr int NE = VPT * VEC;                // elements per thread per chunk and row (8)
+  static constexpr int NE = VPT * VEC;                // elements per thread per chunk and row
+  static constexpr int NP = NE / 2;                   // their pairs (packed arithmetic)
   static constexpr int CE = NE * THREADS;             // elements per chunk and row
   static constexpr uint32_t RB = (uint32_t)VPT * THREADS * 16u;  // bytes per chunk and row
   static constexpr uint32_t SB = 2u * RB;             // bytes per ring stage (target, draft)
-  static constexpr int S = BF16 ? 6 : 3;              // ring stages: 96 KB at 512 threads
+  static constexpr int S = (96 * 1024 * THREADS / 512) / SB;  // ring stages
   static constexpr uint32_t RING = S * SB;
 };
 
@@ -145,21 +154,65 @@ __device__ __forceinline__ uint4 stage_vec(const unsigned char* row, int h, int 
   return reinterpret_cast<const uint4*>(row)[h * threads + (int)threadIdx.x];
 }
 
-// This thread's NE values of a ring stage row as NE / 2 pairs, in the order
-// of its vectors (pair j holds elements 2j, 2j + 1 of the thread's chunk).
+// Element j (0 <= j < NE) of this thread's chunk in a ring stage row.
 template <int THREADS, bool BF16>
-__device__ __forceinline__ void load_pairs(const unsigned char* row, float2 (&z)[4]) {
-  if constexpr (BF16) {
-    const uint4 w = stage_vec(row, 0, THREADS);
-    const uint32_t v[4] = {w.x, w.y, w.z, w.w};
+__device__ __forceinline__ float stage_elem(const unsigned char* row, int j) {
+  constexpr int VEC = BF16 ? 8 : 4;
+  const unsigned char* v =
+      row + ((j / VEC) * THREADS + (int)threadIdx.x) * 16 + (j % VEC) * (BF16 ? 2 : 4);
+  if constexpr (BF16)
+    return __uint_as_float((uint32_t)*reinterpret_cast<const unsigned short*>(v) << 16);
+  else
+    return *reinterpret_cast<const float*>(v);
+}
+
+template <int THREADS, bool BF16>
+struct StageElem {
+  const unsigned char* row;
+  __device__ __forceinline__ float operator()(int j) const {
+    return stage_elem<THREADS, BF16>(row, j);
+  }
+};
+
+// This thread's vectors of a ring stage row, kept packed; element j for a
+// compile-time j.
+template <int THREADS, bool BF16>
+struct ChunkRegs {
+  static constexpr int VPT = StreamGeom<THREADS, BF16>::VPT;
+  uint4 w[VPT];
+  __device__ __forceinline__ explicit ChunkRegs(const unsigned char* row) {
 #pragma unroll
-    for (int i = 0; i < 4; ++i) z[i] = make_float2(bf16_lo(v[i]), bf16_hi(v[i]));
-  } else {
+    for (int h = 0; h < VPT; ++h) w[h] = stage_vec(row, h, THREADS);
+  }
+  __device__ __forceinline__ float operator()(int j) const {
+    constexpr int VEC = BF16 ? 8 : 4;
+    const uint4& v = w[j / VEC];
+    const int e = j % VEC;
+    if constexpr (BF16) {
+      const uint32_t x = (e >> 1) == 0 ? v.x : (e >> 1) == 1 ? v.y : (e >> 1) == 2 ? v.z : v.w;
+      return (e & 1) ? bf16_hi(x) : bf16_lo(x);
+    } else {
+      return __uint_as_float(e == 0 ? v.x : e == 1 ? v.y : e == 2 ? v.z : v.w);
+    }
+  }
+};
+
+// This thread's NE values of a ring stage row as NP = NE / 2 pairs, in the
+// order of its vectors (pair j holds elements 2j, 2j + 1 of the thread's chunk).
+template <int THREADS, bool BF16>
+__device__ __forceinline__ void load_pairs(const unsigned char* row,
+                                           float2 (&z)[StreamGeom<THREADS, BF16>::NP]) {
+  using G = StreamGeom<THREADS, BF16>;
 #pragma unroll
-    for (int h = 0; h < 2; ++h) {
-      const float4 f = *reinterpret_cast<const float4*>(&reinterpret_cast<const uint4*>(row)[h * THREADS + (int)threadIdx.x]);
-      z[2 * h] = make_float2(f.x, f.y);
-      z[2 * h + 1] = make_float2(f.z, f.w);
+  for (int h = 0; h < G::VPT; ++h) {
+    const uint4 w = stage_vec(row, h, THREADS);
+    if constexpr (BF16) {
+      const uint32_t v[4] = {w.x, w.y, w.z, w.w};
+#pragma unroll
+      for (int i = 0; i < 4; ++i) z[4 * h + i] = make_float2(bf16_lo(v[i]), bf16_hi(v[i]));
+    } else {
+      z[2 * h] = make_float2(__uint_as_float(w.x), __uint_as_float(w.y));
+      z[2 * h + 1] = make_float2(__uint_as_float(w.z), __uint_as_float(w.w));
     }
   }
 }
@@ -345,21 +398,37 @@ __device__ __forceinline__ float raw_logit(const void* base, size_t i, bool bf16
 // still makes the sum non-finite (detected by the caller).
 constexpr float kNoRef = -FLT_MAX;
 
-__device__ __forceinline__ float max8(const float2 (&z)[4]) {
-  return fmax3(fmax3(z[0].x, z[0].y, z[1].x), fmax3(z[1].y, z[2].x, z[2].y),
-               fmaxf(z[3].x, z[3].y));
+template <int NP>
+__device__ __forceinline__ float max_pairs(const float2 (&z)[NP]) {
+  if constexpr (NP == 4) {
+    return fmax3(fmax3(z[0].x, z[0].y, z[1].x), fmax3(z[1].y, z[2].x, z[2].y),
+                 fmaxf(z[3].x, z[3].y));
+  } else {
+    static_assert(NP == 2, "two or four pairs per chunk");
+    return fmax3(fmax3(z[0].x, z[0].y, z[1].x), z[1].y, -INFINITY);
+  }
 }
 
-// Smallest z_t - z_d of 8 pairs (the Z_applied bound min p / q is
+// Sum of NP pairs, pairwise.
+template <int NP>
+__device__ __forceinline__ float2 sum_pairs(const float2 (&a)[NP]) {
+  if constexpr (NP == 4) return __fadd2_rn(__fadd2_rn(a[0], a[1]), __fadd2_rn(a[2], a[3]));
+  else return __fadd2_rn(a[0], a[1]);
+}
+
+// Smallest z_t - z_d of a chunk's pairs (the Z_applied bound min p / q is
 // 2^((z_t - z_d) c) scaled by row constants, so it is taken on the logit
 // difference).  A token with q = 0 (z_d = -inf) gives +inf and a padding
 // slot (both -inf) NaN; both are ignored by the minimum.
-__device__ __forceinline__ float dmin8(const float2 (&zt)[4], const float2 (&zd)[4]) {
-  float2 d[4];
+template <int NP>
+__device__ __forceinline__ float dmin_pairs(const float2 (&zt)[NP], const float2 (&zd)[NP]) {
+  float m = INFINITY;
 #pragma unroll
-  for (int j = 0; j < 4; ++j) d[j] = __ffma2_rn(zd[j], dup2(-1.f), zt[j]);
-  return fminf(fminf(fminf(d[0].x, d[0].y), fminf(d[1].x, d[1].y)),
-               fminf(fminf(d[2].x, d[2].y), fminf(d[3].x, d[3].y)));
+  for (int j = 0; j < NP; ++j) {
+    const float2 d = __ffma2_rn(zd[j], dup2(-1.f), zt[j]);
+    m = fminf(m, fminf(d.x, d.y));
+  }
+  return m;
 }
 
 __device__ __forceinline__ void rebase2(float vmax, float c, float& m, float2& s) {
@@ -368,26 +437,28 @@ __device__ __forceinline__ void rebase2(float vmax, float c, float& m, float2& s
   m = mnew;
 }
 
-// Sum of 2^(z c - m) over 8 values (4 pairs), as a pair of partial sums.
-__device__ __forceinline__ float2 exp_sum8(const float2 (&z)[4], float2 c2, float2 nm2) {
-  float2 e[4];
+// Sum of 2^(z c - m) over a chunk's pairs, as a pair of partial sums.
+template <int NP>
+__device__ __forceinline__ float2 exp_sum(const float2 (&z)[NP], float2 c2, float2 nm2) {
+  float2 e[NP];
 #pragma unroll
-  for (int j = 0; j < 4; ++j) e[j] = ex2x2(__ffma2_rn(z[j], c2, nm2));
-  return __fadd2_rn(__fadd2_rn(e[0], e[1]), __fadd2_rn(e[2], e[3]));
+  for (int j = 0; j < NP; ++j) e[j] = ex2x2(__ffma2_rn(z[j], c2, nm2));
+  return sum_pairs<NP>(e);
 }
 
-// One chunk of a thread's values (8 per row) into its online (reference,
-// sum) pairs; the sums are kept as pairs of lanes.
-template <bool TWO>
-__device__ __forceinline__ float2 norm_accumulate(const float2 (&zt)[4], const float2 (&zd)[4],
+// One chunk of a thread's values into its online (reference, sum) pairs;
+// the sums are kept as pairs of lanes.  Returns the chunk's own target terms
+// (and, TWO, its draft terms in dpart).
+template <bool TWO, int NP>
+__device__ __forceinline__ float2 norm_accumulate(const float2 (&zt)[NP], const float2 (&zd)[NP],
                                                   float c, float& mt, float2& st, float& md,
                                                   float2& sd, float2& dpart) {
-  const float vt = max8(zt);
+  const float vt = max_pairs<NP>(zt);
   const bool rt = __fmaf_rn(vt, c, -mt) > 0.f;
   float vd = 0.f;
   bool rd = false;
   if constexpr (TWO) {
-    vd = max8(zd);
+    vd = max_pairs<NP>(zd);
     rd = __fmaf_rn(vd, c, -md) > 0.f;
   }
   if (rt || rd) {  // rare: a new reference for one of the rows
@@ -396,10 +467,10 @@ __device__ __forceinline__ float2 norm_accumulate(const float2 (&zt)[4], const f
       if (rd) rebase2(vd, c, md, sd);
   }
   const float2 c2 = dup2(c);
-  const float2 part = exp_sum8(zt, c2, dup2(-mt));  // this chunk's target terms
+  const float2 part = exp_sum<NP>(zt, c2, dup2(-mt));  // this chunk's target terms
   st = __fadd2_rn(st, part);
   if constexpr (TWO) {
-    dpart = exp_sum8(zd, c2, dup2(-md));  // and its draft terms
+    dpart = exp_sum<NP>(zd, c2, dup2(-md));  // and its draft terms
     sd = __fadd2_rn(sd, dpart);
   }
   return part;
@@ -409,9 +480,10 @@ __device__ __forceinline__ float2 norm_accumulate(const float2 (&zt)[4], const f
 // per chunk of the slice and warp, the warp's share of that distribution's
 // mass, so that the final draw finds the chunk holding its threshold
 // without another pass over the slice.  The mass of chunk k is
-//   kind 1 (a leaf's normaliser: the bonus draw samples p):
+//   kind 1 (a leaf's normaliser: the bonus draw samples p; or, when the
+//           kernel drafts, the draft row q):
 //     sum_w rec1[k, w] 2^(rec0[k, w] - a) b   (warp reference, warp sum;
-//                                              a = M_t, b = 1 / S_t)
+//                                              a = M, b = 1 / S)
 //   kind 2 (the last ResiSpec rejection: R~' = m + lambda t):
 //     sum_w (rec0[k, w] + a rec1[k, w]) b     (a = lambda, b = sigma)
 //   kind 3 (the last SpecInfer rejection): sum_w rec0[k, w] b   (b = 1 / T)
@@ -423,7 +495,8 @@ struct ChunkRec {
 };
 
 // Cluster-wide scalars of a visit after the normaliser.
-static_assert(sizeof(VerifyParams::exp2_tab) == sizeof(float) * 2 * kExp2Tab,
+static_assert(sizeof(VerifyParams::exp2_tab) == sizeof(float) * 2 * kExp2Tab &&
+                  sizeof(float) * 2 * kExp2Tab <= sizeof(float) * kMaxMaps,
               "exp2 table size");
 
 struct VisitScalars {
@@ -921,6 +994,8 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
   // node 0's parent can only be the root).
   auto setup = [&] {
     if (tid < 4) H.pubv[tid] = 0.f;
+    if constexpr (SPEC)  // the 2^(j/64) table, read at lane-dependent indices
+      for (int i = tid; i < 2 * kExp2Tab; i += THREADS) (&S2.tab[0][0])[i] = (&P.exp2_tab[0][0])[i];
     if (tid == 0) {
       mbar_init(smem_addr(&H.xbar[0]), 1);
       mbar_init(smem_addr(&H.xbar[1]), 1);
@@ -1102,12 +1177,12 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
         },
         [&](const unsigned char* rt, const unsigned char* rd, int k) -> bool {
           if (err) return true;  // invalid tree (uniform over the cluster)
-          float2 zt[4], zd[4];
+          float2 zt[G::NP], zd[G::NP];
           load_pairs<THREADS, BF16>(rt, zt);
           if (need_draft) {
             load_pairs<THREADS, BF16>(rd, zd);
             float2 dpart;
-            norm_accumulate<true>(zt, zd, P.scale_log2, mt, st2, md, sd2, dpart);
+            norm_accumulate<true, G::NP>(zt, zd, P.scale_log2, mt, st2, md, sd2, dpart);
             if (rec_draft) {
               const float mw = redux_max(md);
               const float sw =
@@ -1117,11 +1192,11 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
                 S2.crec[1][k * NW + warp] = sw;
               }
             }
-            if (zapp) dmin = fminf(dmin, dmin8(zt, zd));
+            if (zapp) dmin = fminf(dmin, dmin_pairs<G::NP>(zt, zd));
           } else {
             float2 unused;
             const float2 part =
-                norm_accumulate<false>(zt, zd, P.scale_log2, mt, st2, md, sd2, unused);
+                norm_accumulate<false, G::NP>(zt, zd, P.scale_log2, mt, st2, md, sd2, unused);
             if (rec_ok) {
               // a leaf: its bonus draw samples this row; record the warp's
               // chunk mass against the warp's largest reference
@@ -1186,7 +1261,7 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
     K.sig = K.invSt;
     if constexpr (SPEC) {
       K.sc = SpecConst{P.scale_log2, P.scale_log2_lo, K.Mt, K.Md, df(0.f)};
-      K.tab = P.exp2_tab;
+      K.tab = S2.tab;
     }
     // SpecInfer: the double-float normalisers (taken at the node's first
     // rejection) and the current residual mass T
@@ -1274,17 +1349,10 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
           DF acc[2] = {df(0.f), df(0.f)};
           stream_pass<THREADS, BF16, 2>(ring, src, primed, [&](const unsigned char* rt,
                                                             const unsigned char* rd, int) -> bool {
-#pragma unroll
-            for (int h = 0; h < G::VPT; ++h) {
-              float zt[VEC], zd[VEC];
-              unpack_vec<BF16>(stage_vec(rt, h, THREADS), zt);
-              unpack_vec<BF16>(stage_vec(rd, h, THREADS), zd);
-#pragma unroll
-              for (int j = 0; j < VEC; ++j) {
-                acc[0] = df_add(acc[0], unnorm_df(zt[j], K.sc.c_hi, K.sc.c_lo, K.Mt, K.tab));
-                acc[1] = df_add(acc[1], unnorm_df(zd[j], K.sc.c_hi, K.sc.c_lo, K.Md, K.tab));
-              }
-            }
+            unnorm_sum<G::NE>(ChunkRegs<THREADS, BF16>(rt), StageElem<THREADS, BF16>{rt}, K.sc.c_hi,
+                              K.sc.c_lo, K.Mt, K.tab, acc[0]);
+            unnorm_sum<G::NE>(ChunkRegs<THREADS, BF16>(rd), StageElem<THREADS, BF16>{rd}, K.sc.c_hi,
+                              K.sc.c_lo, K.Md, K.tab, acc[1]);
             return false;
           });
           if (!src.held) stream_prime<THREADS, BF16>(ring, src, primed);
@@ -1302,19 +1370,9 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
         const bool rec_last = rec_ok && next_sib[cn] < 0;
         stream_pass<THREADS, BF16, 2>(ring, src, primed, [&](const unsigned char* rt,
                                                           const unsigned char* rd, int k) -> bool {
-          float cr = 0.f;
-#pragma unroll
-          for (int h = 0; h < G::VPT; ++h) {
-            float zt[VEC], zd[VEC];
-            unpack_vec<BF16>(stage_vec(rt, h, THREADS), zt);
-            unpack_vec<BF16>(stage_vec(rd, h, THREADS), zd);
-#pragma unroll
-            for (int j = 0; j < VEC; ++j) {
-              const DF r = spec_residual(zt[j], zd[j], K.sc, K.tab);
-              acc[0] = df_add(acc[0], r);
-              cr = __fadd_rn(cr, r.hi);
-            }
-          }
+          const float cr = residual_sum<G::NE>(
+              ChunkRegs<THREADS, BF16>(rt), ChunkRegs<THREADS, BF16>(rd),
+              StageElem<THREADS, BF16>{rt}, StageElem<THREADS, BF16>{rd}, K.sc, K.tab, acc[0]);
           if (rec_last) {
             const float wr = group_sum<5>(cr);
             if (lane == 0) S2.crec[0][k * NW + warp] = wr;
@@ -1372,19 +1430,20 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
         const float2 c2 = dup2(K.c), nMt = dup2(-K.Mt), nMd = dup2(-K.Md), kq2 = dup2(kq);
         stream_pass<THREADS, BF16, 2>(ring, src, primed, [&](const unsigned char* rt,
                                                           const unsigned char* rd, int k) -> bool {
-          float2 Rv[4], q[4];
+          constexpr int NP = G::NP;
+          float2 Rv[NP], q[NP];
           load_pairs<THREADS, BF16>(rt, Rv);  // -inf past the slice: 0
           load_pairs<THREADS, BF16>(rd, q);
 #pragma unroll
-          for (int j = 0; j < 4; ++j) {
+          for (int j = 0; j < NP; ++j) {
             Rv[j] = ex2x2(__ffma2_rn(Rv[j], c2, nMt));
             q[j] = ex2x2(__ffma2_rn(q[j], c2, nMd));
           }
-          float2 t[4];
-          apply_chain_pairs<4, KIND>(S2, nm, Rv, q);
-          float2 m[4];
+          float2 t[NP];
+          apply_chain_pairs<NP, KIND>(S2, nm, Rv, q);
+          float2 m[NP];
 #pragma unroll
-          for (int j = 0; j < 4; ++j) {
+          for (int j = 0; j < NP; ++j) {
             m[j] = min_part2(kq2, q[j], Rv[j]);
             if constexpr (LEVEL) {
               s3p.x += m[j].x < Rv[j].x ? q[j].x : 0.f;
@@ -1394,8 +1453,8 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
               t[j] = __ffma2_rn(m[j], dup2(-1.f), Rv[j]);
             }
           }
-          const float2 cm = __fadd2_rn(__fadd2_rn(m[0], m[1]), __fadd2_rn(m[2], m[3]));
-          const float2 ct = __fadd2_rn(__fadd2_rn(t[0], t[1]), __fadd2_rn(t[2], t[3]));
+          const float2 cm = sum_pairs<NP>(m);
+          const float2 ct = sum_pairs<NP>(t);
           s1p = __fadd2_rn(s1p, cm);
           s2p = __fadd2_rn(s2p, ct);
           if constexpr (REC) {

@@ -300,13 +300,15 @@ __device__ __forceinline__ unsigned char* held_stage(unsigned char* ring, const 
 // above), calling body(target_stage_row, draft_stage_row, k) with all
 // threads (the draft pointer is meaningful only for passes over both rows);
 // body returns true (uniformly) to end the pass.  pre() runs once, after the
-// first copies are issued.  When `primed` is set the first chunks were
-// issued earlier by stream_prime over the same rows and are not issued again
-// (the flag is cleared).  On return every copy of the pass has landed.
+// first copies are issued.  On return every copy of the pass has landed.
+// A pass issues its first copies when it starts: issuing them earlier, during
+// the cluster exchange before it, measured slower (113 against 108 us on the
+// fp32 binary-tree workload), since after an accepted test the copies were
+// for rows no pass would read, and the next visit had to wait for them.
 // ROWS: 2 or 1 when the caller knows s.rows, 0 to read it.
 template <int THREADS, bool BF16, int ROWS = 0, class Pre, class Body>
-__device__ __forceinline__ void stream_pass_pre(unsigned char* ring, const Src& s, bool& primed,
-                                                Pre&& pre, Body&& body) {
+__device__ __forceinline__ void stream_pass_pre(unsigned char* ring, const Src& s, Pre&& pre,
+                                                Body&& body) {
   using G = StreamGeom<THREADS, BF16>;
   const int NK = (s.nloc + G::CE - 1) / G::CE;
   if (s.held) {  // the rows stayed in the ring since the visit's first pass
@@ -320,13 +322,10 @@ __device__ __forceinline__ void stream_pass_pre(unsigned char* ring, const Src& 
   const bool two = ROWS == 2 || (ROWS == 0 && s.rows == 2);
   const int S = ring_depth<THREADS, BF16>(two);
   const uint32_t stride = ring_stride<THREADS, BF16>(two);
-  if (!primed) {
-    for (int k = 0; k < S - 1; ++k) {
-      if (k < NK) copy_chunk<THREADS, BF16>(s, k, ring + k * stride, two);
-      else cp_async_commit();
-    }
+  for (int k = 0; k < S - 1; ++k) {
+    if (k < NK) copy_chunk<THREADS, BF16>(s, k, ring + k * stride, two);
+    else cp_async_commit();
   }
-  primed = false;
   pre();
   int slot = 0;
   for (int k = 0; k < NK; ++k) {
@@ -346,35 +345,8 @@ __device__ __forceinline__ void stream_pass_pre(unsigned char* ring, const Src& 
 }
 
 template <int THREADS, bool BF16, int ROWS = 0, class Body>
-__device__ __forceinline__ void stream_pass(unsigned char* ring, const Src& s, bool& primed,
-                                            Body&& body) {
-  stream_pass_pre<THREADS, BF16, ROWS>(ring, s, primed, [] {}, body);
-}
-
-// Issues the copies a pass over s starts with (its first depth - 1 chunks,
-// into the ring stages it reads them from), so that they travel while the
-// CTA waits in a cluster exchange.  Every thread copies only into its own
-// slots, which its previous pass has finished reading, so no barrier is
-// needed.  The next pass over the same rows takes them (primed); any other
-// use of the ring first calls stream_drain.
-template <int THREADS, bool BF16>
-__device__ __forceinline__ void stream_prime(unsigned char* ring, const Src& s, bool& primed) {
-  using G = StreamGeom<THREADS, BF16>;
-  const int NK = (s.nloc + G::CE - 1) / G::CE;
-  const bool two = s.rows == 2;
-  const int S = ring_depth<THREADS, BF16>(two);
-  const uint32_t stride = ring_stride<THREADS, BF16>(two);
-  for (int k = 0; k < S - 1; ++k) {
-    if (k < NK) copy_chunk<THREADS, BF16>(s, k, ring + k * stride, two);
-    else cp_async_commit();
-  }
-  primed = true;
-}
-
-// Waits for primed copies that no pass will take.
-__device__ __forceinline__ void stream_drain(bool& primed) {
-  if (primed) cp_async_wait<0>();
-  primed = false;
+__device__ __forceinline__ void stream_pass(unsigned char* ring, const Src& s, Body&& body) {
+  stream_pass_pre<THREADS, BF16, ROWS>(ring, s, [] {}, body);
 }
 
 __device__ __forceinline__ float raw_logit(const void* base, size_t i, bool bf16) {
@@ -662,7 +634,7 @@ constexpr int kMaxSearchChunks = 128;
 template <int THREADS, bool BF16, bool SPEC>
 __device__ int stream_search(Head& H, const StreamHead& S2, unsigned long long* ck,
                              unsigned char* ring, const Src& s, const VisitScalars& K, int chain,
-                             int lo, unsigned long long tau, bool& primed, const ChunkRec& cr) {
+                             int lo, unsigned long long tau, const ChunkRec& cr) {
   using G = StreamGeom<THREADS, BF16>;
   constexpr int VEC = G::VEC;
   constexpr int NW = THREADS / 32;
@@ -686,7 +658,7 @@ __device__ int stream_search(Head& H, const StreamHead& S2, unsigned long long* 
       }
       ck[k] = to_fix(m);
     }
-  } else stream_pass<THREADS, BF16>(ring, s, primed, [&](const unsigned char* rt,
+  } else stream_pass<THREADS, BF16>(ring, s, [&](const unsigned char* rt,
                                                          const unsigned char* rd, int k) -> bool {
     float2 acc2 = make_float2(0.f, 0.f);
 #pragma unroll
@@ -750,7 +722,6 @@ __device__ int stream_search(Head& H, const StreamHead& S2, unsigned long long* 
   if (s.held) {
     stg = held_stage<THREADS, BF16>(ring, s, ks);
   } else {
-    stream_drain(primed);
     copy_chunk<THREADS, BF16>(s, ks, ring, s.rows == 2);
     cp_async_wait<0>();
   }
@@ -822,7 +793,7 @@ __device__ bool stream_sample(Head& H, StreamHead& S2, unsigned char* ring, cons
                               const Src& s_in, const VisitScalars& K, int chain, int mass_kind,
                               const Pending& Pm, float u, int b, int depth, int lo,
                               uint32_t rank, uint32_t C, int& xp, uint32_t& xph, bool& timeout,
-                              bool& primed, const ChunkRec& cr) {
+                              const ChunkRec& cr) {
   using G = StreamGeom<THREADS, BF16>;
   constexpr int VEC = G::VEC;
   constexpr int NW = THREADS / 32;
@@ -834,7 +805,7 @@ __device__ bool stream_sample(Head& H, StreamHead& S2, unsigned char* ring, cons
     // every CTA: values of its slice (written out when asked) and their sum
     float* dist = P.out_dist ? P.out_dist + (size_t)b * P.V + lo : nullptr;
     float sum = 0.f;
-    stream_pass<THREADS, BF16>(ring, s, primed, [&](const unsigned char* rt,
+    stream_pass<THREADS, BF16>(ring, s, [&](const unsigned char* rt,
                                                     const unsigned char* rd, int k) -> bool {
 #pragma unroll
       for (int h = 0; h < G::VPT; ++h) {
@@ -886,8 +857,7 @@ __device__ bool stream_sample(Head& H, StreamHead& S2, unsigned char* ring, cons
   // to zero mass yields its first token.
   // chunk totals of the search: the children's logit slots, unused by the draw
   const int pick = stream_search<THREADS, BF16, SPEC>(
-      H, S2, reinterpret_cast<unsigned long long*>(S2.kzt), ring, s, K, chain, lo, tau, primed,
-      cr);
+      H, S2, reinterpret_cast<unsigned long long*>(S2.kzt), ring, s, K, chain, lo, tau, cr);
   if (threadIdx.x == 0) P.out_tokens[(size_t)b * (P.D + 1) + depth] = lo + max(pick, 0);
   return true;
 }
@@ -978,7 +948,6 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
   int node = -1, row = 0;
   uint32_t xph = 0;
   int xp = 0;
-  bool primed = false;  // the ring holds the first copies of the next pass (stream_prime)
   const int lane = tid & 31, warp = tid >> 5;
   // chunk records for the final draw (ChunkRec; not in the instance with the
   // optional paths)
@@ -1073,12 +1042,11 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
     // before the node's accept tests)
     static_assert(sizeof(StreamHead::map) >= kMaxSearchChunks * sizeof(unsigned long long),
                   "search chunk totals fit the map slots");
-    stream_drain(primed);
     for (int i = 0, cn = c1d; i < nk; ++i, cn = next_sib[cn]) {
       if (owner[i] != (int)rank) continue;
       const int pick = stream_search<THREADS, BF16, SPEC>(
           H, S2, reinterpret_cast<unsigned long long*>(S2.map), ring, sq, Kq, chain, lo, tau[i],
-          primed, ChunkRec{rec_draft ? 1 : 0, K.Md, K.invSd});
+          ChunkRec{rec_draft ? 1 : 0, K.Md, K.invSd});
       if (tid == 0) P.draft_out[(size_t)b * N + cn] = lo + max(pick, 0);
     }
     cluster_sync();  // every drawn token written (release / acquire at cluster scope)
@@ -1128,7 +1096,6 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
     // needed to publish it; the barrier at the end of the previous visit
     // orders these writes after every read of the old values.
     S2.nmaps = 0;
-    stream_drain(primed);  // copies primed for the previous visit's rows
 
     mark(kPhaseNorm);
     // ---- tempered normaliser (S2): online (reference, sum) per row; while
@@ -1151,7 +1118,7 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
     };
     bool have_kid = false;
     float kz_t = 0.f, kz_d = 0.f;
-    stream_pass_pre<THREADS, BF16>(ring, src, primed,
+    stream_pass_pre<THREADS, BF16>(ring, src,
         [&] {
           if (first) {
             setup();
@@ -1214,11 +1181,8 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
     if (err) break;
     // A slice of at most S chunks stays in the ring (chunk k in stage k; not
     // in the instance with the optional paths, whose registers it exceeds):
-    // every later pass of the visit reads it from shared memory.  Otherwise
-    // the next pass over these rows (the first rejection's, or the draw's)
-    // starts its copies now, while the normaliser is exchanged.
+    // every later pass of the visit reads it from shared memory.
     src.held = !VAR && (nloc + G::CE - 1) / G::CE <= (src.rows == 2 ? G::S : 2 * G::S);
-    if (!src.held) stream_prime<THREADS, BF16>(ring, src, primed);
     const float st = __fadd_rn(st2.x, st2.y), sd = __fadd_rn(sd2.x, sd2.y);
     if (have_kid) {
       S2.kzt[tid] = kz_t;
@@ -1283,8 +1247,7 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
       if (rec_ok) crec = ChunkRec{1, K.Mt, K.invSt};
       mark(kPhaseDraw);
       if (!stream_sample<THREADS, BF16, SPEC>(H, S2, ring, P, src, K, chain, mass_kind, Pm,
-                                              S2.ufin, b, depth, lo, rank, C, xp, xph, to, primed,
-                                              crec))
+                                              S2.ufin, b, depth, lo, rank, C, xp, xph, to, crec))
         err |= kErrEmpty;
       if (to) err |= kErrTimeout;
       break;
@@ -1347,7 +1310,7 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
           const DF Kprev = K.sc.K;
         if (!spec_norm) {
           DF acc[2] = {df(0.f), df(0.f)};
-          stream_pass<THREADS, BF16, 2>(ring, src, primed, [&](const unsigned char* rt,
+          stream_pass<THREADS, BF16, 2>(ring, src, [&](const unsigned char* rt,
                                                             const unsigned char* rd, int) -> bool {
             unnorm_sum<G::NE>(ChunkRegs<THREADS, BF16>(rt), StageElem<THREADS, BF16>{rt}, K.sc.c_hi,
                               K.sc.c_lo, K.Mt, K.tab, acc[0]);
@@ -1355,7 +1318,6 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
                               K.sc.c_lo, K.Md, K.tab, acc[1]);
             return false;
           });
-          if (!src.held) stream_prime<THREADS, BF16>(ring, src, primed);
           DF tot[2];
           if (!df_exchange<NW, 2>(H, acc, tot, xp, xph, rank, C)) { err |= kErrTimeout; break; }
           spec_norm = true;
@@ -1368,7 +1330,7 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
         // the last child's rejection defines the final distribution: its
         // pass records it (ChunkRec kind 3)
         const bool rec_last = rec_ok && next_sib[cn] < 0;
-        stream_pass<THREADS, BF16, 2>(ring, src, primed, [&](const unsigned char* rt,
+        stream_pass<THREADS, BF16, 2>(ring, src, [&](const unsigned char* rt,
                                                           const unsigned char* rd, int k) -> bool {
           const float cr = residual_sum<G::NE>(
               ChunkRegs<THREADS, BF16>(rt), ChunkRegs<THREADS, BF16>(rd),
@@ -1379,7 +1341,6 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
           }
           return false;
         });
-        if (!src.held) stream_prime<THREADS, BF16>(ring, src, primed);
         DF tot[1];
         if (!df_exchange<NW, 1>(H, acc, tot, xp, xph, rank, C)) { err |= kErrTimeout; break; }
         mark(kPhaseTest);
@@ -1428,7 +1389,7 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
         constexpr bool LEVEL = decltype(level_c)::value;
         constexpr bool REC = decltype(rec_c)::value;
         const float2 c2 = dup2(K.c), nMt = dup2(-K.Mt), nMd = dup2(-K.Md), kq2 = dup2(kq);
-        stream_pass<THREADS, BF16, 2>(ring, src, primed, [&](const unsigned char* rt,
+        stream_pass<THREADS, BF16, 2>(ring, src, [&](const unsigned char* rt,
                                                           const unsigned char* rd, int k) -> bool {
           constexpr int NP = G::NP;
           float2 Rv[NP], q[NP];
@@ -1503,8 +1464,6 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
           rej_pass(std::integral_constant<int, kChainResi>{}, std::false_type{},
                    std::false_type{});
         }
-        // the next pass over these rows starts its copies during the exchange
-        if (!src.held) stream_prime<THREADS, BF16>(ring, src, primed);
         s1 = __fadd_rn(s1p.x, s1p.y);
         s2 = __fadd_rn(s2p.x, s2p.y);
         s3 = __fadd_rn(s3p.x, s3p.y);
@@ -1621,8 +1580,7 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
       bool to = false;
       mark(kPhaseDraw);
       if (!stream_sample<THREADS, BF16, SPEC>(H, S2, ring, P, src, K, chain, mass_kind, Pm,
-                                              S2.ufin, b, depth, lo, rank, C, xp, xph, to, primed,
-                                              crec))
+                                              S2.ufin, b, depth, lo, rank, C, xp, xph, to, crec))
         err |= kErrEmpty;
       if (to) err |= kErrTimeout;
       break;
@@ -1638,7 +1596,6 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
     __syncthreads();  // every read of this visit's S2 state precedes the next visit's writes
   }
 
-  stream_drain(primed);
   mark(kPhaseSetup);
   if (prof && rank == 0 && tid == 0)
     for (int k = 0; k < kPhases; ++k) P.out_phase[(size_t)b * kPhases + k] = (int64_t)S2.phc[k];

@@ -7,6 +7,9 @@
 #include <stdio.h>
 #include <string.h>
 
+#include <algorithm>
+#include <climits>
+#include <cmath>
 #include <map>
 #include <mutex>
 #include <tuple>
@@ -219,48 +222,79 @@ int plan_resident(const resispec_dims& d, int cs, int dev, int sms, Plan* p) {
   return RESISPEC_OK;
 }
 
-// Streaming kernel: cluster size.  A sequence's passes shrink as 1 / C,
-// and the batch runs in ceil(B / n) waves of n resident clusters; the
-// largest C whose waves stay within a bound wins (per-sequence chains differ
-// in length, so the longest chain, run at C CTAs, sets the time).  The bound
-// (measured on GB300 over four tree shapes): 2 waves for clusters of 16; for
-// trees deeper than 2 levels (long accept/reject chains) a single wave,
-// since a second wave of long chains costs more than halving C; for shallow
-// trees up to 4 waves.  Without a device, 2 CTAs of 512 threads per SM on
-// 152 SMs are assumed and a cluster of 16 is taken to fit 14 times (how many
-// clusters of 16 CTAs GB300 places at once), smaller ones in proportion.
-int plan_stream(const resispec_dims& d, int cs, int dev, int sms, Plan* p) {
+// Streaming kernel: block size and cluster size.  A sequence's passes
+// shrink as 1 / C, and the batch runs in ceil(B / n) waves of n resident
+// clusters (per-sequence chains differ in length, so the longest chain, run
+// at C CTAs, sets the time).  Measured on GB300 (eleven workloads, both
+// block sizes):
+//  - 256-thread CTAs (three per SM, half the ring each) beat 512-thread ones
+//    on trees with about two children per node (N^(1/D) <= 2.5: binary
+//    depth-5 trees 102.7 against 107.9 us at B = 64, single position k = 2
+//    at B = 128 85.8 against 104.4 us), where a sequence spends its time in
+//    normaliser passes rather than in rejection passes; wider trees and
+//    batches that fit 16-CTA clusters of 512 threads keep 512.
+//  - Trees deeper than 2 levels take the largest C that runs the batch in
+//    one wave; when that leaves more than 128 elements per thread and row in
+//    a CTA's slice, the largest C within two waves (tree488 at B = 128:
+//    clusters of 4 in two waves 256.6 us, of 2 in one wave 288.8 us).
+//  - Shallow trees at 512 threads (up to 2 levels: few visits, many
+//    rejection passes) accept up to 4 waves, clusters of 16 up to 2.
+// Without a device, 2 CTAs of 512 threads or 3 of 256 per SM on 152 SMs
+// are assumed and a cluster of 16 is taken to fit 14 times per 304 CTA
+// slots (how many clusters of 16 CTAs GB300 places at once), smaller ones in
+// proportion.
+int plan_stream(const resispec_dims& d, int cs, bool auto_threads, int dev, int sms, Plan* p) {
   const bool bf16 = d.dtype == RESISPEC_BF16;
-  p->smem = stream_smem_for(p->threads, bf16, p->npad);
-  if (p->smem > kMaxSmem) return RESISPEC_E_SHAPE;
   const int B = std::max(d.batch, 1);
-  auto active_for = [&](int C) {
+  auto active_for = [&](int T, int C) {
+    const int smem = stream_smem_for(T, bf16, p->npad);
     if (dev >= 0)
-      return active_clusters(dev, RESISPEC_KERNEL_STREAM, p->var, p->spec, p->threads, bf16, C,
-                             p->smem);
-    const int slots = (sms > 0 ? sms : 152) * (p->threads >= 512 ? 2 : 4);
+      return active_clusters(dev, RESISPEC_KERNEL_STREAM, p->var, p->spec, T, bf16, C, smem);
+    const int slots = (sms > 0 ? sms : 152) * (T >= 512 ? 2 : 3);
     return C == 16 ? 14 * slots / 304 : slots / C;
   };
+  if (auto_threads) {
+    const double g = d.max_depth > 0
+                         ? std::pow((double)std::max(d.num_nodes, 1), 1.0 / d.max_depth)
+                         : 1e30;
+    p->threads = (g <= 2.5 && B > active_for(512, 16)) ? 256 : 512;
+  }
+  const int T = p->threads;
+  p->smem = stream_smem_for(T, bf16, p->npad);
+  if (p->smem > kMaxSmem) return RESISPEC_E_SHAPE;
   if (cs) {
     p->C = cs;
   } else {
+    auto waves = [&](int C) {
+      const int n = active_for(T, C);
+      return n > 0 ? (B + n - 1) / n : INT_MAX;
+    };
     int best = 0;
-    for (int C : {16, 8, 4, 2, 1}) {
-      const int n = active_for(C);
-      if (n <= 0) continue;
-      const int waves = (B + n - 1) / n;
-      const int bound = C == 16 ? 2 : (d.max_depth <= 2 ? 4 : 1);
-      if (waves <= bound || C == 1) {
-        best = C;
-        break;
+    if (T == 512 && d.max_depth <= 2) {
+      for (int C : {16, 8, 4, 2, 1}) {
+        if (waves(C) <= (C == 16 ? 2 : 4) || C == 1) {
+          best = C;
+          break;
+        }
       }
+    } else {
+      static const int kCands[] = {16, 12, 8, 6, 4, 3, 2, 1};
+      for (int C : kCands)
+        if (waves(C) <= 1 || C == 1) {
+          best = C;
+          break;
+        }
+      if (slice_for(d.vocab, best) > 128 * T)
+        for (int C : kCands)
+          if (C > best && waves(C) <= 2) {
+            best = C;
+            break;
+          }
     }
-    if (best == 0) return RESISPEC_E_UNSUPPORTED;
     p->C = best;
   }
   p->L = slice_for(d.vocab, p->C);
-  p->active = active_for(p->C);
-  if (dev < 0) p->active = 0;
+  p->active = dev >= 0 ? active_for(T, p->C) : 0;
   return RESISPEC_OK;
 }
 
@@ -301,7 +335,7 @@ int make_plan(const resispec_dims& d, const resispec_opts& o, int dev, int sms,
     st = plan_resident(d, cs, dev, sms, p);
   } else {
     p->kernel = RESISPEC_KERNEL_STREAM;
-    st = plan_stream(d, cs, dev, sms, p);
+    st = plan_stream(d, cs, o.block_threads == 0, dev, sms, p);
   }
   if (st) return st;
   const int64_t es = d.dtype == RESISPEC_BF16 ? 2 : 4;

@@ -75,17 +75,28 @@ def test_synchronous_argument_errors(lib):
 
 
 def test_plan_without_device(lib):
-    # the bench workload (B = 64, V = 151936 fp32) cannot sit on chip at once:
-    # the automatic choice streams it, in clusters of 4 CTAs (one wave: the
-    # tree is 5 levels deep)
+    # the bench workload (B = 64, V = 151936 fp32, a binary tree) cannot sit
+    # on chip at once: the automatic choice streams it, with 256-thread CTAs
+    # (about two children per node) in clusters of 6 (one wave of 76 on 456
+    # CTA slots: the tree is 5 levels deep)
     p = rs.plan(64, 62, 151936, 5, "f32")
-    assert p["kernel_name"] == "stream" and p["cluster_size"] == 4
-    assert p["smem_bytes"] <= 228 * 1024 // 2 - 1024   # two CTAs per SM
-    assert p["slice_elems"] % 8 == 0 and p["slice_elems"] * 4 >= 151936
+    assert p["kernel_name"] == "stream" and p["cluster_size"] == 6
+    assert p["block_threads"] == 256
+    assert p["smem_bytes"] <= 228 * 1024 // 3 - 1024   # three CTAs per SM
+    assert p["slice_elems"] % 8 == 0 and p["slice_elems"] * 6 >= 151936
+    # 512-thread CTAs for wider trees and for batches that fit clusters of 16
+    assert rs.plan(1, 62, 151936, 5, "f32")["block_threads"] == 512
+    assert rs.plan(128, 16, 256000, 1, "bf16")["block_threads"] == 512
     # shallow trees accept more waves: 128 single-position sequences in
-    # clusters of 8; deep trees of 32 sequences in clusters of 8 (one wave)
+    # clusters of 8; deep trees of 32 sequences in clusters of 8 (one wave);
+    # of 128 sequences, whose one-wave slices would be too long, in clusters
+    # of 4 (two waves)
     assert rs.plan(128, 16, 256000, 1, "bf16", kernel="stream")["cluster_size"] == 8
     assert rs.plan(32, 488, 256000, 6, "bf16", kernel="stream")["cluster_size"] == 8
+    assert rs.plan(128, 488, 256000, 6, "bf16", kernel="stream")["cluster_size"] == 4
+    # an explicit block size is kept
+    p = rs.plan(64, 62, 151936, 5, "f32", block_threads=512)
+    assert p["block_threads"] == 512 and p["cluster_size"] == 4
     # the streaming kernel moves 16-byte vectors with per-thread asynchronous
     # copies, not bulk (TMA) copies; the resident kernel uses bulk copies
     assert p["uses_tma"] == 0 and p["vector_loads"] == 1

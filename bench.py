@@ -84,13 +84,20 @@ def measured_peak():
         return FALLBACK_HBM_GBS, "fallback"
 
 
-def kernel_source_digest():
+def kernel_source_digest(csrc=None):
+    """Digest of the kernel sources (`csrc/`) with their comments removed:
+    the committed ncu counters are keyed to the code they measured, and a
+    change of comments alone does not invalidate them."""
     h = hashlib.sha256()
-    csrc = os.path.join(ROOT, "paper_2608_24411_gb300", "csrc")
+    csrc = csrc or os.path.join(ROOT, "paper_2608_24411_gb300", "csrc")
     for name in sorted(os.listdir(csrc)):
-        with open(os.path.join(csrc, name), "rb") as f:
-            h.update(name.encode())
-            h.update(f.read())
+        with open(os.path.join(csrc, name), encoding="utf-8") as f:
+            code = f.read()
+        code = re.sub(r"/\*.*?\*/", " ", code, flags=re.S)
+        code = re.sub(r"//[^\n]*", "", code)
+        code = "\n".join(line.rstrip() for line in code.splitlines() if line.strip())
+        h.update(name.encode())
+        h.update(code.encode())
     return h.hexdigest()[:16]
 
 

@@ -10,7 +10,7 @@
  *   draft logits into tempered distributions p, q (softmax(z / T)); test the
  *   node's children in ascending node order with u < R(x) / q(x), R starting
  *   at p; after each rejection reshape R (ResiSpec: GetProxy of Algorithm 1;
- *   SpecInfer: Eq. recur); on acceptance emit the child's token and descend
+ *   SpecInfer: Eq. 2); on acceptance emit the child's token and descend
  *   into it; when every child is rejected emit x ~ R; when an accepted node
  *   has no children emit a bonus token x ~ p of that node.
  *
@@ -56,7 +56,7 @@ typedef enum { RESISPEC_F32 = 0, RESISPEC_BF16 = 1 } resispec_dtype;
 
 /* RESISPEC: Algorithm 1 with GetProxy (budget Z = q(x0) - R(x0), deficit
  *   filled in proportion to the remaining capacity R - r off x0).
- * SPECINFER: the residual recurrence R <- (R - q)_+ / sum (Eq. recur). */
+ * SPECINFER: the residual recurrence R <- (R - q)_+ / sum (Eq. 2, Sec. 3). */
 typedef enum { RESISPEC_MODE_RESISPEC = 0, RESISPEC_MODE_SPECINFER = 1 } resispec_mode;
 
 /* Bits of the optional device status word (atomically OR-ed per sequence).

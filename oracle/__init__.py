@@ -8,7 +8,7 @@ fails loudly when its CUDA library is missing.
 Two independent pieces live here:
 
 * ``resispec_oracle.c`` (wrapped below): the literal walk of Algorithm 1 /
-  GetProxy / Eq. (recur) over a draft tree, fp64, threaded over sequences.
+  GetProxy / Eq. 2 (Sec. 3) over a draft tree, fp64, threaded over sequences.
 * ``enumerator.py``: an exact enumerator of the output distribution of the
   same rules for tiny vocabularies (numpy, no sampling), used to pin the C
   oracle.

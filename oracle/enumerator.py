@@ -11,7 +11,7 @@ candidates, so this is for tiny vocabularies only.
 The shaping rules are written here a second time, independently of the C
 oracle and vectorised over the vocabulary:
 
-* SPECINFER: R' = (R - q)_+ / sum (R - q)_+                    (Eq. recur)
+* SPECINFER: R' = (R - q)_+ / sum (R - q)_+                    (Eq. 2, Sec. 3)
 * RESISPEC:  GetProxy of Algorithm 1 with budget Z = q(x0) - R(x0),
   projection r = min(Z q, R) with r(x0) = 0, the deficit filled in
   proportion to the remaining capacity R - r off x0, then

@@ -20,7 +20,7 @@
  *   - on rejection, mode RESISPEC: K = GetProxy(R, Q, x0) and
  *     R <- norm(max(R - K, 0))  (Algorithm 1, function GetProxy; budget from
  *     Sec. 5.3, Eq. for s(x0));
- *     mode SPECINFER: R <- norm(max(R - q, 0))  (Eq. recur, Sec. 3);
+ *     mode SPECINFER: R <- norm(max(R - q, 0))  (Eq. 2, Sec. 3);
  *   - the final sample x ~ R by inverse CDF over ascending token ids
  *     (Algorithm 1, last step), or, when an accepted node has no children,
  *     the bonus token from that node's own target distribution (speculative
@@ -326,7 +326,7 @@ int oracle_reject_z(int mode, int z_rule, int fill, double* R, const double* q, 
                     double* K, double* r, double* tmp, double* inv_err, double* norm_out);
 
 /* One rejection of token x0 applied to the residual R (length V).
- * mode SPECINFER: R <- norm(max(R - q, 0))              (Eq. recur)
+ * mode SPECINFER: R <- norm(max(R - q, 0))              (Eq. 2, Sec. 3)
  * mode RESISPEC:  K = GetProxy(R, q, x0); R <- norm(max(R - K, 0)) (Alg. 1)
  * Returns 1 if R changed, 0 on a degenerate rejection (R5).  When inv_err is
  * non-NULL the GetProxy invariants of Sec. 5.1 / Algorithm 1 are measured and

@@ -1,6 +1,6 @@
 // Element arithmetic of the SpecInfer residual in the streaming kernel.
 //
-// The residual after n rejections at a node is (Eq. recur, Sec. 3)
+// The residual after n rejections at a node is (Eq. 2, Sec. 3)
 //   R_n = (R_{n-1} - q)_+ / S_n = (p - C_n q)_+ / N_n
 // for one scalar C_n: subtracting multiples of q and clipping at zero
 // compose.  In the kernel's unnormalised units (p~ = 2^(z_t c - M_t),

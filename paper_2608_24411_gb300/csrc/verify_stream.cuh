@@ -23,7 +23,7 @@
 // limit it.  A visit runs
 //   NORM   online (reference, sum) of 2^(z c) per thread, c = log2(e) / T,
 //          then one cluster exchange gives the global (M, S) of each row;
-//   REJ    once per rejected candidate (Algorithm 1, GetProxy / Eq. recur):
+//   REJ    once per rejected candidate (Algorithm 1, GetProxy / Eq. 2):
 //          recomputes p = 2^(z_t c - M_t) / S_t and q likewise from the raw
 //          logits (L2 hits), applies the residual maps of the earlier
 //          rejections in order, and sums the terms of the new map;
@@ -936,7 +936,7 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
   const int L = P.slice;
   const int lo = (int)rank * L;
   const int nloc = max(0, min(V, lo + L) - lo);
-  // SPEC: the SpecInfer instance (Eq. recur, evaluated as in specinfer.cuh);
+  // SPEC: the SpecInfer instance (Eq. 2, evaluated as in specinfer.cuh);
   // the others run ResiSpec (Algorithm 1)
   const int chain = SPEC ? kChainSpec : ((VAR && P.denom_update) ? kChainResiDenom : kChainResi);
   const bool drafting = VAR && P.draft_out != nullptr;
@@ -1300,7 +1300,7 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
       if (__fmul_rn(u, qx) < Rx) { accepted = cn; acc_tok = x; break; }
       rejects += 1;
       if constexpr (SPEC) {
-        // ---- SpecInfer rejection (Eq. recur): R <- (R - q)_+ / S, kept as
+        // ---- SpecInfer rejection (Eq. 2, Sec. 3): R <- (R - q)_+ / S, kept as
         // the threshold K of r~ = (p~ - K q~)_+ (specinfer.cuh).  The node's
         // first rejection takes S_t and S_d in double-float (one pass);
         // then K_1 = S_t / S_d, later K_{n+1} = K_n + T_n / S_d, and one pass

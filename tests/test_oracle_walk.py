@@ -1,6 +1,6 @@
 """The oracle's full verification walk pinned against the exact enumerator,
 the textbook exactness of multi-candidate speculative sampling (Sec. 3,
-Eq. recur), closed forms, independent recomputations with numpy/scipy and
+Eq. 2), closed forms, independent recomputations with numpy/scipy and
 the error contract."""
 import numpy as np
 import pytest

@@ -559,22 +559,23 @@ __device__ __forceinline__ void zero_rejected_vec(const StreamHead& S2, int nm, 
   }
 }
 
-// Final values (the distribution being sampled) of vector h of a thread's
-// chunk: p when no map is pending, else the residual, R = sig R~ (zero at
-// the rejected tokens).  base: its first token.
+// Final values (the distribution being sampled) of vector g of a ring
+// stage row (g = h THREADS + t is vector h of thread t's chunk): p when no
+// map is pending, else the residual, R = sig R~ (zero at the rejected
+// tokens).  base: its first token.
 template <int THREADS, bool BF16, bool SPEC>
 __device__ __forceinline__ void final_values(const StreamHead& S2, const VisitScalars& K,
                                              int chain, int nm, int base,
                                              const unsigned char* rt, const unsigned char* rd,
-                                             int h, float (&v)[BF16 ? 8 : 4]) {
+                                             int g, float (&v)[BF16 ? 8 : 4]) {
   constexpr int VEC = BF16 ? 8 : 4;
   constexpr int NP = VEC / 2;
   float z[VEC];
-  unpack_vec<BF16>(stage_vec(rt, h, THREADS), z);
+  unpack_vec<BF16>(reinterpret_cast<const uint4*>(rt)[g], z);
   if constexpr (SPEC) {
     if (nm > 0) {  // SpecInfer residual (p~ - K q~)_+ / T (specinfer.cuh)
       float zd[VEC];
-      unpack_vec<BF16>(stage_vec(rd, h, THREADS), zd);
+      unpack_vec<BF16>(reinterpret_cast<const uint4*>(rd)[g], zd);
 #pragma unroll
       for (int j = 0; j < VEC; ++j)
         v[j] = __fmul_rn(df_value(spec_residual(z[j], zd[j], K.sc, K.tab)), K.sig);
@@ -595,7 +596,7 @@ __device__ __forceinline__ void final_values(const StreamHead& S2, const VisitSc
     }
     return;
   }
-  unpack_vec<BF16>(stage_vec(rd, h, THREADS), z);
+  unpack_vec<BF16>(reinterpret_cast<const uint4*>(rd)[g], z);
   float2 q[NP];
 #pragma unroll
   for (int j = 0; j < NP; ++j)
@@ -631,15 +632,16 @@ __device__ __forceinline__ void final_values(const StreamHead& S2, const VisitSc
 // slice has no mass).
 constexpr int kMaxSearchChunks = 128;
 
+// Step 1 of a search: the slice's chunk totals ck[k] (fixed point), from
+// the records of the pass that defined the distribution, or from a pass.
 template <int THREADS, bool BF16, bool SPEC>
-__device__ int stream_search(Head& H, const StreamHead& S2, unsigned long long* ck,
-                             unsigned char* ring, const Src& s, const VisitScalars& K, int chain,
-                             int lo, unsigned long long tau, const ChunkRec& cr) {
+__device__ void search_totals(const StreamHead& S2, unsigned long long* ck, unsigned char* ring,
+                              const Src& s, const VisitScalars& K, int chain, int lo,
+                              const ChunkRec& cr) {
   using G = StreamGeom<THREADS, BF16>;
   constexpr int VEC = G::VEC;
   constexpr int NW = THREADS / 32;
-  static_assert(G::VPT * NW <= 32, "one scan lane per warp segment");
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
   const int nm = S2.nmaps;
   const int NK = (s.nloc + G::CE - 1) / G::CE;  // <= kMaxSearchChunks (slices <= 2^18)
   for (int k = threadIdx.x; k < NK; k += THREADS) ck[k] = 0ull;
@@ -666,7 +668,7 @@ __device__ int stream_search(Head& H, const StreamHead& S2, unsigned long long* 
       float v[VEC];
       final_values<THREADS, BF16, SPEC>(S2, K, chain, nm,
                                         lo + k * G::CE + (h * THREADS + (int)threadIdx.x) * VEC,
-                                        rt, rd, h, v);
+                                        rt, rd, h * THREADS + (int)threadIdx.x, v);
 #pragma unroll
       for (int j = 0; j < VEC / 2; ++j) acc2 = __fadd2_rn(acc2, make_float2(v[2 * j], v[2 * j + 1]));
     }
@@ -678,53 +680,57 @@ __device__ int stream_search(Head& H, const StreamHead& S2, unsigned long long* 
     return false;
   });
   __syncthreads();
-  if (warp == 0) {
-    // lanes hold chunks lane + 32 i; inclusive prefix over chunk order
-    unsigned long long run = 0;
-    int kfound = -1, klast = -1;
-    unsigned long long before = 0;
-    for (int base = 0; base < NK; base += 32) {
-      const int k = base + lane;
-      const unsigned long long m = k < NK ? ck[k] : 0ull;
-      unsigned long long incl = m;
+}
+
+// Step 2 (warp 0): the chunk holding tau in the inclusive prefix of ck, and
+// tau's remainder inside it; a threshold past the slice's total takes its
+// last chunk with mass (force).  Returns the chunk (-1: no mass).
+__device__ __forceinline__ int search_chunk_of(const unsigned long long* ck, int NK,
+                                               unsigned long long tau, bool& force,
+                                               unsigned long long& rem) {
+  const int lane = threadIdx.x & 31;
+  unsigned long long run = 0;
+  int kfound = -1, klast = -1;
+  unsigned long long before = 0;
+  for (int base = 0; base < NK; base += 32) {
+    const int k = base + lane;
+    const unsigned long long m = k < NK ? ck[k] : 0ull;
+    unsigned long long incl = m;
 #pragma unroll
-      for (int o = 1; o < 32; o <<= 1) {
-        const unsigned long long n = __shfl_up_sync(0xffffffffu, incl, o);
-        if (lane >= o) incl += n;
-      }
-      incl += run;
-      const unsigned cross = __ballot_sync(0xffffffffu, k < NK && incl > tau);
-      const unsigned pos = __ballot_sync(0xffffffffu, m > 0);
-      if (pos) klast = base + 31 - __clz(pos);
-      if (kfound < 0 && cross) {
-        const int l = __ffs(cross) - 1;
-        kfound = base + l;
-        before = __shfl_sync(0xffffffffu, incl - m, l);
-      }
-      run = __shfl_sync(0xffffffffu, incl, 31);
+    for (int o = 1; o < 32; o <<= 1) {
+      const unsigned long long n = __shfl_up_sync(0xffffffffu, incl, o);
+      if (lane >= o) incl += n;
     }
-    if (lane == 0) {
-      H.misc[0] = kfound >= 0 ? kfound : klast;
-      H.misc[3] = kfound < 0;  // threshold past the slice's total: last token with mass
-      H.fixd[0] = kfound >= 0 ? tau - before : 0ull;
-      H.misc[4] = -1;
-      H.misc[7] = -1;
+    incl += run;
+    const unsigned cross = __ballot_sync(0xffffffffu, k < NK && incl > tau);
+    const unsigned pos = __ballot_sync(0xffffffffu, m > 0);
+    if (pos) klast = base + 31 - __clz(pos);
+    if (kfound < 0 && cross) {
+      const int l = __ffs(cross) - 1;
+      kfound = base + l;
+      before = __shfl_sync(0xffffffffu, incl - m, l);
     }
+    run = __shfl_sync(0xffffffffu, incl, 31);
   }
-  __syncthreads();
-  const int ks = H.misc[0];
-  if (ks < 0) return -1;
-  const bool force = H.misc[3] != 0;
-  const unsigned long long t = H.fixd[0];
-  // the chosen chunk's values (this thread's vectors: held in the ring, or
-  // copied again into ring stage 0, which only this thread's copies write)
-  const unsigned char* stg = ring;
-  if (s.held) {
-    stg = held_stage<THREADS, BF16>(ring, s, ks);
-  } else {
-    copy_chunk<THREADS, BF16>(s, ks, ring, s.rows == 2);
-    cp_async_wait<0>();
-  }
+  force = kfound < 0;
+  rem = kfound >= 0 ? tau - before : 0ull;
+  return kfound >= 0 ? kfound : klast;
+}
+
+// Step 3: the token of chunk ks (this thread's vectors at stage stg) whose
+// exact prefix mass crosses t, or with force (or when no vector holds t) the
+// chunk's last token with mass.  Returns its offset in the slice.  H.misc[4]
+// and H.misc[7] hold -1 on entry (set before a barrier).
+template <int THREADS, bool BF16, bool SPEC>
+__device__ int search_in_chunk(Head& H, const StreamHead& S2, const unsigned char* stg,
+                               const Src& s, const VisitScalars& K, int chain, int lo, int ks,
+                               bool force, unsigned long long t) {
+  using G = StreamGeom<THREADS, BF16>;
+  constexpr int VEC = G::VEC;
+  constexpr int NW = THREADS / 32;
+  static_assert(G::VPT * NW <= 32, "one scan lane per warp segment");
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int nm = S2.nmaps;
   float v[G::VPT][VEC];
   unsigned long long mv[G::VPT], ex[G::VPT];
   int lastpos = -1;
@@ -732,7 +738,7 @@ __device__ int stream_search(Head& H, const StreamHead& S2, unsigned long long* 
   for (int h = 0; h < G::VPT; ++h) {
     const int g = h * THREADS + (int)threadIdx.x;
     final_values<THREADS, BF16, SPEC>(S2, K, chain, nm, lo + ks * G::CE + g * VEC, stg,
-                                      stg + G::RB, h, v[h]);
+                                      stg + G::RB, g, v[h]);
     mv[h] = 0;
 #pragma unroll
     for (int j = 0; j < VEC; ++j) {
@@ -786,6 +792,118 @@ __device__ int stream_search(Head& H, const StreamHead& S2, unsigned long long* 
   return pick < 0 ? -1 : ks * G::CE + pick;
 }
 
+
+// Step 3 for one warp, for a row's own distribution (no residual map: the
+// drafting step's draws from q): the token search_in_chunk finds, found by
+// one warp alone over the whole chunk (every vector landed and visible to
+// the warp).  The values are final_values' without a map, bit for bit:
+// 2^(z c - M) / S.  The warp walks the chunk's vectors in token order, 32 at a
+// time (lane l takes vector 32 i + l: conflict-free loads), with an exact
+// 64-bit scan of their fixed-point totals on top of the groups before; the
+// lane whose vector holds t walks its values.  Integer sums are exact, so
+// the crossing token is the one a block-wide scan finds.
+template <int THREADS, bool BF16>
+__device__ int warp_draw_in_chunk(const unsigned char* stg, int nloc, float c, float M, float inv,
+                                  int ks, bool force, unsigned long long t) {
+  using G = StreamGeom<THREADS, BF16>;
+  constexpr int VEC = G::VEC;
+  constexpr int PV = G::VPT * THREADS / 32;  // vectors per lane
+  const int lane = threadIdx.x & 31;
+  auto values = [&](int g, float (&v)[VEC]) {
+    float z[VEC];
+    unpack_vec<BF16>(reinterpret_cast<const uint4*>(stg)[g], z);
+#pragma unroll
+    for (int j = 0; j < VEC; ++j) v[j] = __fmul_rn(ex2(__fmaf_rn(z[j], c, -M)), inv);
+  };
+  int pick = -1;
+  if (!force) {
+    unsigned long long run = 0;  // mass of the groups before
+#pragma unroll 1
+    for (int i = 0; i < PV; ++i) {
+      const int g = i * 32 + lane;
+      float v[VEC];
+      values(g, v);
+      unsigned long long m = 0;
+#pragma unroll
+      for (int j = 0; j < VEC; ++j) m += to_fix(v[j]);
+      unsigned long long incl = m;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const unsigned long long n = __shfl_up_sync(0xffffffffu, incl, o);
+        if (lane >= o) incl += n;
+      }
+      incl += run;
+      const unsigned long long a0 = incl - m;
+      const unsigned hit = __ballot_sync(0xffffffffu, m > 0 && a0 <= t && t < incl);
+      if (hit) {
+        const int l = __ffs(hit) - 1;
+        if (lane == l) {
+          unsigned long long a = a0;
+          pick = g * VEC + VEC - 1;
+#pragma unroll
+          for (int j = 0; j < VEC; ++j) {
+            a += to_fix(v[j]);
+            if (a > t) { pick = g * VEC + j; break; }
+          }
+        }
+        pick = __shfl_sync(0xffffffffu, pick, l);
+        break;
+      }
+      run = __shfl_sync(0xffffffffu, incl, 31);
+    }
+  }
+  if (pick < 0) {  // forced, or t past the chunk's total: its last token with mass
+    int last = -1;
+#pragma unroll 1
+    for (int i = 0; i < PV; ++i) {
+      const int g = i * 32 + lane;
+      float v[VEC];
+      values(g, v);
+#pragma unroll
+      for (int j = 0; j < VEC; ++j)
+        if (v[j] > 0.f && ks * G::CE + g * VEC + j < nloc) last = g * VEC + j;
+    }
+    pick = __reduce_max_sync(0xffffffffu, last);
+  }
+  return pick < 0 ? -1 : ks * G::CE + pick;
+}
+
+template <int THREADS, bool BF16, bool SPEC>
+__device__ int stream_search(Head& H, const StreamHead& S2, unsigned long long* ck,
+                             unsigned char* ring, const Src& s, const VisitScalars& K, int chain,
+                             int lo, unsigned long long tau, const ChunkRec& cr) {
+  using G = StreamGeom<THREADS, BF16>;
+  const int NK = (s.nloc + G::CE - 1) / G::CE;
+  search_totals<THREADS, BF16, SPEC>(S2, ck, ring, s, K, chain, lo, cr);
+  if ((threadIdx.x >> 5) == 0) {
+    bool force;
+    unsigned long long rem;
+    const int k = search_chunk_of(ck, NK, tau, force, rem);
+    if (threadIdx.x == 0) {
+      H.misc[0] = k;
+      H.misc[3] = force;
+      H.fixd[0] = rem;
+      H.misc[4] = -1;
+      H.misc[7] = -1;
+    }
+  }
+  __syncthreads();
+  const int ks = H.misc[0];
+  if (ks < 0) return -1;
+  const bool force = H.misc[3] != 0;
+  const unsigned long long t = H.fixd[0];
+  // the chosen chunk's values (this thread's vectors: held in the ring, or
+  // copied again into ring stage 0, which only this thread's copies write)
+  const unsigned char* stg = ring;
+  if (s.held) {
+    stg = held_stage<THREADS, BF16>(ring, s, ks);
+  } else {
+    copy_chunk<THREADS, BF16>(s, ks, ring, s.rows == 2);
+    cp_async_wait<0>();
+  }
+  return search_in_chunk<THREADS, BF16, SPEC>(H, S2, stg, s, K, chain, lo, ks, force, t);
+}
+
 // Final draw of a visit: every CTA picks the CTA whose mass range holds
 // u * total (as the resident kernel's sampler); that CTA searches its slice.
 template <int THREADS, bool BF16, bool SPEC>
@@ -811,7 +929,8 @@ __device__ bool stream_sample(Head& H, StreamHead& S2, unsigned char* ring, cons
       for (int h = 0; h < G::VPT; ++h) {
         float v[VEC];
         const int e0 = k * G::CE + (h * THREADS + (int)threadIdx.x) * VEC;  // offset in the slice
-        final_values<THREADS, BF16, SPEC>(S2, K, chain, nm, lo + e0, rt, rd, h, v);
+        final_values<THREADS, BF16, SPEC>(S2, K, chain, nm, lo + e0, rt, rd,
+                                          h * THREADS + (int)threadIdx.x, v);
 #pragma unroll
         for (int j = 0; j < VEC; ++j) {
           sum += v[j];
@@ -1002,30 +1121,36 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
                   "draft thresholds fit the logit slots");
     unsigned long long* tau = reinterpret_cast<unsigned long long*>(S2.kzt);
     int* owner = S2.rej;
+    // per-CTA draft masses (fixed point), in the sampler's segment slots
+    static_assert(sizeof(Head::seg) >= kMaxCluster * sizeof(unsigned long long),
+                  "per-CTA masses fit the segment slots");
+    unsigned long long* cmass = H.seg;
+    if (tid < (int)C) cmass[tid] = to_fix(__fmul_rn(H.part[tid][3], ref_scale(H.part[tid][2], K.Md, K.invSd)));
     if (tid == 0) {
-      unsigned long long total = 0;
-      for (uint32_t r = 0; r < C; ++r)
-        total += to_fix(__fmul_rn(H.part[r][3], ref_scale(H.part[r][2], K.Md, K.invSd)));
       int i = 0;
-      for (int cn = c1d; cn >= 0 && i < kMaxKids; cn = next_sib[cn], ++i) {
-        const float u = uniform_draw(P.seed, (uint32_t)b, (uint32_t)(cn + 1), 2);
-        const unsigned long long kk = (unsigned long long)(u * 16777216.f);
-        const unsigned long long t = (__umul64hi(kk, total) << 40) | ((kk * total) >> 24);
-        unsigned long long a = 0;
-        int r_own = total > 0 ? (int)C - 1 : -1;
-        for (uint32_t r = 0; r < C && total > 0; ++r) {
-          const unsigned long long m =
-              to_fix(__fmul_rn(H.part[r][3], ref_scale(H.part[r][2], K.Md, K.invSd)));
-          if (a + m > t) { r_own = (int)r; break; }
-          a += m;
-        }
-        tau[i] = t > a ? t - a : 0ull;
-        owner[i] = r_own;
-      }
+      for (int cn = c1d; cn >= 0 && i < kMaxKids; cn = next_sib[cn]) ++i;
       H.misc[6] = i;
     }
     __syncthreads();
     const int nk = H.misc[6];
+    if (tid < nk) {  // child tid's draw: its CTA and the threshold inside it
+      int cn = c1d;
+      for (int k = 0; k < tid; ++k) cn = next_sib[cn];
+      unsigned long long total = 0;
+      for (uint32_t r = 0; r < C; ++r) total += cmass[r];
+      const unsigned long long kk = tau[tid];  // the draw's 24 bits (normaliser pass)
+      const unsigned long long t = (__umul64hi(kk, total) << 40) | ((kk * total) >> 24);
+      unsigned long long a = 0;
+      int r_own = total > 0 ? (int)C - 1 : -1;
+      for (uint32_t r = 0; r < C && total > 0; ++r) {
+        const unsigned long long m = cmass[r];
+        if (a + m > t) { r_own = (int)r; break; }
+        a += m;
+      }
+      tau[tid] = t > a ? t - a : 0ull;
+      owner[tid] = r_own;
+    }
+    __syncthreads();
     // q values come out of the sampler's search with the draft row in
     // place of the target row and the draft's scalars
     Src sq;
@@ -1038,16 +1163,74 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
     VisitScalars Kq = K;
     Kq.Mt = K.Md;
     Kq.invSt = K.invSd;
-    // chunk totals of the searches: the residual maps' slots (no map exists
-    // before the node's accept tests)
+    // The children this CTA owns: the draft row's chunk totals once (from
+    // the normaliser's records, or one pass), each child's chunk and the
+    // remainder of its threshold (one warp per child), then the owned
+    // children's chunks copied together, one single-row ring stage each, and
+    // one in-chunk search per child, one warp per child (the steps of
+    // stream_search, shared across the children).  Chunk totals in the
+    // residual maps' slots (no map exists before the node's accept tests),
+    // each child's chunk in the rejected-child slots.
     static_assert(sizeof(StreamHead::map) >= kMaxSearchChunks * sizeof(unsigned long long),
                   "search chunk totals fit the map slots");
-    for (int i = 0, cn = c1d; i < nk; ++i, cn = next_sib[cn]) {
-      if (owner[i] != (int)rank) continue;
-      const int pick = stream_search<THREADS, BF16, SPEC>(
-          H, S2, reinterpret_cast<unsigned long long*>(S2.map), ring, sq, Kq, chain, lo, tau[i],
-          ChunkRec{rec_draft ? 1 : 0, K.Md, K.invSd});
-      if (tid == 0) P.draft_out[(size_t)b * N + cn] = lo + max(pick, 0);
+    unsigned long long* ck = reinterpret_cast<unsigned long long*>(S2.map);
+    int16_t* kchunk = S2.rejk;  // -2: not owned; -1: no mass; else chunk | force << 13
+    bool mine = false;
+    for (int i = 0; i < nk; ++i) mine |= owner[i] == (int)rank;
+    if (mine) {
+      search_totals<THREADS, BF16, SPEC>(S2, ck, ring, sq, Kq, chain, lo,
+                                         ChunkRec{rec_draft ? 1 : 0, K.Md, K.invSd});
+      const int NK = (nloc + G::CE - 1) / G::CE;
+      for (int i = warp; i < nk; i += NW) {
+        int16_t code = -2;
+        if (owner[i] == (int)rank) {
+          bool force;
+          unsigned long long rem;
+          const int kc = search_chunk_of(ck, NK, tau[i], force, rem);
+          if (lane == 0) tau[i] = rem;
+          code = (int16_t)(kc < 0 ? -1 : kc | (force ? 1 << 13 : 0));
+        }
+        if (lane == 0) kchunk[i] = code;
+      }
+      __syncthreads();
+      // batches of up to min(ring stages, warps) children with mass
+      const int width = min(ring_depth<THREADS, BF16>(false), NW);
+      for (int i0 = 0, cn0 = c1d; i0 < nk;) {
+        int i1 = i0, n = 0;
+        for (; i1 < nk && n < width; ++i1)
+          if (kchunk[i1] >= 0)
+            copy_chunk<THREADS, BF16>(sq, kchunk[i1] & 0x1fff, ring + (n++) * G::RB, false);
+        cp_async_wait<0>();
+        __syncthreads();  // every thread's vectors of the batch's chunks have landed
+        // up to two children: each searched by the whole CTA (a block-wide
+        // scan); more: one warp per child, all at once
+        const bool by_warp = n > 2;
+        for (int i = i0, j = 0, cn = cn0; i < i1; ++i, cn = next_sib[cn]) {
+          if (kchunk[i] == -2) continue;
+          const int kc = kchunk[i] & 0x1fff;
+          const bool force = (kchunk[i] >> 13) != 0;
+          if (kchunk[i] < 0) {
+            if (tid == 0) P.draft_out[(size_t)b * N + cn] = lo;
+          } else if (by_warp) {
+            if (j++ != warp) continue;
+            const int pick = warp_draw_in_chunk<THREADS, BF16>(ring + warp * G::RB, nloc, K.c,
+                                                               K.Md, K.invSd, kc, force, tau[i]);
+            if (lane == 0) P.draft_out[(size_t)b * N + cn] = lo + max(pick, 0);
+          } else {
+            if (tid == 0) {
+              H.misc[4] = -1;
+              H.misc[7] = -1;
+            }
+            __syncthreads();
+            const int pick = search_in_chunk<THREADS, BF16, SPEC>(
+                H, S2, ring + (j++) * G::RB, sq, Kq, chain, lo, kc, force, tau[i]);
+            if (tid == 0) P.draft_out[(size_t)b * N + cn] = lo + max(pick, 0);
+          }
+        }
+        __syncthreads();  // the stages are reused by the next batch
+        for (int i = i0; i < i1; ++i) cn0 = next_sib[cn0];
+        i0 = i1;
+      }
     }
     cluster_sync();  // every drawn token written (release / acquire at cluster scope)
     // the children's tokens and their raw logits
@@ -1137,7 +1320,16 @@ __global__ void __launch_bounds__(THREADS, THREADS >= 512 ? 2 : 4)
           const int j = THREADS - 1 - tid;  // kMaxKids < THREADS - kMaxKids
           if (j < kMaxKids && need_draft && !err) {
             const int cn = nth_child(j);
-            if (cn >= 0) S2.kua[j] = uniform_draw(P.seed, (uint32_t)b, (uint32_t)(cn + 1), 0);
+            if (cn >= 0) {
+              // U(seed, b, cn + 1, .): word 0 the accept draw; word 2 the
+              // drafting draw, kept as its 24-bit integer in the child's
+              // threshold slot (draft_children)
+              const U64x4 r = philox4x64_10((uint64_t)(cn + 1), (uint64_t)b, 0, 0, P.seed, 0);
+              S2.kua[j] = u24(r.w[0]);
+              if (drafting)
+                reinterpret_cast<unsigned long long*>(S2.kzt)[j] =
+                    (unsigned long long)(u24(r.w[2]) * 16777216.f);
+            }
           } else if (j == kMaxKids) {
             S2.ufin = uniform_draw(P.seed, (uint32_t)b, (uint32_t)row, 1);
           }

@@ -1,5 +1,6 @@
 """GPU parity: the CUDA verification path against the fp64 oracle on the
 same seeded inputs, through the C ABI (see tests/parity.py for the rule)."""
+import dataclasses
 import functools
 
 import numpy as np
@@ -764,6 +765,21 @@ def test_parity_drafting(wl, mode):
     inp = _inputs(w.name, 17, 256 if wl != "chain8x4-v128256-b16" else 16)
     gd, _ = _check_drafting(inp, mode, seed=170 + mode)
     assert (gd[:, :1] >= 0).all()   # the root's first child is always drawn
+
+
+@pytest.mark.parametrize("mode", MODES)
+@pytest.mark.parametrize("cluster,threads", [(1, 256), (1, 512), (2, 256), (2, 512)])
+def test_parity_drafting_wide_fanout(cluster, threads, mode):
+    """Drafting 16 children per node in one or two CTAs: a CTA draws more
+    children than it has warps or single-row ring stages, so its draws run
+    in batches (one warp per child); tokens, accept lengths and drafted
+    candidates against the oracle's drafting walk."""
+    w = dataclasses.replace(W.WORKLOADS["single-k16-v256000-b32"], vocab=20000,
+                            name="single-k16-v20000")
+    inp = W.make_inputs_np(w, seed=23, batch=64)
+    gd, _ = _check_drafting(inp, mode, seed=230 + cluster, cluster_size=cluster,
+                            block_threads=threads)
+    assert (gd >= 0).all()   # a single position: every child is drawn
 
 
 def test_gpu_drafted_candidates_follow_q():

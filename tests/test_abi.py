@@ -309,3 +309,11 @@ int main(int argc, char** argv) {
     assert clean.sum() >= 0.99 * B
     np.testing.assert_array_equal(alen[clean], o["accept_len"][clean])
     np.testing.assert_array_equal(toks[clean], o["tokens"][clean])
+
+
+@pytest.mark.gpu
+def test_graft_entry_smoke():
+    """The round-end smoke entry point: small calls on cuda:0 in every mode
+    and kernel it supports, checked against the oracle."""
+    import __graft_entry__
+    __graft_entry__.smoke()

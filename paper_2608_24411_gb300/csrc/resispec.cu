@@ -230,9 +230,11 @@ int plan_resident(const resispec_dims& d, int cs, int dev, int sms, Plan* p) {
 //  - 256-thread CTAs (three per SM, half the ring each) beat 512-thread ones
 //    on trees with about two children per node (N^(1/D) <= 2.5: binary
 //    depth-5 trees 102.7 against 107.9 us at B = 64, single position k = 2
-//    at B = 128 85.8 against 104.4 us), where a sequence spends its time in
-//    normaliser passes rather than in rejection passes; wider trees and
-//    batches that fit 16-CTA clusters of 512 threads keep 512.
+//    at B = 128 85.8 against 104.4 us) and on shallow trees of at most 4
+//    nodes (single position k = 4 at B = 128: 92.7 against 107.5 us), where
+//    a sequence spends its time in normaliser passes rather than in
+//    rejection passes; wider trees and batches that fit 16-CTA clusters of
+//    512 threads keep 512.
 //  - Trees deeper than 2 levels take the largest C that runs the batch in
 //    one wave; when that leaves more than 128 elements per thread and row in
 //    a CTA's slice, the largest C within two waves (tree488 at B = 128:
@@ -257,7 +259,8 @@ int plan_stream(const resispec_dims& d, int cs, bool auto_threads, int dev, int 
     const double g = d.max_depth > 0
                          ? std::pow((double)std::max(d.num_nodes, 1), 1.0 / d.max_depth)
                          : 1e30;
-    p->threads = (g <= 2.5 && B > active_for(512, 16)) ? 256 : 512;
+    const bool narrow = g <= 2.5 || (d.max_depth <= 2 && d.num_nodes <= 4);
+    p->threads = (narrow && B > active_for(512, 16)) ? 256 : 512;
   }
   const int T = p->threads;
   p->smem = stream_smem_for(T, bf16, p->npad);

@@ -87,6 +87,8 @@ def test_plan_without_device(lib):
     # 512-thread CTAs for wider trees and for batches that fit clusters of 16
     assert rs.plan(1, 62, 151936, 5, "f32")["block_threads"] == 512
     assert rs.plan(128, 16, 256000, 1, "bf16")["block_threads"] == 512
+    p4 = rs.plan(128, 4, 256000, 1, "bf16")   # single position, k = 4
+    assert (p4["cluster_size"], p4["block_threads"]) == (6, 256)
     # shallow trees accept more waves: 128 single-position sequences in
     # clusters of 8; deep trees of 32 sequences in clusters of 8 (one wave);
     # of 128 sequences, whose one-wave slices would be too long, in clusters

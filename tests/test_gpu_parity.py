@@ -67,6 +67,25 @@ def _check(inp, mode, seed, **kw):
     return g, o
 
 
+@pytest.mark.parametrize("mode", MODES)
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+@pytest.mark.parametrize("cluster,threads", [(0, 0), (1, 256), (1, 512), (16, 256)])
+def test_parity_max_vocab(cluster, threads, dtype, mode):
+    """The largest vocabulary (V = 262144): the automatic launch shape, one
+    CTA per sequence (a slice of 128 chunks at 256 threads, the search's
+    chunk-total limit, without chunk records), and clusters of 16; a chain
+    of depth 4 with 3 candidates per level, zipf logits."""
+    _check(_max_vocab_inputs(dtype), mode, seed=410 + cluster, cluster_size=cluster,
+           block_threads=threads, kernel="stream")
+
+
+@functools.lru_cache(maxsize=2)
+def _max_vocab_inputs(dtype):
+    w = dataclasses.replace(W.WORKLOADS["tiny-chain-v64"], vocab=rs.MAX_VOCAB, dtype=dtype,
+                            gen="zipf", scale=3.0, slope=1.1, name="tiny-chain-vmax")
+    return W.make_inputs_np(w, seed=41, batch=8)
+
+
 def test_device_philox_matches_numpy():
     import torch
     from tests.test_oracle_pins import _np_philox_block

@@ -17,7 +17,8 @@
 // next S - 1 chunks into its own slots of a shared-memory ring with
 // cp.async (16-byte asynchronous copies) and reads back only what it copied
 // itself, so no barrier is needed between chunks and the bytes in flight
-// cost no registers.  With 1024 threads per SM this saturates HBM, and one
+// cost no registers.  With two 512-thread or three 256-thread CTAs per SM
+// this saturates HBM, and one
 // CTA alone streams about twice as fast as through a bulk-copy (TMA) ring
 // of the same size, whose single issuing thread and per-chunk barrier
 // limit it.  A visit runs
